@@ -1,0 +1,331 @@
+// Device-side building blocks shared by the libsparoa kernels (sm_103a).
+//
+//  * PTX wrappers: mbarrier, TMA (cp.async.bulk.tensor), cp.async, tcgen05
+//    (alloc / mma / commit / ld), proxy fences, named barriers.
+//  * Bounded waits: every spin on an mbarrier gives up after kWaitLimitNs,
+//    records an error bit in the context's device flag and lets the CTA
+//    unwind, so a broken pipeline never hangs the GPU.
+//  * Occupancy emission: every kernel that writes a bf16 activation builds, per
+//    128-row x 64-column tile, a shared-memory bitmap (one 64-bit word per row,
+//    bit c = element (r, c) is non-zero) and flushes it into the Eq. 1 count
+//    and occupancy bitmaps of the output (Sec. 3.1 sparsity).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace sparoa {
+
+constexpr uint64_t kWaitLimitNs = 1000ull * 1000ull * 1000ull;  // 1 s
+
+enum ErrBits : uint32_t {
+  kErrTimeoutFull = 1u,
+  kErrTimeoutEmpty = 2u,
+  kErrTimeoutAcc = 4u,
+};
+
+// Occupancy outputs of a [R, C] bf16 tensor (mirrors sparoa_occupancy).
+struct OccDev {
+  unsigned long long* nnz;
+  uint32_t* col_nnz;
+  uint32_t* tile_nnz;
+  unsigned long long* row_bm;
+  uint32_t* blk_mask;
+  int64_t R;
+  int32_t C;
+  int32_t W64;  // words per row of row_bm
+  int32_t C32;  // words per 128-row block of blk_mask
+};
+
+// Inputs of the on-device dispatch decision.
+struct DispatchDev {
+  const unsigned long long* in_nnz;  // Eq. 1 count of the operator's input
+  unsigned long long numel;
+  double s_thr;
+  int32_t fpb_ok;     // host: intensity >= c_thr
+  int32_t force;      // 0 rule, 1 dense, 2 zero-skip
+  int32_t* path_out;  // nullable; written once by CTA (0,0,0) thread 0
+};
+
+// The threshold rule, in IEEE double (path 1 = dense, 2 = zero-skip).
+__device__ __forceinline__ int decide_path(const DispatchDev& d) {
+  if (d.force == 1) return 1;
+  if (d.force == 2) return 2;
+  const unsigned long long nnz = *d.in_nnz;
+  const double zeros = (double)(d.numel - nnz);
+  const double bound = __dmul_rn(d.s_thr, (double)d.numel);
+  if (zeros >= bound) return 2;
+  return d.fpb_ok ? 1 : 2;
+}
+
+__device__ __forceinline__ void record_path(const DispatchDev& d, int path) {
+  if (d.path_out && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && threadIdx.x == 0)
+    *d.path_out = path;
+}
+
+// bf16 zero test on the bit pattern: +0 and -0 are zero, everything else not.
+__device__ __forceinline__ bool bf16_nz(uint16_t b) { return (b & 0x7FFFu) != 0; }
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// ---------------------------------------------------------------------------
+// mbarrier
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Wait for the phase with the given parity to complete.  Gives up after
+// kWaitLimitNs, or as soon as another role of the CTA raised *abort; then it
+// records `bit` in *err, raises *abort and returns false.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t* err,
+                                          volatile int* abort, uint32_t bit) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort) return false;
+    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      atomicOr(err, bit);
+      *abort = 1;
+      return false;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// TMA and cp.async
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, uint32_t bar, int x,
+                                            int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void prefetch_tmap(const void* tmap) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");
+}
+
+// 16-byte async copy global -> shared; src_bytes 0 writes 16 zero bytes.
+__device__ __forceinline__ void cp_async_16(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+               "r"(src_bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Make generic-proxy writes to shared memory visible to the async proxy
+// (tensor cores / TMA).
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Named barrier over `count` threads (whole warps).
+__device__ __forceinline__ void named_bar_sync(int id, int count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
+// OR of `pred` over the `count` threads of named barrier `id`.
+__device__ __forceinline__ bool named_bar_or(int id, int count, bool pred) {
+  uint32_t out;
+  asm volatile(
+      "{\n\t.reg .pred pi, po;\n\t"
+      "setp.ne.u32 pi, %1, 0;\n\t"
+      "bar.red.or.pred po, %2, %3, pi;\n\t"
+      "selp.u32 %0, 1, 0, po;\n\t}"
+      : "=r"(out)
+      : "r"((uint32_t)pred), "r"(id), "r"(count)
+      : "memory");
+  return out != 0;
+}
+
+// ---------------------------------------------------------------------------
+// tcgen05 (5th-generation tensor cores, accumulators in tensor memory)
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, kind::f16 (bf16 inputs, fp32 accumulate).
+__device__ __forceinline__ void tc_mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                            uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive once on `bar` when every tcgen05.mma issued so far by this thread is done.
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+
+// Load 16 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32"
+      " {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor for a K-major operand tile written with the
+// 64-byte swizzle: rows of 32 bf16 (64 B), 8-row core-matrix groups 512 B apart.
+__device__ __forceinline__ uint64_t smem_desc_sw64(uint32_t addr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((addr >> 4) & 0x3FFF);        // start address
+  d |= (uint64_t)(16 >> 4) << 16;                // leading byte offset (unused here)
+  d |= (uint64_t)(512 >> 4) << 32;               // stride byte offset: 8 rows * 64 B
+  d |= (uint64_t)1 << 46;                        // descriptor version (sm_100 family)
+  d |= (uint64_t)4 << 61;                        // layout: 64-byte swizzle
+  return d;
+}
+
+// Instruction descriptor: kind::f16, A = B = bf16, D = fp32, both K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
+  return (1u << 4)                         // D format f32
+         | (1u << 7)                       // A format bf16
+         | (1u << 10)                      // B format bf16
+         | ((uint32_t)(N >> 3) << 17)      // N / 8
+         | ((uint32_t)(M >> 4) << 24);     // M / 16
+}
+
+// Byte offset of 16-byte chunk j (0..3) of row r in a 64-byte-swizzled tile
+// (the layout TMA writes with CU_TENSOR_MAP_SWIZZLE_64B): address bits [4,6)
+// are XORed with bits [7,9).
+__device__ __forceinline__ uint32_t sw64_offset(int r, int j) {
+  return (uint32_t)(r * 64 + ((j ^ ((r >> 1) & 3)) << 4));
+}
+
+// ---------------------------------------------------------------------------
+// Epilogue math
+// ---------------------------------------------------------------------------
+struct EpiDev {
+  const float* bias;   // [C]
+  const float* bn;     // [4][C]
+  float eps;
+  int32_t act;
+  const __nv_bfloat16* residual;  // same layout as the output
+};
+
+// Per-channel affine form of bias + batch norm: v * scale + shift.
+__device__ __forceinline__ void epi_affine(const EpiDev& e, int C, int c, float& scale,
+                                           float& shift) {
+  const float b = e.bias ? e.bias[c] : 0.f;
+  if (e.bn) {
+    const float g = e.bn[c], beta = e.bn[C + c], mean = e.bn[2 * C + c], var = e.bn[3 * C + c];
+    scale = g * rsqrtf(var + e.eps);
+    shift = (b - mean) * scale + beta;
+  } else {
+    scale = 1.f;
+    shift = b;
+  }
+}
+
+__device__ __forceinline__ float epi_act(float v, int act) {
+  if (act == 1) return v > 0.f ? v : 0.f;
+  if (act == 2) return v > 0.f ? (v < 6.f ? v : 6.f) : 0.f;
+  return v;
+}
+
+// ---------------------------------------------------------------------------
+// Occupancy flush of one 128-row x 64-column tile
+// ---------------------------------------------------------------------------
+// nzrow[r] bit c: element (row0 + r, col0 + c) is non-zero (zero outside the
+// tensor).  Called by `nthreads` threads (a multiple of 32, >= 64) with local
+// index `tid`; row0 must be a multiple of 128 and col0 a multiple of 64.
+__device__ __forceinline__ void flush_tile(const uint64_t* nzrow, int64_t row0, int col0,
+                                           const OccDev& o, int tid, int nthreads) {
+  const int t = col0 >> 6;
+  for (int r = tid; r < 128; r += nthreads) {
+    if (nzrow[r] != 0ull && row0 + r < o.R)
+      atomicOr(&o.row_bm[(row0 + r) * o.W64 + (t >> 6)], 1ull << (t & 63));
+  }
+  if (tid < 64) {
+    uint32_t cnt = 0;
+#pragma unroll 8
+    for (int r = 0; r < 128; ++r) cnt += (uint32_t)((nzrow[r] >> tid) & 1ull);
+    const int c = col0 + tid;
+    if (cnt && c < o.C) atomicAdd(&o.col_nnz[c], cnt);
+    const uint32_t word = __ballot_sync(0xffffffffu, cnt != 0);
+    uint32_t sum = cnt;
+#pragma unroll
+    for (int s = 16; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
+    if ((tid & 31) == 0) {
+      const int w = (col0 >> 5) + (tid >> 5);
+      if (word && w < o.C32) atomicOr(&o.blk_mask[(row0 >> 7) * o.C32 + w], word);
+      if (sum) {
+        atomicAdd(&o.tile_nnz[t], sum);
+        atomicAdd(o.nnz, (unsigned long long)sum);
+      }
+    }
+  }
+}
+
+}  // namespace sparoa

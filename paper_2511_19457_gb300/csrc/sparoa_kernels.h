@@ -1,0 +1,96 @@
+// Host-side launch interface of the libsparoa kernels (internal to the library).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "sparoa_dev.cuh"
+
+namespace sparoa {
+
+// ----------------------------------------------------------------------------
+// Implicit-GEMM tensor-core kernel (dense path and zero-skip path)
+// ----------------------------------------------------------------------------
+struct IgemmArgs {
+  // Output y[M, N] (conv: M = images * Ho * Wo output pixels, N = C_out).
+  int M = 0, N = 0;
+  // conv = 0: A = x[M, K] row-major, loaded by TMA.  K = Ktot, K % 8 == 0.
+  // conv = 1: A gathered from NHWC x (implicit GEMM over (tap, channel)).
+  int conv = 0;
+  const __nv_bfloat16* x = nullptr;
+  int H = 1, W = 1, Cp = 0;          // conv input geometry; Cp = channel pitch (% 8 == 0)
+  int Ho = 1, Wo = 1, kh = 1, kw = 1, stride = 1, pad = 0;
+  int Ktot = 0;                      // GEMM K, or kh*kw*Cp
+  const __nv_bfloat16* w = nullptr;  // [N, Ktot] K-major
+  EpiDev ep{};
+  void* y = nullptr;
+  int y_f32 = 0;
+  DispatchDev disp{};
+  int dense_only = 0;                // 1: exit when the rule picks zero-skip
+  // occupancy of the input (zero-skip path)
+  const uint32_t* in_blk = nullptr;            // GEMM: blk_mask of x
+  int in_C32 = 0;
+  const unsigned long long* in_rowbm = nullptr;  // conv: row_bm of x
+  int in_W64 = 0;
+  // occupancy of the output
+  OccDev out_occ{};
+  int emit = 0;
+  uint32_t* err = nullptr;
+};
+
+// Picks the N tile, encodes the tensor maps and launches.
+cudaError_t launch_igemm(const IgemmArgs& a, cudaStream_t s);
+
+// ----------------------------------------------------------------------------
+// Column-compacting zero-skip FC for few rows (M <= 128 per row block)
+// ----------------------------------------------------------------------------
+struct FcSkipArgs {
+  const __nv_bfloat16* x = nullptr;   // [M, K]
+  const __nv_bfloat16* w_kn = nullptr;  // [K, N]
+  int M = 0, K = 0, N = 0;
+  const uint32_t* in_blk = nullptr;   // blk_mask of x, [ceil(M/128)][ceil(K/32)]
+  int in_C32 = 0;
+  EpiDev ep{};
+  void* y = nullptr;
+  int y_f32 = 0;
+  DispatchDev disp{};
+  OccDev out_occ{};
+  int emit = 0;
+};
+cudaError_t launch_fcskip(const FcSkipArgs& a, cudaStream_t s);
+
+// ----------------------------------------------------------------------------
+// Memory-bound kernels (128-row x 64-channel tiles, occupancy fused)
+// ----------------------------------------------------------------------------
+// Eq. 1 statistics and bitmaps of x viewed as [R, C].
+cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev& o, cudaStream_t s);
+
+// Copy [P, C] to [P, Cp] with zero channels C..Cp-1.
+cudaError_t launch_pad_channels(const __nv_bfloat16* x, int64_t P, int C, int Cp,
+                                __nv_bfloat16* y, cudaStream_t s);
+
+struct DwArgs {
+  const __nv_bfloat16* x = nullptr;  // [N, H, W, C]
+  const __nv_bfloat16* w = nullptr;  // [C, kh, kw]
+  int N = 0, H = 0, W = 0, C = 0, kh = 3, kw = 3, stride = 1, pad = 1, Ho = 0, Wo = 0;
+  EpiDev ep{};
+  __nv_bfloat16* y = nullptr;
+  OccDev out_occ{};
+  int emit = 0;
+  int32_t* path_out = nullptr;
+};
+cudaError_t launch_dwconv(const DwArgs& a, cudaStream_t s);
+
+cudaError_t launch_maxpool(const __nv_bfloat16* x, int N, int H, int W, int C, int k, int stride,
+                           int pad, int Ho, int Wo, __nv_bfloat16* y, const OccDev& o, int emit,
+                           cudaStream_t s);
+
+cudaError_t launch_avgpool(const __nv_bfloat16* x, int N, int HW, int C, __nv_bfloat16* y,
+                           const OccDev& o, int emit, cudaStream_t s);
+
+cudaError_t launch_bn_act(const __nv_bfloat16* x, int64_t R, int C, const EpiDev& ep,
+                          __nv_bfloat16* y, const OccDev& o, int emit, cudaStream_t s);
+
+}  // namespace sparoa
