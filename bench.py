@@ -1,0 +1,498 @@
+#!/usr/bin/env python
+"""Benchmark of the sparsity/intensity-dispatched operator path on GB300.
+
+Default workload (one step = one pass of the per-operator hot path over one
+batch): the 3x3 convolution NHWC bf16 [8, 56, 56, 64] -> 64 channels, stride 1,
+pad 1, input ReLU(N(0,1)) (about half zeros), BN + ReLU epilogue:
+  1. Eq. 1 statistics and occupancy bitmaps of the input (stats kernel),
+  2. Eq. 2 work as FLOPs per input byte (host arithmetic on the shape),
+  3. threshold dispatch on the device (s_thr 0.5, c_thr 32 FLOP/B),
+  4. the chosen tcgen05 kernel (dense or zero-skip) with the fused epilogue,
+     which also writes the output's occupancy for the next operator.
+Metric: effective TFLOP/s = dense-equivalent FLOPs / time.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl sparoa|reference]
+       [--workload conv|fc|resnet18|mobilenet_v2] [--batch B]
+For N > 1 launch one process per GPU with torch.distributed.run; every rank
+runs its own replica (weak scaling), timing is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "effective TFLOP/s & % roofline per op; synthetic CNN images/s at batch 1/32"
+NBUF = 40   # rotating input/output sets per step, 40 x 6.6 MB > 129 MB L2
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=60000)
+    p.add_argument("--warmup", type=int, default=400)
+    p.add_argument("--impl", default="sparoa", choices=["sparoa", "reference"])
+    p.add_argument("--workload", default="conv", choices=["conv", "fc", "resnet18", "mobilenet_v2"])
+    p.add_argument("--batch", type=int, default=32)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained", d["bf16_tflops"]),
+                "sm_max_mhz": d.get("sm_max_mhz"), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "sm_max_mhz": 2070.0, "source": "fallback"}
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.samples = []
+        self.proc = None
+        self.marks = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [s.strip() for s in line.split(",")]
+            if len(parts) >= 8:
+                self.samples.append((time.time(), parts))
+
+    def mark(self):
+        self.marks.append(time.time())
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        def num(s):
+            try:
+                return float(s)
+            except ValueError:
+                return None
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"]}
+        t0, t1 = (self.marks[0], self.marks[-1]) if len(self.marks) >= 2 else (0, 1e30)
+        inside = [p for t, p in self.samples if t0 <= t <= t1] or [p for _, p in self.samples]
+        sm = [num(p[0]) for p in inside if num(p[0]) is not None]
+        mx = [num(p[1]) for p in inside if num(p[1]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for p in inside for n, v in zip(names, p[4:8]) if v.lower() == "active"})
+        pw = [num(p[2]) for p in inside if num(p[2]) is not None]
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "power_w_max": max(pw) if pw else None, "samples": len(inside)}
+
+
+# ---------------------------------------------------------------------------
+# distributed helpers (one process per GPU; no data-path collective)
+# ---------------------------------------------------------------------------
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)), \
+        int(os.environ.get("WORLD_SIZE", 1))
+
+
+def max_over_ranks(value: float, world: int, device):
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2511_19457_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(key: str):
+    """Per-launch DRAM bytes of `key` from the committed ncu summary, or None
+    when the kernels changed since that capture."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        d = json.load(f)
+    e = d.get(key)
+    if not e or e.get("kernel_source_sha") != kernel_source_hash():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+# ---------------------------------------------------------------------------
+# CPU baseline: the oracle as it stands, on the host cores
+# ---------------------------------------------------------------------------
+def oracle_conv_step(d):
+    from oracle import oracle as orc
+    N, H, W, C = d["N"], d["H"], d["W"], d["Cin"]
+    st = orc.stats(d["x"], N * H * W, C)
+    wk = orc.conv_work(N, H, W, C, d["Cout"], 3, 3, 1, 1)
+    path = orc.decide(st.numel, st.nnz, wk.flops_per_byte, wk.macs_eq2, 0.5, 32.0)
+    y = orc.conv2d(d["x"], N, H, W, C, d["w"], d["Cout"], 3, 3, 1, 1, bn=d["bn"], act=1,
+                   skip_zeros=(path == 2))
+    bits = orc.f64_to_bf16(y)
+    orc.stats(bits, N * H * W, d["Cout"])
+    return wk.flops
+
+
+def cpu_baseline_conv(budget_s: float = 10.0, min_reps: int = 2):
+    from oracle import oracle as orc
+    from paper_2511_19457_gb300 import synth
+    d = synth.conv_layer(seed=0)
+    oracle_conv_step(d)  # load / first touch
+    reps, flops, t0 = 0, 0, time.perf_counter()
+    while reps < min_reps or time.perf_counter() - t0 < budget_s:
+        flops += oracle_conv_step(d)
+        reps += 1
+    dt = time.perf_counter() - t0
+    return {"value": flops / dt / 1e12, "unit": "TFLOP/s", "cores": orc.num_threads(),
+            "kind": "oracle",
+            "sample": f"{reps} full passes of the conv workload (stats, rule, fp64 direct conv, "
+                      f"bf16 rounding, output stats) in {dt:.1f} s"}
+
+
+# ---------------------------------------------------------------------------
+# the reference arm: the oracle, timed on the host
+# ---------------------------------------------------------------------------
+def run_reference(args):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return 0
+    from oracle import oracle as orc
+    from paper_2511_19457_gb300 import synth
+    d = synth.conv_layer(seed=0)
+    for _ in range(max(args.warmup, 0)):
+        oracle_conv_step(d)
+    steps = max(args.steps, 1)
+    t0 = time.perf_counter()
+    flops = 0
+    for _ in range(steps):
+        flops += oracle_conv_step(d)
+    dt = time.perf_counter() - t0
+    v = flops / dt / 1e12
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "TFLOP/s", "n_gpus": args.gpus,
+            "steps": steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": conv_config(),
+            "cpu_baseline": {"kind": "oracle", "cores": orc.num_threads(),
+                             "sample": f"{steps} full passes of the conv workload per timed region",
+                             "value": v, "unit": "TFLOP/s"},
+            "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def conv_config():
+    return {"workload": "conv3x3 s1 p1 NHWC bf16 [8,56,56,64]->64, BN+ReLU epilogue; "
+                        "Eq.1 stats + threshold dispatch + next-op occupancy",
+            "global_batch": 8, "seq_len": None, "parallelism": "replicas",
+            "thresholds": {"s_thr": 0.5, "c_thr_flops_per_byte": 32.0}}
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def graph_of(fn, count):
+    import torch
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for j in range(count):
+            fn(j)
+    return g
+
+
+def time_graph(g, replays):
+    import torch
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(replays):
+        g.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1)
+
+
+def run_conv(args, rank, local_rank, world, peaks):
+    import numpy as np
+    import torch
+
+    from paper_2511_19457_gb300 import sparoa as sp
+    from paper_2511_19457_gb300 import synth
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    ctx = sp.Context(local_rank)
+    d = synth.conv_layer(seed=0)
+    N, H, W, C, Co = 8, 56, 56, 64, 64
+    R = N * H * W
+    x0 = sp.bits_to_device(d["x"]).view(N, H, W, C)
+    xs = [x0.clone() for _ in range(NBUF)]
+    w = sp.bits_to_device(d["w"]).view(Co, 3, 3, C)
+    bn = torch.from_numpy(d["bn"]).to(dev)
+    ys = [torch.empty(N, H, W, Co, dtype=torch.bfloat16, device=dev) for _ in range(NBUF)]
+    xo = [sp.OccupancyBuffer(R, C) for _ in range(NBUF)]
+    yo = [sp.OccupancyBuffer(R, Co) for _ in range(NBUF)]
+    thr = sp.thresholds()
+    flops = 2 * N * H * W * Co * C * 9
+
+    def stats(j):
+        sp.sparoa_op_stats(ctx, xs[j], (N, H, W, C), occ=xo[j], host=False)
+
+    def conv(j):
+        sp.sparoa_conv2d(ctx, xs[j], w, ys[j], stride=1, pad=1, bn=bn, act=sp.ACT_RELU, thr=thr,
+                         x_occ=xo[j], y_occ=yo[j])
+
+    def step(j):
+        stats(j)
+        conv(j)
+
+    # path actually taken and the occupied share of K blocks (algorithmic work)
+    st = sp.sparoa_conv2d(ctx, xs[0], w, ys[0], stride=1, pad=1, bn=bn, act=sp.ACT_RELU, thr=thr,
+                          host=True)
+    path = "zero-skip" if st.path == sp.PATH_SKIP else "dense"
+    occ_frac = 1.0
+    if st.path == sp.PATH_SKIP:
+        sp.sparoa_op_stats(ctx, xs[0], (N, H, W, C), occ=xo[0], host=False)
+        occ_frac = conv_occupied_fraction(xo[0].to_host(), N, H, W, C)
+
+    for j in range(max(args.warmup, 3)):
+        step(j % NBUF)
+    torch.cuda.synchronize()
+    g_full = graph_of(step, NBUF)
+    rem = args.steps % NBUF
+    g_rem = graph_of(step, rem) if rem else None
+    g_full.replay()
+    torch.cuda.synchronize()
+
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    clocks = ClockSampler(int(vis.split(",")[local_rank]) if vis else local_rank)
+    clocks.start()
+    time.sleep(0.3)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.mark()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps // NBUF):
+        g_full.replay()
+    if g_rem is not None:
+        g_rem.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    clocks.mark()
+    ms = e0.elapsed_time(e1)
+    barrier(world)
+    ms = max_over_ranks(ms, world, dev)
+
+    # per-kernel durations (same launches, same buffers), measured live
+    reps = max(1, min(200, args.steps // NBUF))
+    g_stats = graph_of(stats, NBUF)
+    g_conv = graph_of(conv, NBUF)
+    g_stats.replay()
+    g_conv.replay()
+    stats_us = time_graph(g_stats, reps) * 1e3 / (reps * NBUF)
+    conv_us = time_graph(g_conv, reps) * 1e3 / (reps * NBUF)
+    clocks.stop()
+
+    # end to end through the public API: pinned host input -> device, step, result -> host
+    xh = torch.from_numpy(d["x"].view(np.int16)).view(torch.bfloat16).view(N, H, W, C).pin_memory()
+    yh = torch.empty(N, H, W, Co, dtype=torch.bfloat16).pin_memory()
+
+    def e2e_step(j):
+        xs[j].copy_(xh, non_blocking=True)
+        step(j)
+        yh.copy_(ys[j], non_blocking=True)
+
+    g_e2e = graph_of(e2e_step, NBUF)
+    g_e2e.replay()
+    e2e_reps = max(1, min(args.steps // NBUF, 250))
+    e2e_ms = time_graph(g_e2e, e2e_reps)
+    e2e_ms = max_over_ranks(e2e_ms, world, dev)
+    e2e_steps = e2e_reps * NBUF
+
+    # the roofline of the dominant kernel (the conv; stats kernel also reported)
+    alg_flops = flops * occ_frac
+    conv_bytes = (R * C + R * Co + Co * 9 * C) * 2 + 2 * int(sp._lib.sparoa_occupancy_bytes(R, Co))
+    achieved_tf = alg_flops / (conv_us * 1e-6) / 1e12
+    stats_bytes = R * C * 2 + int(sp._lib.sparoa_occupancy_bytes(R, C))
+    roof = {"bound": "tensor", "achieved": achieved_tf, "peak": peaks["bf16_tflops"],
+            "unit": "TFLOP/s", "frac": achieved_tf / peaks["bf16_tflops"],
+            "traffic": ncu_traffic("igemm_conv3x3_8x56x56x64"),
+            "kernel": "igemm_kernel<64> (" + path + ")", "kernel_us": conv_us,
+            "algorithmic_flops": alg_flops, "algorithmic_bytes": conv_bytes,
+            "hbm_view": {"achieved_gbs": conv_bytes / (conv_us * 1e-6) / 1e9,
+                         "frac": conv_bytes / (conv_us * 1e-6) / 1e9 / peaks["hbm_gbs"]},
+            "peak_source": peaks["source"]}
+    stats_kernel = {"kernel": "stats_kernel", "kernel_us": stats_us, "bytes": stats_bytes,
+                    "achieved_gbs": stats_bytes / (stats_us * 1e-6) / 1e9,
+                    "frac_hbm": stats_bytes / (stats_us * 1e-6) / 1e9 / peaks["hbm_gbs"]}
+
+    total_flops = flops * args.steps * world
+    value = total_flops / (ms * 1e-3) / 1e12
+    e2e_value = flops * e2e_steps * world / (e2e_ms * 1e-3) / 1e12
+    cfg = conv_config()
+    cfg.update({"path": path, "rho": st.sparsity, "occupied_k_fraction": occ_frac,
+                "l2": f"rotating {NBUF} input/output sets ({NBUF * 2 * R * C * 2 / 1e6:.0f} MB > 129 MB L2)",
+                "cuda_graph": True, "parallelism": f"replicas x{world}"})
+    line = {"metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded; stands in for ImageNet activations)", "config": cfg,
+            "roofline": roof, "stats_kernel": stats_kernel,
+            "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": R * C * 2,
+                    "d2h_bytes_per_step": R * Co * 2, "steps": e2e_steps},
+            "gpu_launches": 2 * args.steps,
+            "clocks": clocks.summary()}
+    ctx.close()
+    return line
+
+
+def conv_occupied_fraction(occ, N, H, W, C, k=3, pad=1):
+    """Share of (128-pixel M tile, tap, 32-channel block) K slices the zero-skip
+    kernel must stage: a slice is left out when none of the tile's 128 shifted
+    input pixels has an occupied 64-channel tile there."""
+    import numpy as np
+    T = (C + 63) // 64
+    bm = occ["row_bm"].reshape(N, H, W, -1)
+    tile_occ = np.stack([((bm[..., t // 64] >> np.uint64(t % 64)) & np.uint64(1)).astype(bool)
+                         for t in range(T)], axis=-1)            # [N, H, W, T]
+    M = N * H * W
+    m = np.arange(M)
+    n, oh, ow = m // (H * W), (m // W) % H, m % W
+    cb = (C + 31) // 32
+    total = occupied = 0
+    for r in range(k):
+        for s in range(k):
+            ih, iw = oh - pad + r, ow - pad + s
+            ok = (ih >= 0) & (ih < H) & (iw >= 0) & (iw < W)
+            vals = np.zeros((M, T), dtype=bool)
+            vals[ok] = tile_occ[n[ok], ih[ok], iw[ok]]
+            tiles = vals.reshape(-1, 128, T) if M % 128 == 0 else None
+            if tiles is None:
+                pad_rows = (-M) % 128
+                tiles = np.concatenate([vals, np.zeros((pad_rows, T), bool)]).reshape(-1, 128, T)
+            any_t = tiles.any(axis=1)                              # [tiles, T]
+            for b in range(cb):
+                total += any_t.shape[0]
+                occupied += int(any_t[:, (b * 32) // 64].sum())
+    return occupied / total if total else 1.0
+
+
+def run_graph_workload(args, rank, local_rank, world, peaks, name):
+    """CNN images/s through sparoa_run_graph (not the default bench line)."""
+    import torch
+
+    from paper_2511_19457_gb300 import sparoa as sp
+    from paper_2511_19457_gb300 import synth
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    ctx = sp.Context(local_rank)
+    ops, xb, shape = (synth.resnet18 if name == "resnet18" else synth.mobilenet_v2)(batch=args.batch)
+    graph = sp.Graph(ops)
+    x = sp.bits_to_device(xb).view(*shape)
+    recs = sp.sparoa_run_graph(ctx, graph, x, records=True)
+    flops = sum(r.stats.flops for r in recs)
+    for _ in range(max(args.warmup, 3)):
+        sp.sparoa_run_graph(ctx, graph, x)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        sp.sparoa_run_graph(ctx, graph, x)
+    g.replay()
+    ms = time_graph(g, args.steps) / args.steps
+    ms = max_over_ranks(ms, world, dev)
+    line = {"metric": METRIC, "value": args.batch * world / (ms * 1e-3), "unit": "images/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic", "effective_tflops": flops / (ms * 1e-3) / 1e12,
+            "config": {"workload": f"{name} B={args.batch} through sparoa_run_graph (CUDA graph)",
+                       "global_batch": args.batch * world},
+            "paths": [int(r.stats.path) for r in recs]}
+    ctx.close()
+    return line
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    rank, local_rank, world = dist_env()
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    peaks = measured_peaks()
+    if args.workload == "conv":
+        line = run_conv(args, rank, local_rank, world, peaks)
+        if rank == 0 and not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline_conv()
+    elif args.workload in ("resnet18", "mobilenet_v2"):
+        line = run_graph_workload(args, rank, local_rank, world, peaks, args.workload)
+    else:
+        raise SystemExit(f"workload {args.workload} is not wired into bench.py")
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

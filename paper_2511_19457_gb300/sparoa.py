@@ -334,3 +334,41 @@ def sparoa_run_graph(ctx: Context, graph: Graph, x, y=None, records=False):
     ctx._check(_lib.sparoa_run_graph(ctx.h, graph.ops, graph.n, _ptr(x), N, H, W, C, _ptr(y),
                                      0 if y is None else y.numel() * y.element_size(), recs))
     return list(recs) if records else None
+
+
+class _DevView:
+    def __init__(self, ptr, shape, typestr):
+        self.__cuda_array_interface__ = {"shape": tuple(shape), "typestr": typestr,
+                                         "data": (int(ptr), False), "version": 2}
+
+
+def view_device(ptr: int, shape, dtype=torch.bfloat16) -> torch.Tensor:
+    """A torch view (no copy) of device memory owned by the library, e.g. a
+    graph record's output; valid only as long as the library keeps it."""
+    if dtype == torch.bfloat16:
+        t = torch.as_tensor(_DevView(ptr, shape, "<i2"), device="cuda")
+        return t.view(torch.bfloat16)
+    typestr = {torch.float32: "<f4", torch.int32: "<i4", torch.uint8: "|u1"}[dtype]
+    return torch.as_tensor(_DevView(ptr, shape, typestr), device="cuda")
+
+
+def record_occupancy(rec: Record) -> dict:
+    """Copy a graph record's output occupancy to the host (same layout as
+    OccupancyBuffer.to_host)."""
+    o = rec.out_occ.contents
+    R, C = o.R, o.C
+    raw = view_device(o.nnz, (int(o.bytes),), torch.uint8).cpu().numpy()
+    base = o.nnz
+    T = (C + 63) // 64
+    W64 = (T + 63) // 64
+    RB = (R + 127) // 128
+    C32 = (C + 31) // 32
+
+    def view(ptr, dt, n):
+        off = ptr - base
+        return raw[off:off + n * np.dtype(dt).itemsize].view(dt).copy()
+
+    return {"nnz": int(view(o.nnz, np.uint64, 1)[0]), "col_nnz": view(o.col_nnz, np.uint32, C),
+            "tile_nnz": view(o.tile_nnz, np.uint32, T),
+            "row_bm": view(o.row_bm, np.uint64, R * W64).reshape(R, W64),
+            "blk_mask": view(o.blk_mask, np.uint32, RB * C32).reshape(RB, C32)}

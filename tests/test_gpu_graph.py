@@ -1,0 +1,99 @@
+"""sparoa_run_graph on ResNet-18 and MobileNetV2 topologies against the oracle (GPU).
+
+Teacher forcing: every operator is checked on exactly the bf16 tensor the GPU
+fed it (its input read back from the library's workspace), so that Eq. 1
+counts, bitmaps and dispatch decisions are compared bit for bit and each
+operator's output within the float tolerance.  The chained run (oracle fed only
+the graph input) is compared at the end with a looser bound, since bf16
+storage rounding at each of 20-50 operator boundaries compounds.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as orc
+from paper_2511_19457_gb300 import synth
+from tests._parity import assert_close, assert_occ_equal
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def sp():
+    from paper_2511_19457_gb300 import sparoa
+    return sparoa
+
+
+def _run(sp, name, batch, thr=None):
+    ops, xb, shape = getattr(synth, name)(batch=batch, seed=0, thr=thr)
+    ctx = sp.Context(0)
+    graph = sp.Graph(ops)
+    x = sp.bits_to_device(xb).view(*shape)
+    last = ops[-1]
+    recs = sp.sparoa_run_graph(ctx, graph, x, records=True)
+    torch.cuda.synchronize()
+    outs, occs = [], []
+    for r in recs:
+        shp = tuple(int(v) for v in r.out_shape)
+        t = sp.view_device(r.output, (int(np.prod(shp)),))
+        outs.append((sp.device_to_bits(t), shp))
+        occs.append(sp.record_occupancy(r))
+    ctx.close()
+    return ops, xb, shape, recs, outs, occs
+
+
+def _teacher_check(sp, ops, xb, shape, recs, outs, occs):
+    values = {0: (xb, shape)}
+    for i, (bits, shp) in enumerate(outs):
+        values[i + 1] = (bits, shp)
+    flips = 0
+    for i, op in enumerate(ops):
+        src = op["input"]
+        xin, xs = values[src]
+        res = values[op["residual"]][0] if op.get("residual", -1) >= 0 else None
+        ref = orc.run_op(op, xin, xs, res)
+        r = recs[i]
+        assert r.stats.nnz == ref.in_stats.nnz, f"op {i} ({op['kind']}): input nnz"
+        assert r.stats.path == ref.path, f"op {i} ({op['kind']}): path {r.stats.path} != {ref.path}"
+        if ref.work is not None:
+            assert r.stats.flops == ref.work.flops and r.stats.macs_eq2 == ref.work.macs_eq2
+        got_bits, got_shape = outs[i]
+        assert tuple(got_shape[-1:]) == tuple(ref.out_shape[-1:])
+        got = synth.bits_to_f32(got_bits).astype(np.float64).reshape(-1)
+        if op["kind"] == "maxpool":
+            assert np.array_equal(got, ref.out_f64.reshape(-1)), f"op {i} maxpool"
+        else:
+            assert_close(got, ref.out_f64, what=f"op {i} ({op['kind']})")
+        R = int(np.prod(got_shape[:-1]))
+        assert_occ_equal(occs[i], orc.stats(got_bits, R, got_shape[-1]), f"op {i} out occupancy")
+    return flips
+
+
+@pytest.mark.parametrize("name", ["resnet18", "mobilenet_v2"])
+def test_graph_teacher_forced(sp, name):
+    ops, xb, shape, recs, outs, occs = _run(sp, name, batch=1)
+    assert len(recs) == len(ops)
+    _teacher_check(sp, ops, xb, shape, recs, outs, occs)
+    kinds = [int(r.stats.path) for r in recs]
+    assert sp.PATH_DENSE in kinds or sp.PATH_SKIP in kinds
+    if name == "mobilenet_v2":
+        assert kinds.count(sp.PATH_DEPTHWISE) == 17
+
+
+def test_graph_batch8_resnet_forced_paths(sp):
+    """Both forced paths give the same network output within tolerance."""
+    logits = []
+    for force in (1, 2):
+        ops, xb, shape, recs, outs, occs = _run(sp, "resnet18", batch=8, thr={"force_path": force})
+        assert all(int(r.stats.path) in (force, 0) for r in recs)
+        logits.append(synth.bits_to_f32(outs[-1][0]).astype(np.float64))
+    assert_close(logits[1], logits[0], what="skip vs dense logits")
+
+
+@pytest.mark.parametrize("name", ["resnet18", "mobilenet_v2"])
+def test_graph_chained_end_to_end(sp, name):
+    ops, xb, shape, recs, outs, occs = _run(sp, name, batch=1)
+    ref = orc.run_graph(ops, xb, shape)
+    got = synth.bits_to_f32(outs[-1][0]).astype(np.float64)
+    # per-op parity is the bar; the chained drift of bf16 storage is bounded loosely
+    assert_close(got, ref[-1].out_f64, max_rel=8e-2, fro_rel=3e-2, what=f"{name} chained logits")
