@@ -308,6 +308,43 @@ sparoa_status sparoa_run_graph(sparoa_ctx *ctx, const sparoa_op *ops, int32_t n_
                                const void *x, int64_t N, int64_t H, int64_t W, int64_t C, void *y,
                                uint64_t y_bytes, sparoa_record *records);
 
+/* ------------------------------------------------------------------------ */
+/* Variant for callers that cannot allocate device memory                     */
+/* ------------------------------------------------------------------------ */
+
+/* Size of the library's static device scratch array used by
+ * sparoa_gemm_noalloc (4 MiB; every GPU that loads the library holds it until
+ * the process exits). */
+#define SPAROA_NOALLOC_SCRATCH_BYTES (4u << 20)
+
+/*
+ * sparoa_gemm without any device allocation.  The paper has no counterpart:
+ * this exists for callers that cannot call cudaMalloc -- work recorded into a
+ * CUDA graph by stream capture (an allocation cannot be captured), plugins
+ * inside a framework whose allocator owns the device memory, and loops with a
+ * memory budget fixed at start-up.  It computes exactly what sparoa_gemm
+ * computes with x_occ = y_occ = NULL, but needs no context: work goes to
+ * `stream` (a cudaStream_t; NULL = legacy default stream) on the current
+ * device, and the input's occupancy (the only scratch) lives in a static
+ * device array of SPAROA_NOALLOC_SCRATCH_BYTES bytes, 256 of which hold
+ * control words.
+ *   - The first call on a device looks the array's address up with
+ *     cudaGetSymbolAddress while that device is current; make that first call
+ *     before any stream capture starts.
+ *   - Calls share the array and each clears the part it uses before writing;
+ *     calls whose work overlaps on the GPU (other streams or host threads)
+ *     race on it and must be serialised by the caller.
+ *   - x [M, K], W [N, K], optional W_kn [K, N], y [M, N] as in sparoa_gemm.
+ *   - host_out (nullable) synchronises `stream` and fills the record.
+ * Errors: INVALID_ARG (as sparoa_gemm); UNSUPPORTED when the occupancy of a
+ * [M, K] input (sparoa_occupancy_bytes(M, K)) exceeds the array minus 256
+ * bytes, or a dimension exceeds 2^30; CUDA; TIMEOUT (host_out only).
+ */
+sparoa_status sparoa_gemm_noalloc(void *stream, const void *x, int64_t M, int64_t K,
+                                  const void *W, const void *W_kn, int64_t N,
+                                  const sparoa_epilogue *ep, const sparoa_thresholds *thr,
+                                  void *y, int32_t y_dtype, sparoa_stats *host_out);
+
 #ifdef __cplusplus
 }
 #endif

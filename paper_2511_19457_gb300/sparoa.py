@@ -102,11 +102,14 @@ _sig("sparoa_avgpool_global", [_P, _P, _I64, _I64, _I64, _I64, _P, ctypes.POINTE
 _sig("sparoa_bn_act", [_P, _P, _I64, _I64, ctypes.POINTER(Epilogue), _P, ctypes.POINTER(Occupancy)])
 _sig("sparoa_run_graph", [_P, ctypes.POINTER(Op), _I32, _P, _I64, _I64, _I64, _I64, _P,
                           ctypes.c_uint64, ctypes.POINTER(Record)])
+_sig("sparoa_gemm_noalloc", [_P, _P, _I64, _I64, _P, _P, _I64, ctypes.POINTER(Epilogue),
+                             ctypes.POINTER(Thresholds), _P, _I32, ctypes.POINTER(Stats)])
 
 EXPORTED = ["sparoa_create", "sparoa_destroy", "sparoa_set_stream", "sparoa_sync",
             "sparoa_status_str", "sparoa_last_error", "sparoa_occupancy_bytes",
             "sparoa_occupancy_init", "sparoa_op_stats", "sparoa_gemm", "sparoa_conv2d",
-            "sparoa_maxpool2d", "sparoa_avgpool_global", "sparoa_bn_act", "sparoa_run_graph"]
+            "sparoa_maxpool2d", "sparoa_avgpool_global", "sparoa_bn_act", "sparoa_run_graph",
+            "sparoa_gemm_noalloc"]
 
 
 class SparoaError(RuntimeError):
@@ -265,6 +268,25 @@ def sparoa_bn_act(ctx: Context, x, y, bias=None, bn=None, eps=1e-5, act=ACT_NONE
     ctx._bind()
     ep = _epi(bias, bn, eps, act, residual)
     ctx._check(_lib.sparoa_bn_act(ctx.h, _ptr(x), R, C, ctypes.byref(ep), _ptr(y), _occ(y_occ)))
+
+
+def sparoa_gemm_noalloc(x, W, y, W_kn=None, bias=None, bn=None, eps=1e-5, act=ACT_NONE,
+                        residual=None, thr: Thresholds | None = None, host=False):
+    """sparoa_gemm for callers that cannot allocate: no context, the input's
+    occupancy lives in the library's static device array (see sparoa.h).
+    Runs on the current torch stream of the current device."""
+    M, K = x.shape
+    N = W.shape[0]
+    ep = _epi(bias, bn, eps, act, residual)
+    st = Stats() if host else None
+    ydt = F32 if y.dtype == torch.float32 else BF16
+    rc = _lib.sparoa_gemm_noalloc(ctypes.c_void_p(torch.cuda.current_stream().cuda_stream),
+                                  _ptr(x), M, K, _ptr(W), _ptr(W_kn), N, ctypes.byref(ep),
+                                  ctypes.byref(thr) if thr is not None else None, _ptr(y), ydt,
+                                  ctypes.byref(st) if host else None)
+    if rc != OK:
+        raise SparoaError(rc, "sparoa_gemm_noalloc")
+    return st
 
 
 # ---------------------------------------------------------------------------
