@@ -368,8 +368,9 @@ sparoa_status run_conv(sparoa_ctx* ctx, const ConvPlan& c) {
   const bool pointwise = c.kh == 1 && c.kw == 1 && c.stride == 1 && c.pad == 0;
   a.M = (int)(c.N * c.Ho * c.Wo);
   a.N = (int)c.Cout;
-  a.conv = pointwise ? 0 : 1;
+  a.conv = pointwise ? 0 : ((c.Cp % 32) == 0 ? 2 : 1);
   a.x = static_cast<const __nv_bfloat16*>(c.x);
+  a.Nimg = (int)c.N;
   a.H = (int)c.H;
   a.W = (int)c.W;
   a.Cp = (int)c.Cp;
@@ -393,6 +394,7 @@ sparoa_status run_conv(sparoa_ctx* ctx, const ConvPlan& c) {
   if (c.yo) a.out_occ = to_dev(*c.yo);
   a.emit = c.yo ? 1 : 0;
   a.err = ctx->d_err();
+  if (a.conv == 2) choose_spatial_tile(a);
   SP_CUDA(launch_igemm(a, ctx->stream));
   return SPAROA_OK;
 }
@@ -611,8 +613,8 @@ sparoa_status sparoa_conv2d(sparoa_ctx* ctx, const void* x, int64_t N, int64_t H
   const bool depthwise = groups > 1 && groups == C_in && groups == C_out;
   if (groups > 1 && !depthwise)
     return fail(ctx, SPAROA_ERR_UNSUPPORTED, "conv2d: grouped convolution other than depthwise");
-  if (depthwise && (C_in % 8 || kh * kw > 9))
-    return fail(ctx, SPAROA_ERR_UNSUPPORTED, "conv2d: depthwise needs C %% 8 == 0 and kh*kw <= 9");
+  if (depthwise && (C_in % 8 || kh != 3 || kw != 3))
+    return fail(ctx, SPAROA_ERR_UNSUPPORTED, "conv2d: depthwise needs C %% 8 == 0 and a 3x3 kernel");
   if (!depthwise && (C_out % 8))
     return fail(ctx, SPAROA_ERR_INVALID_ARG, "conv2d: C_out must be a multiple of 8");
   DeviceGuard g(ctx->device);
@@ -798,7 +800,7 @@ sparoa_status sparoa_run_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_
             op.pad < 0 || op.groups <= 0 || !op.weight)
           return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: op %d conv geometry", i);
         const bool dw = op.groups > 1;
-        if (dw && (op.groups != op.c_in || op.groups != op.c_out || op.c_in % 8 || op.kh * op.kw > 9))
+        if (dw && (op.groups != op.c_in || op.groups != op.c_out || op.c_in % 8 || op.kh != 3 || op.kw != 3))
           return fail(ctx, SPAROA_ERR_UNSUPPORTED, "run_graph: op %d grouped conv", i);
         if (!dw && op.c_out % 8)
           return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: op %d C_out %% 8", i);

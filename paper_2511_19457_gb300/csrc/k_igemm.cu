@@ -1,30 +1,39 @@
 // Dense and zero-skipping implicit-GEMM kernel on the 5th-generation tensor
 // cores (tcgen05, accumulators in tensor memory), sm_103a.
 //
-// One CTA computes a 128 x BN tile of y = epilogue(A * B^T):
-//   A [M, K]  GEMM: the activation matrix, loaded by TMA (64-byte swizzle).
-//             Conv: gathered from the NHWC activation (implicit GEMM; K runs
-//             over (tap, channel) in [kh][kw][C] order) by 128 producer
-//             threads with cp.async, written in the same swizzled layout.
-//   B [N, K]  the weights, K-major, loaded by TMA.
-// K advances in 32-wide blocks (one 64-byte swizzle row, two MMAs of K = 16).
+// Persistent: one CTA per SM walks the output tiles (128 rows x BN columns)
+// of y = epilogue(A * B^T) with a static round-robin schedule.  Two tensor-
+// memory accumulators alternate between tiles, so the epilogue of tile i
+// (TMEM -> registers -> swizzled shared memory -> TMA store) overlaps the MMAs
+// of tile i + 1, and the shared-memory stage ring never drains between tiles.
 //
-// Threshold dispatch (Sec. 3 rule, thresholds as parameters) happens inside
-// the kernel: every CTA reads the Eq. 1 non-zero count of its input and
-// evaluates the rule, so no host round trip separates statistics and compute.
-// On the zero-skip path the producers leave out every K block whose
-// activations are all zero over the tile's 128 rows (Sec. 2.1: zero-valued
-// operations can be skipped without changing the output):
-//   GEMM: K block kb of row block b is skipped iff word kb of the input's
-//         block-column mask is 0 (no non-zero in those 32 columns x 128 rows);
-//   conv: a (tap, channel) block is skipped iff none of the 128 shifted input
-//         pixels has an occupied 64-channel tile there (row bitmaps; padding
-//         counts as unoccupied).
+// B [N, K] holds the weights (K-major; [C_out][kh][kw][C] for a convolution)
+// and is loaded by TMA.  A (128 rows of K) comes in one of three ways:
+//   mode 0  GEMM: A = x[M, K] row-major; rows m0..m0+127; 2-D TMA box.
+//   mode 2  convolution, C % BK == 0: the 128 rows are a spatial output tile
+//           of bw x bh pixels in bn images; for K block (tap r,s; BK channels)
+//           one 4-D TMA box {BK channels, bw, bh, bn} of the NHWC input at the
+//           shifted, strided origin (element strides = conv stride) is the A
+//           tile; out-of-range coordinates read zeros, which is the padding.
+//   mode 1  convolution, any C % 8 == 0 (the RGB stem): 128 consecutive output
+//           pixels, gathered by 128 producer threads with cp.async.
+// K advances in BK-wide blocks: BK = 64 with the 128-byte swizzle (four
+// tcgen05.mma of K = 16 per stage) or BK = 32 with the 64-byte swizzle.
+//
+// Threshold dispatch (Sec. 3 rule, thresholds as parameters) is evaluated in
+// the kernel prologue from the input's Eq. 1 count, so no host round trip
+// separates statistics and compute.  On the zero-skip path each tile leaves
+// out the K blocks whose activations are all zero over its 128 rows (Sec. 2.1:
+// products with zero activations can be skipped without changing the result):
+//   GEMM: from the 128-row block-column mask of x (one word per 32 columns);
+//   conv: from the row bitmaps of the tile's shifted input pixels, reduced
+//         per tile into a per-tap mask of occupied 64-channel tiles.
 // The epilogue applies bias / batch norm / residual / activation, stores y and
 // writes y's Eq. 1 count and occupancy bitmaps for the next operator.
 //
-// Warp roles (288 threads): warps 0-3 producers, warps 4-7 epilogue (TMEM lane
-// quarters 0-3), warp 8 TMEM allocation + MMA issue (lane 0).
+// Warp roles (288 threads): warps 0-3 producers (the skip masks; thread 0
+// issues TMA; all 128 gather in mode 1), warps 4-7 epilogue (TMEM lane
+// quarters), warp 8 TMEM allocation and MMA issue (lane 0).
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -38,30 +47,127 @@ namespace {
 
 constexpr int kThreads = 288;
 constexpr int kBM = 128;
-constexpr int kBK = 32;                   // K elements per stage
-constexpr int kAStageBytes = kBM * kBK * 2;  // 8 KiB
-constexpr int kLag = 2;                   // cp.async stages in flight per producer
+constexpr int kMaxKWords = 128;  // K-block occupancy bits: up to 4096 blocks
+constexpr int kMaxTaps = 64;
+constexpr int kStgBytes = 128 * 128;  // one 128-row x 128-byte output staging tile
+constexpr int kMaxAccCols = 2048;     // per-CTA column counters (output occupancy)
 
-template <int BN>
+template <int BN, int BK>
 struct Cfg {
-  static constexpr int kStages = BN == 64 ? 8 : (BN == 128 ? 6 : 4);
-  static constexpr int kBStageBytes = BN * kBK * 2;
+  static constexpr int kAStage = kBM * BK * 2;
+  static constexpr int kBStage = BN * BK * 2;
+  static constexpr int kStageBytes = kAStage + kBStage;
+  static constexpr int kBudget = 200 * 1024 - 2 * kStgBytes - 6 * 1024 - kMaxAccCols * 4;
+  static constexpr int kStagesRaw = kBudget / kStageBytes;
+  static constexpr int kStages = kStagesRaw > 12 ? 12 : kStagesRaw;
+  static constexpr int kLag = kStages - 2;  // cp.async stages in flight (mode 1)
   static constexpr int kAOff = 0;
-  static constexpr int kBOff = kAOff + kStages * kAStageBytes;
-  static constexpr int kBarOff = kBOff + kStages * kBStageBytes;    // 1024-aligned
-  static constexpr int kFlagOff = kBarOff + (2 * kStages + 1) * 8;
-  static constexpr int kScaleOff = (kFlagOff + (kStages + 8) * 4 + 15) & ~15;
+  static constexpr int kBOff = kAOff + kStages * kAStage;
+  static constexpr int kStgOff = kBOff + kStages * kBStage;          // 1024-aligned
+  static constexpr int kBarOff = kStgOff + 2 * kStgBytes;
+  static constexpr int kNumBars = 2 * kStages + 4;                   // full, empty, accf[2], acce[2]
+  static constexpr int kFlagOff = kBarOff + kNumBars * 8;
+  static constexpr int kKBitsOff = (kFlagOff + (kStages + 8) * 4 + 15) & ~15;
+  static constexpr int kTapOff = kKBitsOff + kMaxKWords * 4;
+  static constexpr int kScaleOff = kTapOff + kMaxTaps * 8;
   static constexpr int kShiftOff = kScaleOff + BN * 4;
-  static constexpr int kNzOff = (kShiftOff + BN * 4 + 15) & ~15;
-  static constexpr int kBytes = kNzOff + (BN / 64) * 128 * 8;
+  static constexpr int kCntOff = kShiftOff + BN * 4;
+  static constexpr int kAccOff = kCntOff + 4 * BN * 4;
+  static constexpr int kBytes = kAccOff + kMaxAccCols * 4 + 16;
   static constexpr int kSmem = kBytes + 1024;  // slack for 1024-byte alignment
+  static_assert(kStages >= 2, "stages");
+  static_assert(kSmem <= 227 * 1024, "shared memory");
 };
 
-template <int BN>
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const void* tmap, uint32_t bar, int c0,
+                                            int c1, int c2, int c3) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar)
+      : "memory");
+}
+
+// Launch geometry copied out of the kernel parameters into registers once:
+// reading IgemmArgs fields through a reference is a memory load, and every
+// asm statement with a memory clobber would force it again.
+struct Geo {
+  int conv, M, N, Nimg, H, W, Cp, Ho, Wo, kh, kw, stride, pad, bw, bh, bn, tw, th, Ktot;
+};
+
+__device__ __forceinline__ Geo make_geo(const IgemmArgs& a) {
+  Geo g;
+  g.conv = a.conv; g.M = a.M; g.N = a.N; g.Nimg = a.Nimg; g.H = a.H; g.W = a.W; g.Cp = a.Cp;
+  g.Ho = a.Ho; g.Wo = a.Wo; g.kh = a.kh; g.kw = a.kw; g.stride = a.stride; g.pad = a.pad;
+  g.bw = a.bw; g.bh = a.bh; g.bn = a.bn; g.tw = a.tw; g.th = a.th; g.Ktot = a.Ktot;
+  return g;
+}
+
+struct TileGeo {
+  int m0, tn0, th0, tw0, n0;
+};
+
+__device__ __forceinline__ TileGeo tile_geo(const Geo& p, int t, int nt, int BN) {
+  TileGeo g;
+  const int mi = t / nt;
+  g.n0 = (t - mi * nt) * BN;
+  g.m0 = 0;
+  g.tn0 = g.th0 = g.tw0 = 0;
+  if (p.conv == 2) {
+    const int per_img = p.th * p.tw;
+    g.tn0 = (mi / per_img) * p.bn;
+    const int rem = mi - (mi / per_img) * per_img;
+    g.th0 = (rem / p.tw) * p.bh;
+    g.tw0 = (rem - (rem / p.tw) * p.tw) * p.bw;
+  } else {
+    g.m0 = mi * kBM;
+  }
+  return g;
+}
+
+// Output pixel / row of tile row r and whether it exists.
+__device__ __forceinline__ int64_t tile_row(const Geo& p, const TileGeo& g, int r, bool& valid,
+                                            int& img, int& oh, int& ow) {
+  if (p.conv == 2) {
+    const int wl = r % p.bw, hl = (r / p.bw) % p.bh, nl = r / (p.bw * p.bh);
+    img = g.tn0 + nl;
+    oh = g.th0 + hl;
+    ow = g.tw0 + wl;
+    valid = img < p.Nimg && oh < p.Ho && ow < p.Wo;
+    return ((int64_t)img * p.Ho + oh) * p.Wo + ow;
+  }
+  const int64_t m = (int64_t)g.m0 + r;
+  valid = m < p.M;
+  if (p.conv == 1) {
+    const int hw = p.Ho * p.Wo;
+    img = valid ? (int)(m / hw) : 0;
+    const int rem = (int)(m - (int64_t)img * hw);
+    oh = valid ? rem / p.Wo : 0;
+    ow = valid ? rem - oh * p.Wo : 0;
+  } else {
+    img = oh = ow = 0;
+  }
+  return m;
+}
+
+template <int BN, int BK>
 __global__ void __launch_bounds__(kThreads, 1)
     igemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                 const IgemmArgs p) {
-  using C = Cfg<BN>;
+                 const __grid_constant__ CUtensorMap tmY, const IgemmArgs P) {
+  using C = Cfg<BN, BK>;
+  const Geo p = make_geo(P);
+  const EpiDev ep = P.ep;
+  const int act = P.ep.act;
+  const __nv_bfloat16* const residual = P.ep.residual;
+  const int y_f32 = P.y_f32;
+  const int emit = P.emit;
+  const __nv_bfloat16* const xin = P.x;
+  const uint32_t* const in_blk = P.in_blk;
+  const int in_C32 = P.in_C32;
+  const unsigned long long* const in_rowbm = P.in_rowbm;
+  const int in_W64 = P.in_W64;
+  uint32_t* const err = P.err;
+  void* const yout = P.y;
   constexpr int S = C::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -69,50 +175,56 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t sbase = smem_u32(smem);
   const uint32_t sA = sbase + C::kAOff;
   const uint32_t sB = sbase + C::kBOff;
-  const uint32_t bar_full = sbase + C::kBarOff;            // + 8*s
-  const uint32_t bar_empty = bar_full + 8 * S;             // + 8*s
-  const uint32_t bar_acc = bar_empty + 8 * S;
+  const uint32_t sStg = sbase + C::kStgOff;
+  const uint32_t bar_full = sbase + C::kBarOff;  // + 8*s
+  const uint32_t bar_empty = bar_full + 8 * S;   // + 8*s
+  const uint32_t bar_accf = bar_empty + 8 * S;   // + 8*b
+  const uint32_t bar_acce = bar_accf + 16;       // + 8*b
   int* flags = reinterpret_cast<int*>(smem + C::kFlagOff);
-  int* stage_end = flags;                  // [S]
-  volatile int* s_abort = flags + S;       // CTA-wide abort request
-  int* s_acc_has = flags + S + 1;          // accumulator holds MMA results
-  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(flags + S + 2);
-  volatile int* s_go = flags + S + 3;      // [2] producer broadcast
+  int* stage_last = flags;                // [S]: 1 = last stage of its tile
+  volatile int* s_abort = flags + S;      // CTA-wide abort request
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(flags + S + 1);
+  uint32_t* s_kbits = reinterpret_cast<uint32_t*>(smem + C::kKBitsOff);
+  unsigned long long* s_tap = reinterpret_cast<unsigned long long*>(smem + C::kTapOff);
   float* s_scale = reinterpret_cast<float*>(smem + C::kScaleOff);
   float* s_shift = reinterpret_cast<float*>(smem + C::kShiftOff);
-  uint64_t* s_nz = reinterpret_cast<uint64_t*>(smem + C::kNzOff);  // [BN/64][128]
+  const uint32_t sScale = sbase + C::kScaleOff;
+  const uint32_t sShift = sbase + C::kShiftOff;
+  uint32_t* s_cnt = reinterpret_cast<uint32_t*>(smem + C::kCntOff);  // [4][BN]
+  uint32_t* s_acc = reinterpret_cast<uint32_t*>(smem + C::kAccOff);  // [N] non-zeros per column
+  // Column counts of all tiles a CTA handles are summed here and flushed once
+  // (atomics on one address from every tile would serialise in L2).
+  const bool acc_smem = emit && p.N <= kMaxAccCols;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int path = decide_path(p.disp);
-  if (p.dense_only && path == 2) return;  // the zero-skip kernel of this launch runs instead
-  record_path(p.disp, path);
+  const int path = decide_path(P.disp);
+  if (P.dense_only && path == 2) return;  // the zero-skip kernel of this launch runs instead
+  record_path(P.disp, path);
   const bool skip = (path == 2);
-  const int m0 = blockIdx.x * kBM;
-  const int n0 = blockIdx.y * BN;
+  const int kblocks = (p.Ktot + BK - 1) / BK;
+  const int nt = (p.N + BN - 1) / BN;
+  const int mtiles = p.conv == 2 ? ((p.Nimg + p.bn - 1) / p.bn) * p.th * p.tw : (p.M + kBM - 1) / kBM;
+  const int tiles = mtiles * nt;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      mbar_init(bar_full + 8 * s, p.conv ? 129u : 1u);
+      mbar_init(bar_full + 8 * s, p.conv == 1 ? 129u : 1u);
       mbar_init(bar_empty + 8 * s, 1u);
     }
-    mbar_init(bar_acc, 1u);
-    *s_abort = 0;
-    *s_acc_has = 1;
-    fence_mbar_init();
-    if (!p.conv) prefetch_tmap(&tmA);
-    prefetch_tmap(&tmB);
-  }
-  if (warp == 8) tmem_alloc(smem_u32(s_tmem), (uint32_t)BN);
-  if (warp >= 4 && warp < 8) {
-    const int et = threadIdx.x - 128;
-    for (int c = et; c < BN; c += 128) {
-      float sc = 1.f, sh = 0.f;
-      if (n0 + c < p.N) epi_affine(p.ep, p.N, n0 + c, sc, sh);
-      s_scale[c] = sc;
-      s_shift[c] = sh;
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(bar_accf + 8 * b, 1u);
+      mbar_init(bar_acce + 8 * b, 128u);
     }
+    *s_abort = 0;
+    fence_mbar_init();
+    if (p.conv != 1) prefetch_tmap(&tmA);
+    prefetch_tmap(&tmB);
+    if (!y_f32) prefetch_tmap(&tmY);
   }
+  if (warp == 8) tmem_alloc(smem_u32(s_tmem), (uint32_t)(2 * BN));
+  if (acc_smem && warp >= 4 && warp < 8)
+    for (int c = threadIdx.x - 128; c < p.N; c += 128) s_acc[c] = 0u;
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -120,160 +232,203 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp < 4) {
     // ------------------------------------------------------------------ producers
-    const int r = threadIdx.x;  // A-tile row owned in conv mode
-    if (!p.conv) {
-      if (r == 0) {
-        int i = 0;
-        bool ok = true;
-        for (int kb = 0; kb * kBK < p.Ktot; ++kb) {
-          if (skip && p.in_blk[blockIdx.x * p.in_C32 + kb] == 0u) continue;
-          const int slot = i % S;
-          const uint32_t ph = (uint32_t)((i / S) & 1);
-          if (!mbar_wait(bar_empty + 8 * slot, ph ^ 1u, p.err, s_abort, kErrTimeoutEmpty)) {
-            ok = false;
-            break;
+    const int r = threadIdx.x;
+    const int cb_per_tap = p.Cp / BK;
+    int it = 0;        // stages filled so far (ring position)
+    int pending = 0;   // mode 1: filled stages whose A arrivals are still owed
+    bool ok = true;
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x) {
+      const TileGeo g = tile_geo(p, t, nt, BN);
+      bool rvalid;
+      int img, oh, ow;
+      tile_row(p, g, r, rvalid, img, oh, ow);
+      int last = kblocks - 1;
+      if (skip) {
+        // ---- occupied K blocks of this tile
+        named_bar_sync(1, 128);  // thread 0 is done with the previous tile's bits
+        if (p.conv == 0) {
+          for (int w0 = 0; w0 < kblocks && w0 < kMaxKWords * 32; w0 += 128) {
+            const int kb = w0 + r;
+            // a K block covers BK / 32 words of the 128-row block-column mask
+            bool occ = false;
+            if (kb < kblocks) {
+              const uint32_t* words = in_blk + (int64_t)(g.m0 >> 7) * in_C32;
+              occ = words[kb * (BK / 32)] != 0u;
+              if (BK == 64 && kb * 2 + 1 < in_C32) occ |= words[kb * 2 + 1] != 0u;
+            }
+            const uint32_t bits = __ballot_sync(0xffffffffu, occ);
+            if (lane == 0 && (w0 >> 5) + warp < kMaxKWords) s_kbits[(w0 >> 5) + warp] = bits;
           }
-          stage_end[slot] = 0;
-          mbar_arrive_expect_tx(bar_full + 8 * slot, (uint32_t)(kAStageBytes + C::kBStageBytes));
-          tma_load_2d(sA + slot * kAStageBytes, &tmA, bar_full + 8 * slot, kb * kBK, m0);
-          tma_load_2d(sB + slot * C::kBStageBytes, &tmB, bar_full + 8 * slot, kb * kBK, n0);
-          ++i;
-        }
-        if (ok) {
-          const int slot = i % S;
-          const uint32_t ph = (uint32_t)((i / S) & 1);
-          if (mbar_wait(bar_empty + 8 * slot, ph ^ 1u, p.err, s_abort, kErrTimeoutEmpty)) {
-            stage_end[slot] = 1;
-            mbar_arrive(bar_full + 8 * slot);
-          }
-        }
-      }
-    } else {
-      // Implicit GEMM gather.  Row r of the tile is output pixel m0 + r.
-      const int m = m0 + r;
-      const bool mvalid = m < p.M;
-      int img = 0, oh = 0, ow = 0;
-      if (mvalid) {
-        const int hw = p.Ho * p.Wo;
-        img = m / hw;
-        const int rem = m - img * hw;
-        oh = rem / p.Wo;
-        ow = rem - oh * p.Wo;
-      }
-      const int ih0 = oh * p.stride - p.pad;
-      const int iw0 = ow * p.stride - p.pad;
-      const __nv_bfloat16* ximg = p.x + (int64_t)img * p.H * p.W * p.Cp;
-      const int64_t pix0 = (int64_t)img * p.H * p.W;
-      const bool cp32 = (p.Cp % 32) == 0;
-      int i = 0;           // stages filled
-      int pending = 0;     // filled stages whose A arrivals are still owed
-      bool ok = true;
-      for (int kb = 0; kb * kBK < p.Ktot; ++kb) {
-        // geometry of this thread's four 16-byte chunks
-        const __nv_bfloat16* src[4];
-        bool val[4];
-        bool occ = false;
-        int tap = 0, cbase = 0;
-        if (cp32) {
-          const int flat = kb * kBK;
-          tap = flat / p.Cp;
-          cbase = flat - tap * p.Cp;
-        }
+        } else {
+          if (r < kMaxTaps) s_tap[r] = 0ull;
+          named_bar_sync(1, 128);
+          const int taps = p.kh * p.kw < kMaxTaps ? p.kh * p.kw : kMaxTaps;
+          for (int t0 = 0; t0 < taps; t0 += 8) {
+            unsigned long long wv[8];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          int t, c;
-          const int flat = kb * kBK + 8 * j;
-          if (cp32) {
-            t = tap;
-            c = cbase + 8 * j;
-          } else {
-            t = flat / p.Cp;
-            c = flat - t * p.Cp;
+            for (int u = 0; u < 8; ++u) {  // issue 8 taps' loads before reducing any
+              const int tp = t0 + u;
+              const int ih = oh * p.stride - p.pad + tp / p.kw;
+              const int iw = ow * p.stride - p.pad + tp % p.kw;
+              wv[u] = 0ull;
+              if (tp < taps && rvalid && ih >= 0 && ih < p.H && iw >= 0 && iw < p.W)
+                wv[u] = in_rowbm[(((int64_t)img * p.H + ih) * p.W + iw) * in_W64];
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+              unsigned long long w = wv[u];
+#pragma unroll
+              for (int s = 16; s > 0; s >>= 1) w |= __shfl_xor_sync(0xffffffffu, w, s);
+              if (lane == 0 && w) atomicOr(&s_tap[t0 + u], w);
+            }
           }
-          const int rr = t / p.kw;
-          const int ss = t - rr * p.kw;
-          const int ih = ih0 + rr, iw = iw0 + ss;
-          val[j] = mvalid && flat < p.Ktot && ih >= 0 && ih < p.H && iw >= 0 && iw < p.W;
-          src[j] = val[j] ? ximg + ((int64_t)ih * p.W + iw) * p.Cp + c : p.x;
-          if (skip && val[j]) {
-            const int tile = c >> 6;
-            const unsigned long long wbits =
-                p.in_rowbm[(pix0 + (int64_t)ih * p.W + iw) * p.in_W64 + (tile >> 6)];
-            occ |= ((wbits >> (tile & 63)) & 1ull) != 0ull;
-          }
-        }
-        if (skip && !named_bar_or(1, 128, occ)) continue;
-        const int slot = i % S;
-        const uint32_t ph = (uint32_t)((i / S) & 1);
-        if (r == 0) {
-          const bool go = mbar_wait(bar_empty + 8 * slot, ph ^ 1u, p.err, s_abort, kErrTimeoutEmpty);
-          s_go[i & 1] = go ? 1 : 0;
-          if (go) {
-            stage_end[slot] = 0;
-            mbar_arrive_expect_tx(bar_full + 8 * slot, (uint32_t)C::kBStageBytes);
-            tma_load_2d(sB + slot * C::kBStageBytes, &tmB, bar_full + 8 * slot, kb * kBK, n0);
+          named_bar_sync(1, 128);
+          const bool many = p.kh * p.kw > kMaxTaps || in_W64 > 1;  // no per-tap masks: keep all
+          for (int w0 = 0; w0 < kblocks && w0 < kMaxKWords * 32; w0 += 128) {
+            const int kb = w0 + r;
+            bool occ = false;
+            if (kb < kblocks) {
+              if (many) {
+                occ = true;
+              } else {
+#pragma unroll
+                for (int j = 0; j < BK / 8; ++j) {
+                  const int flat = kb * BK + 8 * j;
+                  if (flat >= p.Ktot) break;
+                  const int tp = flat / p.Cp;
+                  const int c = flat - tp * p.Cp;
+                  occ |= ((s_tap[tp] >> (c >> 6)) & 1ull) != 0ull;
+                }
+              }
+            }
+            const uint32_t bits = __ballot_sync(0xffffffffu, occ);
+            if (lane == 0 && (w0 >> 5) + warp < kMaxKWords) s_kbits[(w0 >> 5) + warp] = bits;
           }
         }
         named_bar_sync(1, 128);
-        if (!s_go[i & 1]) {
-          ok = false;
-          break;
-        }
-        const uint32_t dst = sA + slot * kAStageBytes;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) cp_async_16(dst + sw64_offset(r, j), src[j], val[j] ? 16u : 0u);
-        cp_async_commit();
-        ++i;
-        ++pending;
-        if (pending > kLag) {
-          cp_async_wait<kLag>();
-          fence_proxy_async_smem();
-          mbar_arrive(bar_full + 8 * ((i - 1 - kLag) % S));
-          --pending;
+        // last occupied block; a tile with none still runs block 0 (its data is all zero)
+        last = 0;
+        const int wtop = (kblocks - 1) >> 5;
+        for (int w = wtop; w >= 0; --w) {
+          uint32_t bits = w < kMaxKWords ? s_kbits[w] : 0xffffffffu;
+          if (w == wtop) bits &= 0xffffffffu >> (31 - ((kblocks - 1) & 31));
+          if (bits) {
+            last = w * 32 + 31 - __clz(bits);
+            break;
+          }
         }
       }
+      if (!ok) continue;  // keep the skip-mask barriers in step; issue nothing more
+      if (p.conv != 1) {
+        if (r == 0) {
+          for (int kb = 0; kb <= last; ++kb) {
+            if (skip && kb != last && kb < kMaxKWords * 32 && !((s_kbits[kb >> 5] >> (kb & 31)) & 1u))
+              continue;
+            const int slot = it % S;
+            const uint32_t ph = (uint32_t)((it / S) & 1);
+            if (!mbar_wait(bar_empty + 8 * slot, ph ^ 1u, err, s_abort, kErrTimeoutEmpty)) {
+              ok = false;
+              break;
+            }
+            stage_last[slot] = (kb == last) ? 1 : 0;
+            mbar_arrive_expect_tx(bar_full + 8 * slot, (uint32_t)C::kStageBytes);
+            if (p.conv == 0) {
+              tma_load_2d(sA + slot * C::kAStage, &tmA, bar_full + 8 * slot, kb * BK, g.m0);
+            } else {
+              const int tap = kb / cb_per_tap;
+              const int cb = kb - tap * cb_per_tap;
+              const int rr = tap / p.kw, ss = tap - (tap / p.kw) * p.kw;
+              tma_load_4d(sA + slot * C::kAStage, &tmA, bar_full + 8 * slot, cb * BK,
+                          g.tw0 * p.stride - p.pad + ss, g.th0 * p.stride - p.pad + rr, g.tn0);
+            }
+            tma_load_2d(sB + slot * C::kBStage, &tmB, bar_full + 8 * slot, kb * BK, g.n0);
+            ++it;
+          }
+        }
+      } else {
+        // Implicit-GEMM gather: row r is output pixel m0 + r.
+        const int ih0 = oh * p.stride - p.pad;
+        const int iw0 = ow * p.stride - p.pad;
+        const __nv_bfloat16* ximg = xin + (int64_t)img * p.H * p.W * p.Cp;
+        for (int kb = 0; kb <= last; ++kb) {
+          if (skip && kb != last && kb < kMaxKWords * 32 && !((s_kbits[kb >> 5] >> (kb & 31)) & 1u))
+            continue;
+          const int slot = it % S;
+          const uint32_t ph = (uint32_t)((it / S) & 1);
+          if (!mbar_wait(bar_empty + 8 * slot, ph ^ 1u, err, s_abort, kErrTimeoutEmpty)) {
+            ok = false;
+            break;
+          }
+          if (r == 0) {
+            stage_last[slot] = (kb == last) ? 1 : 0;
+            mbar_arrive_expect_tx(bar_full + 8 * slot, (uint32_t)C::kBStage);
+            tma_load_2d(sB + slot * C::kBStage, &tmB, bar_full + 8 * slot, kb * BK, g.n0);
+          }
+          const uint32_t dst = sA + slot * C::kAStage;
+#pragma unroll
+          for (int j = 0; j < BK / 8; ++j) {
+            const int flat = kb * BK + 8 * j;
+            const int tp = flat / p.Cp;
+            const int c = flat - tp * p.Cp;
+            const int rr = tp / p.kw;
+            const int ss = tp - rr * p.kw;
+            const int ih = ih0 + rr, iw = iw0 + ss;
+            const bool val = rvalid && flat < p.Ktot && ih >= 0 && ih < p.H && iw >= 0 && iw < p.W;
+            const __nv_bfloat16* src = val ? ximg + ((int64_t)ih * p.W + iw) * p.Cp + c : xin;
+            cp_async_16(dst + swz_offset<BK>(r, j), src, val ? 16u : 0u);
+          }
+          cp_async_commit();
+          ++it;
+          ++pending;
+          if (pending > C::kLag) {
+            cp_async_wait<C::kLag>();
+            fence_proxy_async_smem();
+            mbar_arrive(bar_full + 8 * ((it - 1 - C::kLag) % S));
+            --pending;
+          }
+        }
+      }
+    }
+    if (p.conv == 1) {
       cp_async_wait<0>();
       fence_proxy_async_smem();
-      for (int q = pending; q > 0; --q) mbar_arrive(bar_full + 8 * ((i - q) % S));
-      named_bar_sync(1, 128);
-      if (ok && r == 0) {
-        const int slot = i % S;
-        const uint32_t ph = (uint32_t)((i / S) & 1);
-        if (mbar_wait(bar_empty + 8 * slot, ph ^ 1u, p.err, s_abort, kErrTimeoutEmpty)) {
-          stage_end[slot] = 1;
-          asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0], %1;" ::"r"(bar_full + 8 * slot),
-                       "r"(129)
-                       : "memory");
-        }
-      }
+      for (int q = pending; q > 0; --q) mbar_arrive(bar_full + 8 * ((it - q) % S));
     }
   } else if (warp == 8) {
     // ------------------------------------------------------------------ MMA issue
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(kBM, BN);
-      int i = 0;
-      bool any = false;
-      while (true) {
-        const int slot = i % S;
-        const uint32_t ph = (uint32_t)((i / S) & 1);
-        if (!mbar_wait(bar_full + 8 * slot, ph, p.err, s_abort, kErrTimeoutFull)) break;
-        if (stage_end[slot]) break;
+      int it = 0, j = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++j) {
+        const int b = j & 1;
+        if (!mbar_wait(bar_acce + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort,
+                       kErrTimeoutAcc))
+          break;
         tc_fence_after();
-        const uint32_t a = sA + slot * kAStageBytes;
-        const uint32_t b = sB + slot * C::kBStageBytes;
+        const uint32_t d = tmem + (uint32_t)(b * BN);
+        bool first = true;
+        while (true) {
+          const int slot = it % S;
+          const uint32_t ph = (uint32_t)((it / S) & 1);
+          if (!mbar_wait(bar_full + 8 * slot, ph, err, s_abort, kErrTimeoutFull)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const bool last = stage_last[slot] != 0;
+          const uint32_t a = sA + slot * C::kAStage;
+          const uint32_t bb = sB + slot * C::kBStage;
 #pragma unroll
-        for (int k = 0; k < kBK / 16; ++k)
-          tc_mma_bf16(tmem, smem_desc_sw64(a + 32 * k), smem_desc_sw64(b + 32 * k), idesc,
-                      (any || k > 0) ? 1u : 0u);
-        any = true;
-        tc_commit(bar_empty + 8 * slot);
-        ++i;
-      }
-      if (any) {
-        tc_commit(bar_acc);
-      } else {
-        *s_acc_has = 0;
-        mbar_arrive(bar_acc);
+          for (int k = 0; k < BK / 16; ++k)
+            tc_mma_bf16(d, smem_desc_kmajor<BK>(a + 32 * k), smem_desc_kmajor<BK>(bb + 32 * k),
+                        idesc, (!first || k > 0) ? 1u : 0u);
+          first = false;
+          tc_commit(bar_empty + 8 * slot);
+          ++it;
+          if (last) break;
+        }
+        if (ok) tc_commit(bar_accf + 8 * b);
       }
     }
   } else {
@@ -281,101 +436,206 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int q = warp & 3;            // TMEM lane quarter of this warp
     const int r = q * 32 + lane;       // tile row
     const int et = threadIdx.x - 128;  // 0..127
-    const int64_t m = (int64_t)m0 + r;
-    const bool mvalid = m < p.M;
-    bool ok = mbar_wait(bar_acc, 0u, p.err, s_abort, kErrTimeoutAcc);
-    ok = __all_sync(0xffffffffu, ok);
-    tc_fence_after();
-    const bool has = ok && (*s_acc_has != 0);
     const bool vec = (p.N % 8) == 0;
-    for (int c0 = 0; c0 < BN; c0 += 16) {
-      float v[16];
-      if (has) {
-        tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, v);
-      } else {
-#pragma unroll
-        for (int j = 0; j < 16; ++j) v[j] = 0.f;
+    int j = 0;
+    int stg_count = 0;  // staging tiles handed to TMA so far
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++j) {
+      const int b = j & 1;
+      const TileGeo g = tile_geo(p, t, nt, BN);
+      bool mvalid;
+      int img, oh, ow;
+      const int64_t m = tile_row(p, g, r, mvalid, img, oh, ow);
+      // per-tile column affine (the previous tile's readers are past its last barrier)
+      for (int c = et; c < BN; c += 128) {
+        float sc = 1.f, sh = 0.f;
+        if (g.n0 + c < p.N) epi_affine(ep, p.N, g.n0 + c, sc, sh);
+        s_scale[c] = sc;
+        s_shift[c] = sh;
       }
-      const int nb = n0 + c0;
-      const bool full = vec && (nb + 16 <= p.N);
-      float res[16];
-#pragma unroll
-      for (int j = 0; j < 16; ++j) res[j] = 0.f;
-      if (p.ep.residual && mvalid) {
-        const __nv_bfloat16* rp = p.ep.residual + m * p.N + nb;
-        if (full) {
-          const uint4 r0 = *reinterpret_cast<const uint4*>(rp);
-          const uint4 r1 = *reinterpret_cast<const uint4*>(rp + 8);
-          const __nv_bfloat16* h0 = reinterpret_cast<const __nv_bfloat16*>(&r0);
-          const __nv_bfloat16* h1 = reinterpret_cast<const __nv_bfloat16*>(&r1);
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            res[j] = __bfloat162float(h0[j]);
-            res[8 + j] = __bfloat162float(h1[j]);
-          }
-        } else {
-          for (int j = 0; j < 16; ++j)
-            if (nb + j < p.N) res[j] = __bfloat162float(rp[j]);
-        }
-      }
-      uint32_t nzbits = 0;
-      if (p.y_f32) {
-        float o[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j)
-          o[j] = epi_act(fmaf(v[j], s_scale[c0 + j], s_shift[c0 + j]) + res[j], p.ep.act);
-        if (mvalid) {
-          float* yp = reinterpret_cast<float*>(p.y) + m * p.N + nb;
-          if (full && (p.N % 4) == 0) {
-#pragma unroll
-            for (int j = 0; j < 16; j += 4)
-              *reinterpret_cast<float4*>(yp + j) = make_float4(o[j], o[j + 1], o[j + 2], o[j + 3]);
-          } else {
-            for (int j = 0; j < 16; ++j)
-              if (nb + j < p.N) yp[j] = o[j];
-          }
-        }
-      } else {
-        __align__(16) __nv_bfloat16 o[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          o[j] = __float2bfloat16_rn(
-              epi_act(fmaf(v[j], s_scale[c0 + j], s_shift[c0 + j]) + res[j], p.ep.act));
-          const uint16_t bits = __bfloat16_as_ushort(o[j]);
-          if (mvalid && nb + j < p.N && bf16_nz(bits)) nzbits |= 1u << j;
-        }
-        if (mvalid) {
-          __nv_bfloat16* yp = reinterpret_cast<__nv_bfloat16*>(p.y) + m * p.N + nb;
-          if (full) {
-            *reinterpret_cast<uint4*>(yp) = *reinterpret_cast<const uint4*>(&o[0]);
-            *reinterpret_cast<uint4*>(yp + 8) = *reinterpret_cast<const uint4*>(&o[8]);
-          } else {
-            for (int j = 0; j < 16; ++j)
-              if (nb + j < p.N) yp[j] = o[j];
-          }
-        }
-      }
-      if (p.emit) {
-        uint64_t* w = &s_nz[(c0 >> 6) * 128 + r];
-        const int sh = c0 & 63;
-        if (sh == 0) *w = (uint64_t)nzbits;
-        else *w |= (uint64_t)nzbits << sh;
-      }
-    }
-    if (p.emit) {
-      tc_fence_before();
+      bool ok = mbar_wait(bar_accf + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutAcc);
+      ok = __all_sync(0xffffffffu, ok);
       named_bar_sync(2, 128);
-      for (int g = 0; g < BN / 64; ++g) {
-        if (n0 + 64 * g < p.N) flush_tile(&s_nz[g * 128], m0, n0 + 64 * g, p.out_occ, et, 128);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * BN);
+      const OccDev o = P.out_occ;  // registers, not parameter-space loads
+      const int blk = mvalid ? (int)(m >> 7) : -1;
+      const uint32_t grp = p.conv == 2 ? __match_any_sync(0xffffffffu, blk) : 0xffffffffu;
+      const bool leader = (__ffs(grp) - 1) == lane;
+      unsigned long long tl = 0ull;  // this row's occupied 64-column tiles
+      // One 64-column group per iteration, kept as a loop (not unrolled) so the
+      // epilogue's instructions stay in the instruction cache across groups.
+#pragma unroll 1
+      for (int gcol = 0; gcol < BN / 64; ++gcol) {
+        const int nbase = g.n0 + gcol * 64;
+        if (nbase >= p.N) break;  // uniform across the epilogue warps
+        uint32_t stg = 0;
+        if (!y_f32) {
+          stg = sStg + (uint32_t)((stg_count & 1) * kStgBytes);
+          if (et == 0) bulk_wait_read<1>();  // the store that used this buffer has read it
+          named_bar_sync(2, 128);
+        }
+        uint32_t raw2[2][32];
+        tmem_ld32_nowait(tbase + (uint32_t)(gcol * 64), raw2[0]);
+        tmem_ld32_nowait(tbase + (uint32_t)(gcol * 64 + 32), raw2[1]);
+        tmem_wait_ld32(raw2[0]);
+        tmem_wait_ld32(raw2[1]);
+        uint32_t rwg[2] = {0u, 0u};  // non-zero bits of this row in the group's two 32-column words
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+#pragma unroll
+          for (int c16s = 0; c16s < 2; ++c16s) {
+            const int cg0 = half * 32 + c16s * 16;  // column inside the group
+            const int nb = nbase + cg0;
+            const bool full = vec && (nb + 16 <= p.N);
+            const float4* sc4 = reinterpret_cast<const float4*>(s_scale + gcol * 64 + cg0);
+            const float4* sh4 = reinterpret_cast<const float4*>(s_shift + gcol * 64 + cg0);
+            float o32[16];
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) {
+              const float4 sc = sc4[q4];
+              const float4 sh = sh4[q4];
+              o32[4 * q4 + 0] = fmaf(__uint_as_float(raw2[half][c16s * 16 + 4 * q4 + 0]), sc.x, sh.x);
+              o32[4 * q4 + 1] = fmaf(__uint_as_float(raw2[half][c16s * 16 + 4 * q4 + 1]), sc.y, sh.y);
+              o32[4 * q4 + 2] = fmaf(__uint_as_float(raw2[half][c16s * 16 + 4 * q4 + 2]), sc.z, sh.z);
+              o32[4 * q4 + 3] = fmaf(__uint_as_float(raw2[half][c16s * 16 + 4 * q4 + 3]), sc.w, sh.w);
+            }
+            if (residual && mvalid) {
+              const __nv_bfloat16* rp = residual + m * p.N + nb;
+              if (full) {
+                const uint4 r0 = *reinterpret_cast<const uint4*>(rp);
+                const uint4 r1 = *reinterpret_cast<const uint4*>(rp + 8);
+                const __nv_bfloat162* h0 = reinterpret_cast<const __nv_bfloat162*>(&r0);
+                const __nv_bfloat162* h1 = reinterpret_cast<const __nv_bfloat162*>(&r1);
+#pragma unroll
+                for (int jj = 0; jj < 4; ++jj) {
+                  const float2 a0 = __bfloat1622float2(h0[jj]);
+                  const float2 a1 = __bfloat1622float2(h1[jj]);
+                  o32[2 * jj] += a0.x;
+                  o32[2 * jj + 1] += a0.y;
+                  o32[8 + 2 * jj] += a1.x;
+                  o32[8 + 2 * jj + 1] += a1.y;
+                }
+              } else {
+                for (int jj = 0; jj < 16; ++jj)
+                  if (nb + jj < p.N) o32[jj] += __bfloat162float(rp[jj]);
+              }
+            }
+            if (act == 1) {
+#pragma unroll
+              for (int jj = 0; jj < 16; ++jj) o32[jj] = o32[jj] > 0.f ? o32[jj] : 0.f;
+            } else if (act == 2) {
+#pragma unroll
+              for (int jj = 0; jj < 16; ++jj) o32[jj] = o32[jj] > 0.f ? (o32[jj] < 6.f ? o32[jj] : 6.f) : 0.f;
+            }
+            if (y_f32) {
+              if (mvalid) {
+                float* yp = reinterpret_cast<float*>(yout) + m * p.N + nb;
+                if (full && (p.N % 4) == 0) {
+#pragma unroll
+                  for (int jj = 0; jj < 16; jj += 4)
+                    *reinterpret_cast<float4*>(yp + jj) = make_float4(o32[jj], o32[jj + 1], o32[jj + 2], o32[jj + 3]);
+                } else {
+                  for (int jj = 0; jj < 16; ++jj)
+                    if (nb + jj < p.N) yp[jj] = o32[jj];
+                }
+              }
+            } else {
+              uint32_t pk[8];
+              uint32_t nzbits = 0;
+#pragma unroll
+              for (int jj = 0; jj < 8; ++jj) {
+                const __nv_bfloat162 h2 = __floats2bfloat162_rn(o32[2 * jj], o32[2 * jj + 1]);
+                pk[jj] = *reinterpret_cast<const uint32_t*>(&h2);
+                nzbits |= ((pk[jj] & 0x7FFFu) ? 1u : 0u) << (2 * jj);
+                nzbits |= ((pk[jj] & 0x7FFF0000u) ? 1u : 0u) << (2 * jj + 1);
+              }
+              const int nvalid = p.N - nb;  // columns of this chunk inside the tensor
+              if (!mvalid) nzbits = 0;
+              else if (nvalid < 16) nzbits &= nvalid > 0 ? ((1u << nvalid) - 1u) : 0u;
+              rwg[half] |= nzbits << (c16s * 16);
+              // staging tile: 128 rows x 128 bytes with the 128-byte swizzle the TMA store reads
+              const uint32_t row_addr = stg + (uint32_t)r * 128u;
+              const int j0 = (half * 2 + c16s) * 2;
+              sts_u4(row_addr + (uint32_t)((j0 ^ (r & 7)) << 4), make_uint4(pk[0], pk[1], pk[2], pk[3]));
+              sts_u4(row_addr + (uint32_t)(((j0 + 1) ^ (r & 7)) << 4), make_uint4(pk[4], pk[5], pk[6], pk[7]));
+            }
+          }
+        }
+        if (!y_f32) {
+          fence_proxy_async_smem();
+          named_bar_sync(2, 128);
+          if (et == 0) {
+            if (p.conv == 2) tma_store_4d(&tmY, stg, nbase, g.tw0, g.th0, g.tn0);
+            else tma_store_2d(&tmY, stg, nbase, g.m0);
+            bulk_commit();
+          }
+          ++stg_count;
+        }
+        if (emit) {
+          // this group's share of the output occupancy
+          if (rwg[0] | rwg[1]) tl |= 1ull << ((nbase >> 6) & 63);
+#pragma unroll
+          for (int w = 0; w < 2; ++w) {
+            const uint32_t bits = __reduce_or_sync(grp, rwg[w]);
+            const int word = (nbase >> 5) + w;
+            if (leader && blk >= 0 && bits && word < o.C32) atomicOr(&o.blk_mask[blk * o.C32 + word], bits);
+            // lane j: non-zeros of column 32w + j of this group in the warp's 32 rows
+            s_cnt[q * BN + gcol * 64 + w * 32 + lane] = __popc(warp_transpose32(rwg[w]));
+          }
+        }
       }
+      // accumulator b is free for the MMA of tile j + 2
+      tc_fence_before();
+      mbar_arrive(bar_acce + 8 * b);
+      if (emit) {
+        if (mvalid && tl) atomicOr(&o.row_bm[m * o.W64 + ((g.n0 >> 6) >> 6)], tl);
+        named_bar_sync(2, 128);
+        for (int c = et; c < BN; c += 128) {
+          const bool live = g.n0 + c < o.C;
+          const uint32_t cnt =
+              live ? s_cnt[c] + s_cnt[BN + c] + s_cnt[2 * BN + c] + s_cnt[3 * BN + c] : 0u;
+          if (acc_smem) {
+            if (live) s_acc[g.n0 + c] += cnt;  // one thread per column of this tile
+          } else {
+            if (cnt) atomicAdd(&o.col_nnz[g.n0 + c], cnt);
+            uint32_t sum = cnt;
+#pragma unroll
+            for (int s = 16; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
+            if (lane == 0 && sum) {
+              atomicAdd(&o.tile_nnz[(g.n0 + c) >> 6], sum);
+              atomicAdd(o.nnz, (unsigned long long)sum);
+            }
+          }
+        }
+      }
+      named_bar_sync(2, 128);  // s_scale / s_cnt / staging reuse by the next tile
     }
+    if (acc_smem) {
+      // flush the CTA's column counts: per column, per 64-column tile, total
+      named_bar_sync(2, 128);
+      const OccDev& o = P.out_occ;
+      unsigned long long total = 0ull;
+      for (int c0 = 0; c0 < p.N; c0 += 128) {
+        const int c = c0 + et;
+        const uint32_t cnt = c < p.N ? s_acc[c] : 0u;
+        if (cnt) atomicAdd(&o.col_nnz[c], cnt);
+        uint32_t sum = cnt;
+#pragma unroll
+        for (int s = 16; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
+        total += sum;
+        if (lane == 0 && sum) atomicAdd(&o.tile_nnz[c >> 6], sum);
+      }
+      if (lane == 0 && total) atomicAdd(o.nnz, total);
+    }
+    if (et == 0) bulk_wait_all();
   }
 
   tc_fence_before();
   __syncthreads();
   if (warp == 8) {
     tc_fence_after();
-    tmem_dealloc(tmem, (uint32_t)BN);
+    tmem_dealloc(tmem, (uint32_t)(2 * BN));
   }
 }
 
@@ -396,58 +656,138 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return fn;
 }
 
-// 2-D bf16 tensor [rows, cols] (cols contiguous), box {32, box_rows}, 64-byte swizzle.
-bool make_tmap(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+CUtensorMapSwizzle swz_of(int inner_bytes) {
+  return inner_bytes == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+}
+
+// 2-D bf16 tensor [rows, cols] (cols contiguous), box {box_cols, box_rows}.
+bool make_tmap_2d(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_cols,
+                  uint32_t box_rows) {
   auto enc = get_encode();
   if (!enc) return false;
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {cols * 2};
-  cuuint32_t box[2] = {32, box_rows};
+  cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
-                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz_of((int)box_cols * 2),
                    CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
 
-template <int BN>
-cudaError_t launch_bn(const IgemmArgs& a, const CUtensorMap& tA, const CUtensorMap& tB,
-                      cudaStream_t s) {
+// 4-D NHWC bf16 tensor [n, h, w, c], box {box_c, bw, bh, bn} traversed with
+// element strides {1, stride, stride, 1}.
+bool make_tmap_nhwc(CUtensorMap* m, const void* base, int n, int h, int w, int c, int box_c, int bw,
+                    int bh, int bn, int stride) {
+  auto enc = get_encode();
+  if (!enc) return false;
+  cuuint64_t dims[4] = {(cuuint64_t)c, (cuuint64_t)w, (cuuint64_t)h, (cuuint64_t)n};
+  cuuint64_t strides[3] = {(cuuint64_t)c * 2, (cuuint64_t)w * c * 2, (cuuint64_t)h * w * c * 2};
+  cuuint32_t box[4] = {(cuuint32_t)box_c, (cuuint32_t)(bw * stride), (cuuint32_t)(bh * stride),
+                       (cuuint32_t)bn};
+  cuuint32_t estr[4] = {1, (cuuint32_t)stride, (cuuint32_t)stride, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides,
+                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz_of(box_c * 2),
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+int num_sms() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 148;
+  }
+  return n;
+}
+
+template <int BN, int BK>
+cudaError_t launch_cfg(const IgemmArgs& a, const CUtensorMap& tA, const CUtensorMap& tB,
+                       const CUtensorMap& tY, int64_t tiles, cudaStream_t s) {
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(igemm_kernel<BN>,
+    cudaError_t e = cudaFuncSetAttribute(igemm_kernel<BN, BK>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         Cfg<BN>::kSmem);
+                                         Cfg<BN, BK>::kSmem);
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  dim3 grid((a.M + kBM - 1) / kBM, (a.N + BN - 1) / BN);
-  igemm_kernel<BN><<<grid, kThreads, Cfg<BN>::kSmem, s>>>(tA, tB, a);
+  const int64_t grid = tiles < num_sms() ? tiles : num_sms();
+  igemm_kernel<BN, BK><<<(unsigned)grid, kThreads, Cfg<BN, BK>::kSmem, s>>>(tA, tB, tY, a);
   return cudaGetLastError();
 }
 
 }  // namespace
 
+void choose_spatial_tile(IgemmArgs& a) {
+  int64_t best = -1;
+  for (int bw = 1; bw <= 128; bw *= 2) {
+    if (bw * a.stride > 256) break;
+    for (int bh = 1; bw * bh <= 128; bh *= 2) {
+      if (bh * a.stride > 256) break;
+      const int bn = 128 / (bw * bh);
+      const int64_t tw = (a.Wo + bw - 1) / bw, th = (a.Ho + bh - 1) / bh,
+                    tn = (a.Nimg + bn - 1) / bn;
+      const int64_t cost = tw * bw * th * bh * tn * bn;
+      // fewest padded pixels; then the widest (most contiguous) box
+      if (best < 0 || cost < best || (cost == best && bw > a.bw)) {
+        best = cost;
+        a.bw = bw;
+        a.bh = bh;
+        a.bn = bn;
+        a.tw = (int)tw;
+        a.th = (int)th;
+      }
+    }
+  }
+}
+
 cudaError_t launch_igemm(const IgemmArgs& a, cudaStream_t s) {
   if (a.M <= 0 || a.N <= 0) return cudaSuccess;
-  const int mt = (a.M + kBM - 1) / kBM;
+  if (a.conv == 2 && (a.Cp % 32 != 0 || a.bw * a.bh * a.bn != 128)) return cudaErrorInvalidValue;
+  const int64_t mtiles =
+      a.conv == 2 ? (int64_t)((a.Nimg + a.bn - 1) / a.bn) * a.th * a.tw : (a.M + kBM - 1) / kBM;
   int bn = 64;
   if (a.N > 64) {
     bn = 256;
-    while (bn > 64 && (bn / 2 >= a.N || (int64_t)mt * ((a.N + bn - 1) / bn) < 148)) bn /= 2;
+    while (bn > 64 && (bn / 2 >= a.N || mtiles * ((a.N + bn - 1) / bn) < num_sms())) bn /= 2;
   }
-  CUtensorMap tA, tB;
+  // K block: 64 (128-byte swizzle) when the channel layout allows it and the
+  // stage ring still holds at least four stages; 32 otherwise
+  const int bk = (bn < 256 && (a.conv == 2 ? (a.Cp % 64 == 0) : (a.Ktot > 32))) ? 64 : 32;
+  CUtensorMap tA, tB, tY;
   memset(&tA, 0, sizeof(tA));
-  if (!a.conv) {
-    if (!make_tmap(&tA, a.x, (uint64_t)a.M, (uint64_t)a.Ktot, kBM)) return cudaErrorInvalidValue;
+  memset(&tY, 0, sizeof(tY));
+  if (a.conv == 0) {
+    if (!make_tmap_2d(&tA, a.x, (uint64_t)a.M, (uint64_t)a.Ktot, (uint32_t)bk, kBM))
+      return cudaErrorInvalidValue;
+  } else if (a.conv == 2) {
+    if (!make_tmap_nhwc(&tA, a.x, a.Nimg, a.H, a.W, a.Cp, bk, a.bw, a.bh, a.bn, a.stride))
+      return cudaErrorInvalidValue;
   }
-  if (!make_tmap(&tB, a.w, (uint64_t)a.N, (uint64_t)a.Ktot, (uint32_t)bn))
+  if (!make_tmap_2d(&tB, a.w, (uint64_t)a.N, (uint64_t)a.Ktot, (uint32_t)bk, (uint32_t)bn))
     return cudaErrorInvalidValue;
-  if (a.conv) tA = tB;  // unused by the gather producers
+  if (!a.y_f32) {
+    bool okY = a.conv == 2
+                   ? make_tmap_nhwc(&tY, a.y, a.Nimg, a.Ho, a.Wo, a.N, 64, a.bw, a.bh, a.bn, 1)
+                   : make_tmap_2d(&tY, a.y, (uint64_t)a.M, (uint64_t)a.N, 64, kBM);
+    if (!okY) return cudaErrorInvalidValue;
+  }
+  if (a.conv == 1) tA = tB;  // unused by the gather producers
+  const int64_t tiles = mtiles * ((a.N + bn - 1) / bn);
+  if (bk == 64) {
+    switch (bn) {
+      case 64: return launch_cfg<64, 64>(a, tA, tB, tY, tiles, s);
+      case 128: return launch_cfg<128, 64>(a, tA, tB, tY, tiles, s);
+      default: return launch_cfg<256, 64>(a, tA, tB, tY, tiles, s);
+    }
+  }
   switch (bn) {
-    case 64: return launch_bn<64>(a, tA, tB, s);
-    case 128: return launch_bn<128>(a, tA, tB, s);
-    default: return launch_bn<256>(a, tA, tB, s);
+    case 64: return launch_cfg<64, 32>(a, tA, tB, tY, tiles, s);
+    case 128: return launch_cfg<128, 32>(a, tA, tB, tY, tiles, s);
+    default: return launch_cfg<256, 32>(a, tA, tB, tY, tiles, s);
   }
 }
 

@@ -50,51 +50,137 @@ __device__ __forceinline__ uint4 pack8(const float (&f)[8]) {
   return u;
 }
 
-// Combine the 8-bit masks of the 8 lanes that share a row into the row's
-// 64-bit tile word and store it (lane with t%8 == 0).
-__device__ __forceinline__ void put_row_bits(uint64_t* s_nz, int row, uint32_t mask8) {
-  const int cg = threadIdx.x & 7;
-  uint32_t lo = cg < 4 ? (mask8 << (8 * cg)) : 0u;
-  uint32_t hi = cg >= 4 ? (mask8 << (8 * (cg - 4))) : 0u;
+// Occupancy of the 128-row x 64-column tiles a CTA produces.  Each thread
+// holds an 8-bit non-zero mask per row it owns (lanes 8k..8k+7 of a warp share
+// a row).  row() sets the row's bit in the row bitmap and counts columns in
+// registers; tile_done() writes the tile's block-column mask words and adds
+// its column counts to the CTA's shared counters s_acc[C]; cta_done() flushes
+// those counters once (column, 64-column tile and total counts), so the
+// atomics on one address number one per CTA, not one per tile.  Tensors wider
+// than kMaxAccCols columns flush per tile instead.
+constexpr int kMaxAccCols = 4096;
+
+struct TileEmit {
+  uint32_t cnt[8];
+  __device__ __forceinline__ void init() {
 #pragma unroll
-  for (int s = 1; s < 8; s <<= 1) {
-    lo |= __shfl_xor_sync(0xffffffffu, lo, s);
-    hi |= __shfl_xor_sync(0xffffffffu, hi, s);
+    for (int j = 0; j < 8; ++j) cnt[j] = 0u;
   }
-  if (cg == 0) s_nz[row] = (uint64_t)lo | ((uint64_t)hi << 32);
+  // Every thread of the CTA calls this with its mask (0 outside the tensor).
+  __device__ __forceinline__ void row(uint32_t mask, int64_t grow, int col0, const OccDev& o) {
+    const int lane = threadIdx.x & 31;
+    const uint32_t b = __ballot_sync(0xffffffffu, mask != 0u);
+    if ((lane & 7) == 0 && ((b >> lane) & 0xFFu) != 0u)
+      atomicOr(&o.row_bm[grow * o.W64 + (col0 >> 12)], 1ull << ((col0 >> 6) & 63));
+#pragma unroll
+    for (int j = 0; j < 8; ++j) cnt[j] += (mask >> j) & 1u;
+  }
+  // All threads; s_cnt holds 8 warps x 64 columns.
+  __device__ __forceinline__ void tile_done(int64_t row0, int col0, const OccDev& o,
+                                            uint32_t* s_cnt, uint32_t* s_acc, bool acc) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, cg = threadIdx.x & 7;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      cnt[j] += __shfl_xor_sync(0xffffffffu, cnt[j], 8);
+      cnt[j] += __shfl_xor_sync(0xffffffffu, cnt[j], 16);
+    }
+    if (lane < 8) {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) s_cnt[warp * 64 + cg * 8 + j] = cnt[j];
+    }
+    __syncthreads();
+    if (threadIdx.x < 64) {
+      uint32_t c = 0;
+#pragma unroll
+      for (int w = 0; w < kTileThreads / 32; ++w) c += s_cnt[w * 64 + threadIdx.x];
+      const int col = col0 + threadIdx.x;
+      const uint32_t word = __ballot_sync(0xffffffffu, c != 0u);
+      const int w = (col0 >> 5) + (threadIdx.x >> 5);
+      if (lane == 0 && word && w < o.C32) atomicOr(&o.blk_mask[(row0 >> 7) * o.C32 + w], word);
+      if (acc) {
+        if (col < o.C) s_acc[col] += c;
+      } else {
+        if (c && col < o.C) atomicAdd(&o.col_nnz[col], c);
+        uint32_t sum = c;
+#pragma unroll
+        for (int s = 16; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
+        if (lane == 0 && sum) {
+          atomicAdd(&o.tile_nnz[col0 >> 6], sum);
+          atomicAdd(o.nnz, (unsigned long long)sum);
+        }
+      }
+    }
+    __syncthreads();
+    init();
+  }
+};
+
+__device__ __forceinline__ void acc_init(uint32_t* s_acc, int C, bool acc) {
+  if (acc)
+    for (int c = threadIdx.x; c < C; c += kTileThreads) s_acc[c] = 0u;
+  __syncthreads();
 }
 
-__device__ __forceinline__ void zero_rows(uint64_t* s_nz) {
-  if (threadIdx.x < 128) s_nz[threadIdx.x] = 0ull;
+__device__ __forceinline__ void cta_done(const OccDev& o, const uint32_t* s_acc, bool acc) {
+  if (!acc) return;
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  unsigned long long total = 0ull;
+  for (int c0 = 0; c0 < o.C; c0 += kTileThreads) {
+    const int c = c0 + threadIdx.x;
+    const uint32_t cnt = c < o.C ? s_acc[c] : 0u;
+    if (cnt) atomicAdd(&o.col_nnz[c], cnt);
+    uint32_t sum = cnt;
+#pragma unroll
+    for (int s = 16; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
+    total += sum;
+    if (lane == 0 && sum) atomicAdd(&o.tile_nnz[c >> 6], sum);
+  }
+  if (lane == 0 && total) atomicAdd(o.nnz, total);
 }
+
+// Tiles of a [R, C] output: rt = t / ct_count row tile, ct = t % ct_count column tile.
+#define SPAROA_TILE_LOOP(R, C)                                                   \
+  const int ctn = ((C) + 63) / 64;                                               \
+  const int64_t ntiles = (((R) + 127) / 128) * (int64_t)ctn;                     \
+  for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
 
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kTileThreads) stats_kernel(const __nv_bfloat16* __restrict__ x,
-                                                             int64_t R, int C, OccDev o) {
-  __shared__ uint64_t s_nz[128];
+                                                             int64_t R, int C, OccDev o_param) {
+  const OccDev o = o_param;  // registers, not parameter-space loads
+  __shared__ uint32_t s_cnt[8 * 64];
+  __shared__ uint32_t s_acc[kMaxAccCols];
+  const bool acc = C <= kMaxAccCols;
   const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
-  const int64_t row0 = (int64_t)blockIdx.x * 128;
-  const int c0 = blockIdx.y * 64 + cg * 8;
   const bool vec = (C & 7) == 0;
-  uint32_t m[4];
+  acc_init(s_acc, C, acc);
+  TileEmit e;
+  e.init();
+  SPAROA_TILE_LOOP(R, C) {
+    const int64_t row0 = (tile / ctn) * 128;
+    const int col0 = (int)(tile % ctn) * 64;
+    const int c0 = col0 + cg * 8;
+    uint32_t m[4];
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int64_t r = row0 + rs + 32 * i;
-    m[i] = 0;
-    if (r < R && c0 < C) {
-      const __nv_bfloat16* p = x + r * C + c0;
-      if (vec) {
-        m[i] = nz_mask8(__ldg(reinterpret_cast<const uint4*>(p)));
-      } else {
-        for (int j = 0; j < 8 && c0 + j < C; ++j)
-          if (bf16_nz(__bfloat16_as_ushort(p[j]))) m[i] |= 1u << j;
+    for (int i = 0; i < 4; ++i) {
+      const int64_t r = row0 + rs + 32 * i;
+      m[i] = 0;
+      if (r < R && c0 < C) {
+        const __nv_bfloat16* p = x + r * C + c0;
+        if (vec) {
+          m[i] = nz_mask8(__ldg(reinterpret_cast<const uint4*>(p)));
+        } else {
+          for (int j = 0; j < 8 && c0 + j < C; ++j)
+            if (bf16_nz(__bfloat16_as_ushort(p[j]))) m[i] |= 1u << j;
+        }
       }
     }
-  }
 #pragma unroll
-  for (int i = 0; i < 4; ++i) put_row_bits(s_nz, rs + 32 * i, m[i]);
-  __syncthreads();
-  flush_tile(s_nz, row0, blockIdx.y * 64, o, threadIdx.x, kTileThreads);
+    for (int i = 0; i < 4; ++i) e.row(m[i], row0 + rs + 32 * i, col0, o);
+    e.tile_done(row0, col0, o, s_cnt, s_acc, acc);
+  }
+  cta_done(o, s_acc, acc);
 }
 
 // ---------------------------------------------------------------------------
@@ -108,190 +194,237 @@ __global__ void pad_kernel(const __nv_bfloat16* __restrict__ x, int64_t P, int C
 }
 
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kTileThreads) dwconv_kernel(const DwArgs a) {
-  __shared__ uint64_t s_nz[128];
-  zero_rows(s_nz);
+// Depthwise 3x3 convolution (stride 1 or 2, any padding) + epilogue.
+__global__ void __launch_bounds__(kTileThreads) dwconv_kernel(const DwArgs a_param) {
+  const DwArgs a = a_param;  // registers, not parameter-space loads
+  __shared__ uint32_t s_cnt[8 * 64];
+  __shared__ uint32_t s_acc[kMaxAccCols];
+  __shared__ __align__(16) float s_w[9][64];
   const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
-  const int64_t row0 = (int64_t)blockIdx.x * 128;
-  const int c0 = blockIdx.y * 64 + cg * 8;
   const int64_t R = (int64_t)a.N * a.Ho * a.Wo;
-  const int taps = a.kh * a.kw;
-  if (a.path_out && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *a.path_out = 3;
-  __syncthreads();
-  const bool cvalid = c0 < a.C;
-  float wr[9][8];
+  const bool acc = a.emit && a.C <= kMaxAccCols;
+  if (a.path_out && blockIdx.x == 0 && threadIdx.x == 0) *a.path_out = 3;
+  acc_init(s_acc, a.C, acc);
+  TileEmit e;
+  e.init();
+  const int hw = a.Ho * a.Wo;
+  int cur_col0 = -1;
   float sc[8], sh[8];
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    sc[j] = 1.f;
-    sh[j] = 0.f;
-    if (cvalid) epi_affine(a.ep, a.C, c0 + j, sc[j], sh[j]);
-#pragma unroll
-    for (int t = 0; t < 9; ++t)
-      wr[t][j] = (cvalid && t < taps) ? __bfloat162float(a.w[(int64_t)(c0 + j) * taps + t]) : 0.f;
-  }
-  for (int i = 0; i < 4; ++i) {
-    const int row = rs + 32 * i;
-    const int64_t mrow = row0 + row;
-    uint32_t mask = 0;
-    if (cvalid && mrow < R) {
-      const int hw = a.Ho * a.Wo;
-      const int img = (int)(mrow / hw);
-      const int rem = (int)(mrow - (int64_t)img * hw);
-      const int oh = rem / a.Wo, ow = rem - (rem / a.Wo) * a.Wo;
-      float acc[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) acc[j] = 0.f;
-      for (int r = 0; r < a.kh; ++r) {
-        const int ih = oh * a.stride - a.pad + r;
-        if (ih < 0 || ih >= a.H) continue;
-        for (int s = 0; s < a.kw; ++s) {
-          const int iw = ow * a.stride - a.pad + s;
-          if (iw < 0 || iw >= a.W) continue;
-          const uint4 u = __ldg(reinterpret_cast<const uint4*>(
-              a.x + (((int64_t)img * a.H + ih) * a.W + iw) * a.C + c0));
-          float f[8];
-          unpack8(u, f);
-          const int t = r * a.kw + s;
-#pragma unroll
-          for (int j = 0; j < 8; ++j) acc[j] = fmaf(f[j], wr[t][j], acc[j]);
-        }
+  SPAROA_TILE_LOOP(R, a.C) {
+    const int64_t row0 = (tile / ctn) * 128;
+    const int col0 = (int)(tile % ctn) * 64;
+    const int c0 = col0 + cg * 8;
+    const bool cvalid = c0 < a.C;
+    if (col0 != cur_col0) {  // (uniform) new channel slice: weights and affine
+      __syncthreads();
+      for (int idx = threadIdx.x; idx < 9 * 64; idx += kTileThreads) {
+        const int t = idx / 64, c = idx % 64;
+        s_w[t][c] = (col0 + c < a.C) ? __bfloat162float(a.w[(int64_t)(col0 + c) * 9 + t]) : 0.f;
       }
-      float rv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      if (a.ep.residual) unpack8(*reinterpret_cast<const uint4*>(a.ep.residual + mrow * a.C + c0), rv);
-      float o[8];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) o[j] = epi_act(fmaf(acc[j], sc[j], sh[j]) + rv[j], a.ep.act);
-      const uint4 u = pack8(o);
-      *reinterpret_cast<uint4*>(a.y + mrow * a.C + c0) = u;
-      mask = nz_mask8(u);
+      for (int j = 0; j < 8; ++j) {
+        sc[j] = 1.f;
+        sh[j] = 0.f;
+        if (cvalid) epi_affine(a.ep, a.C, c0 + j, sc[j], sh[j]);
+      }
+      __syncthreads();
+      cur_col0 = col0;
     }
-    if (a.emit) put_row_bits(s_nz, row, mask);
+    for (int i = 0; i < 4; ++i) {
+      const int64_t mrow = row0 + rs + 32 * i;
+      uint32_t mask = 0;
+      if (cvalid && mrow < R) {
+        const int img = (int)(mrow / hw);
+        const int rem = (int)(mrow - (int64_t)img * hw);
+        const int oh = rem / a.Wo, ow = rem - (rem / a.Wo) * a.Wo;
+        const __nv_bfloat16* xi = a.x + (int64_t)img * a.H * a.W * a.C + c0;
+        float accv[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) accv[j] = 0.f;
+#pragma unroll
+        for (int r = 0; r < 3; ++r) {
+          const int ih = oh * a.stride - a.pad + r;
+#pragma unroll
+          for (int s = 0; s < 3; ++s) {
+            const int iw = ow * a.stride - a.pad + s;
+            if (ih >= 0 && ih < a.H && iw >= 0 && iw < a.W) {
+              float f[8];
+              unpack8(__ldg(reinterpret_cast<const uint4*>(xi + ((int64_t)ih * a.W + iw) * a.C)), f);
+              const float4 w0 = *reinterpret_cast<const float4*>(&s_w[r * 3 + s][cg * 8]);
+              const float4 w1 = *reinterpret_cast<const float4*>(&s_w[r * 3 + s][cg * 8 + 4]);
+              const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+#pragma unroll
+              for (int j = 0; j < 8; ++j) accv[j] = fmaf(f[j], wv[j], accv[j]);
+            }
+          }
+        }
+        float rv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        if (a.ep.residual) unpack8(*reinterpret_cast<const uint4*>(a.ep.residual + mrow * a.C + c0), rv);
+        float o[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) o[j] = epi_act(fmaf(accv[j], sc[j], sh[j]) + rv[j], a.ep.act);
+        const uint4 u = pack8(o);
+        *reinterpret_cast<uint4*>(a.y + mrow * a.C + c0) = u;
+        mask = nz_mask8(u);
+      }
+      if (a.emit) e.row(mask, mrow, col0, a.out_occ);
+    }
+    if (a.emit) e.tile_done(row0, col0, a.out_occ, s_cnt, s_acc, acc);
   }
-  if (a.emit) {
-    __syncthreads();
-    flush_tile(s_nz, row0, blockIdx.y * 64, a.out_occ, threadIdx.x, kTileThreads);
-  }
+  if (a.emit) cta_done(a.out_occ, s_acc, acc);
 }
 
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kTileThreads)
     maxpool_kernel(const __nv_bfloat16* __restrict__ x, int N, int H, int W, int C, int k,
-                   int stride, int pad, int Ho, int Wo, __nv_bfloat16* __restrict__ y, OccDev o,
+                   int stride, int pad, int Ho, int Wo, __nv_bfloat16* __restrict__ y, OccDev o_param,
                    int emit) {
-  __shared__ uint64_t s_nz[128];
+  const OccDev o = o_param;
+  __shared__ uint32_t s_cnt[8 * 64];
+  __shared__ uint32_t s_acc[kMaxAccCols];
   const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
-  const int64_t row0 = (int64_t)blockIdx.x * 128;
-  const int c0 = blockIdx.y * 64 + cg * 8;
   const int64_t R = (int64_t)N * Ho * Wo;
-  for (int i = 0; i < 4; ++i) {
-    const int row = rs + 32 * i;
-    const int64_t mrow = row0 + row;
-    uint32_t mask = 0;
-    if (mrow < R && c0 < C) {
-      const int hw = Ho * Wo;
-      const int img = (int)(mrow / hw);
-      const int rem = (int)(mrow - (int64_t)img * hw);
-      const int oh = rem / Wo, ow = rem - (rem / Wo) * Wo;
-      float mx[8];
+  const bool acc = emit && C <= kMaxAccCols;
+  acc_init(s_acc, C, acc);
+  TileEmit e;
+  e.init();
+  SPAROA_TILE_LOOP(R, C) {
+    const int64_t row0 = (tile / ctn) * 128;
+    const int col0 = (int)(tile % ctn) * 64;
+    const int c0 = col0 + cg * 8;
+    for (int i = 0; i < 4; ++i) {
+      const int64_t mrow = row0 + rs + 32 * i;
+      uint32_t mask = 0;
+      if (mrow < R && c0 < C) {
+        const int hw = Ho * Wo;
+        const int img = (int)(mrow / hw);
+        const int rem = (int)(mrow - (int64_t)img * hw);
+        const int oh = rem / Wo, ow = rem - (rem / Wo) * Wo;
+        float mx[8];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) mx[j] = -INFINITY;
-      for (int r = 0; r < k; ++r) {
-        const int ih = oh * stride - pad + r;
-        if (ih < 0 || ih >= H) continue;
-        for (int s = 0; s < k; ++s) {
-          const int iw = ow * stride - pad + s;
-          if (iw < 0 || iw >= W) continue;
-          float f[8];
-          unpack8(__ldg(reinterpret_cast<const uint4*>(x + (((int64_t)img * H + ih) * W + iw) * C + c0)), f);
+        for (int j = 0; j < 8; ++j) mx[j] = -INFINITY;
+        for (int r = 0; r < k; ++r) {
+          const int ih = oh * stride - pad + r;
+          if (ih < 0 || ih >= H) continue;
+          for (int s = 0; s < k; ++s) {
+            const int iw = ow * stride - pad + s;
+            if (iw < 0 || iw >= W) continue;
+            float f[8];
+            unpack8(__ldg(reinterpret_cast<const uint4*>(x + (((int64_t)img * H + ih) * W + iw) * C + c0)), f);
 #pragma unroll
-          for (int j = 0; j < 8; ++j)
-            if (f[j] > mx[j]) mx[j] = f[j];
+            for (int j = 0; j < 8; ++j)
+              if (f[j] > mx[j]) mx[j] = f[j];
+          }
         }
+        const uint4 u = pack8(mx);
+        *reinterpret_cast<uint4*>(y + mrow * C + c0) = u;
+        mask = nz_mask8(u);
       }
-      const uint4 u = pack8(mx);
-      *reinterpret_cast<uint4*>(y + mrow * C + c0) = u;
-      mask = nz_mask8(u);
+      if (emit) e.row(mask, mrow, col0, o);
     }
-    if (emit) put_row_bits(s_nz, row, mask);
+    if (emit) e.tile_done(row0, col0, o, s_cnt, s_acc, acc);
   }
-  if (emit) {
-    __syncthreads();
-    flush_tile(s_nz, row0, blockIdx.y * 64, o, threadIdx.x, kTileThreads);
-  }
+  if (emit) cta_done(o, s_acc, acc);
 }
 
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kTileThreads)
     avgpool_kernel(const __nv_bfloat16* __restrict__ x, int N, int HW, int C,
-                   __nv_bfloat16* __restrict__ y, OccDev o, int emit) {
-  __shared__ uint64_t s_nz[128];
+                   __nv_bfloat16* __restrict__ y, OccDev o_param, int emit) {
+  const OccDev o = o_param;
+  __shared__ uint32_t s_cnt[8 * 64];
+  __shared__ uint32_t s_acc[kMaxAccCols];
   const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
-  const int64_t row0 = (int64_t)blockIdx.x * 128;
-  const int c0 = blockIdx.y * 64 + cg * 8;
-  for (int i = 0; i < 4; ++i) {
-    const int row = rs + 32 * i;
-    const int64_t n = row0 + row;
-    uint32_t mask = 0;
-    if (n < N && c0 < C) {
-      float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      const __nv_bfloat16* p = x + n * (int64_t)HW * C + c0;
-      for (int q = 0; q < HW; ++q) {
-        float f[8];
-        unpack8(__ldg(reinterpret_cast<const uint4*>(p + (int64_t)q * C)), f);
+  const bool acc = emit && C <= kMaxAccCols;
+  acc_init(s_acc, C, acc);
+  TileEmit e;
+  e.init();
+  SPAROA_TILE_LOOP((int64_t)N, C) {
+    const int64_t row0 = (tile / ctn) * 128;
+    const int col0 = (int)(tile % ctn) * 64;
+    const int c0 = col0 + cg * 8;
+    for (int i = 0; i < 4; ++i) {
+      const int64_t n = row0 + rs + 32 * i;
+      uint32_t mask = 0;
+      if (n < N && c0 < C) {
+        float a8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        const __nv_bfloat16* p = x + n * (int64_t)HW * C + c0;
+        for (int q = 0; q < HW; ++q) {
+          float f[8];
+          unpack8(__ldg(reinterpret_cast<const uint4*>(p + (int64_t)q * C)), f);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) acc[j] += f[j];
+          for (int j = 0; j < 8; ++j) a8[j] += f[j];
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) a8[j] = a8[j] / (float)HW;
+        const uint4 u = pack8(a8);
+        *reinterpret_cast<uint4*>(y + n * C + c0) = u;
+        mask = nz_mask8(u);
       }
-#pragma unroll
-      for (int j = 0; j < 8; ++j) acc[j] = acc[j] / (float)HW;
-      const uint4 u = pack8(acc);
-      *reinterpret_cast<uint4*>(y + n * C + c0) = u;
-      mask = nz_mask8(u);
+      if (emit) e.row(mask, n, col0, o);
     }
-    if (emit) put_row_bits(s_nz, row, mask);
+    if (emit) e.tile_done(row0, col0, o, s_cnt, s_acc, acc);
   }
-  if (emit) {
-    __syncthreads();
-    flush_tile(s_nz, row0, blockIdx.y * 64, o, threadIdx.x, kTileThreads);
-  }
+  if (emit) cta_done(o, s_acc, acc);
 }
 
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kTileThreads)
-    bn_act_kernel(const __nv_bfloat16* __restrict__ x, int64_t R, int C, EpiDev ep,
-                  __nv_bfloat16* __restrict__ y, OccDev o, int emit) {
-  __shared__ uint64_t s_nz[128];
+    bn_act_kernel(const __nv_bfloat16* __restrict__ x, int64_t R, int C, EpiDev ep_param,
+                  __nv_bfloat16* __restrict__ y, OccDev o_param, int emit) {
+  const OccDev o = o_param;
+  const EpiDev ep = ep_param;
+  __shared__ uint32_t s_cnt[8 * 64];
+  __shared__ uint32_t s_acc[kMaxAccCols];
   const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
-  const int64_t row0 = (int64_t)blockIdx.x * 128;
-  const int c0 = blockIdx.y * 64 + cg * 8;
-  float sc[8], sh[8];
-  if (c0 < C) {
+  const bool acc = emit && C <= kMaxAccCols;
+  acc_init(s_acc, C, acc);
+  TileEmit e;
+  e.init();
+  SPAROA_TILE_LOOP(R, C) {
+    const int64_t row0 = (tile / ctn) * 128;
+    const int col0 = (int)(tile % ctn) * 64;
+    const int c0 = col0 + cg * 8;
+    float sc[8], sh[8];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) epi_affine(ep, C, c0 + j, sc[j], sh[j]);
-  }
-  for (int i = 0; i < 4; ++i) {
-    const int row = rs + 32 * i;
-    const int64_t r = row0 + row;
-    uint32_t mask = 0;
-    if (r < R && c0 < C) {
-      float f[8], rv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      unpack8(__ldg(reinterpret_cast<const uint4*>(x + r * C + c0)), f);
-      if (ep.residual) unpack8(*reinterpret_cast<const uint4*>(ep.residual + r * C + c0), rv);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) f[j] = epi_act(fmaf(f[j], sc[j], sh[j]) + rv[j], ep.act);
-      const uint4 u = pack8(f);
-      *reinterpret_cast<uint4*>(y + r * C + c0) = u;
-      mask = nz_mask8(u);
+    for (int j = 0; j < 8; ++j) {
+      sc[j] = 1.f;
+      sh[j] = 0.f;
+      if (c0 < C) epi_affine(ep, C, c0 + j, sc[j], sh[j]);
     }
-    if (emit) put_row_bits(s_nz, row, mask);
+    for (int i = 0; i < 4; ++i) {
+      const int64_t r = row0 + rs + 32 * i;
+      uint32_t mask = 0;
+      if (r < R && c0 < C) {
+        float f[8], rv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        unpack8(__ldg(reinterpret_cast<const uint4*>(x + r * C + c0)), f);
+        if (ep.residual) unpack8(*reinterpret_cast<const uint4*>(ep.residual + r * C + c0), rv);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) f[j] = epi_act(fmaf(f[j], sc[j], sh[j]) + rv[j], ep.act);
+        const uint4 u = pack8(f);
+        *reinterpret_cast<uint4*>(y + r * C + c0) = u;
+        mask = nz_mask8(u);
+      }
+      if (emit) e.row(mask, r, col0, o);
+    }
+    if (emit) e.tile_done(row0, col0, o, s_cnt, s_acc, acc);
   }
-  if (emit) {
-    __syncthreads();
-    flush_tile(s_nz, row0, blockIdx.y * 64, o, threadIdx.x, kTileThreads);
-  }
+  if (emit) cta_done(o, s_acc, acc);
 }
 
-dim3 tile_grid(int64_t R, int C) { return dim3((unsigned)((R + 127) / 128), (unsigned)((C + 63) / 64)); }
+// Grid-stride over 128 x 64 tiles with at most 4 CTAs per SM.
+unsigned tile_grid(int64_t R, int C) {
+  static int sms = 0;
+  if (!sms) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
+      sms = 148;
+  }
+  const int64_t tiles = ((R + 127) / 128) * ((C + 63) / 64);
+  const int64_t cap = 4LL * sms;
+  return (unsigned)(tiles < cap ? tiles : cap);
+}
 
 }  // namespace
 

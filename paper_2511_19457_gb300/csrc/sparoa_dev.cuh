@@ -17,7 +17,8 @@
 
 namespace sparoa {
 
-constexpr uint64_t kWaitLimitNs = 1000ull * 1000ull * 1000ull;  // 1 s
+// Bounded waits give up after about a second of SM clock cycles.
+constexpr long long kWaitLimitCycles = 1ll << 31;
 
 enum ErrBits : uint32_t {
   kErrTimeoutFull = 1u,
@@ -109,20 +110,39 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Wait for the phase with the given parity to complete.  Gives up after
-// kWaitLimitNs, or as soon as another role of the CTA raised *abort; then it
-// records `bit` in *err, raises *abort and returns false.
+// try_wait that suspends the thread in hardware until the phase completes or
+// about `hint_ns` nanoseconds pass, so waiting warps leave the issue slots to
+// the warps doing work on the same scheduler.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+
+// Wait for the phase with the given parity to complete.  Waiting threads are
+// suspended by the hardware between polls (woken when the phase completes);
+// the cycle counter and the CTA abort flag are checked every 16 polls.  Gives up after kWaitLimitCycles
+// or once another role of the CTA raised *abort; then it records `bit` in
+// *err, raises *abort and returns false.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t* err,
                                           volatile int* abort, uint32_t bit) {
   if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer_ns();
-  while (true) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if (*abort) return false;
-    if (globaltimer_ns() - t0 > kWaitLimitNs) {
-      atomicOr(err, bit);
-      *abort = 1;
-      return false;
+  const long long t0 = clock64();
+  for (uint32_t n = 1;; ++n) {
+    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+    if ((n & 15u) == 0u) {
+      if (*abort) return false;
+      if (clock64() - t0 > kWaitLimitCycles) {
+        atomicOr(err, bit);
+        *abort = 1;
+        return false;
+      }
     }
   }
 }
@@ -137,6 +157,33 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, uint
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(bar)
       : "memory");
+}
+
+// Shared -> global tensor stores (bulk-group completion).
+__device__ __forceinline__ void tma_store_2d(const void* tmap, uint32_t src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(tmap)),
+               "r"(src), "r"(x), "r"(y)
+               : "memory");
+}
+__device__ __forceinline__ void tma_store_4d(const void* tmap, uint32_t src, int c0, int c1, int c2,
+                                             int c3) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.global.shared::cta.bulk_group [%0, {%2, %3, %4, %5}], [%1];" ::"l"(
+          reinterpret_cast<uint64_t>(tmap)),
+      "r"(src), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+      : "memory");
+}
+__device__ __forceinline__ void bulk_commit() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// Wait until at most N committed store groups still read their shared source.
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() {
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 
 __device__ __forceinline__ void prefetch_tmap(const void* tmap) {
@@ -235,6 +282,67 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// Issue a load of 32 consecutive fp32 columns of this thread's TMEM lane;
+// the registers are valid after tmem_wait_ld().
+__device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32"
+      " {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+        "=r"(r[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+// Wait for the loads into r[]; the registers are operands so that no use of
+// them can be scheduled before the wait.
+__device__ __forceinline__ void tmem_wait_ld32(uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.wait::ld.sync.aligned;"
+      : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
+        "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]),
+        "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]),
+        "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]),
+        "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]),
+        "+r"(r[31]));
+}
+
+// Shared-memory vector load / store that stay ordered with the other volatile
+// asm (barriers, fences) but do not make the compiler reload unrelated memory.
+__device__ __forceinline__ float4 lds_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr));
+  return v;
+}
+__device__ __forceinline__ void sts_u4(uint32_t addr, const uint4& v) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z),
+               "r"(v.w));
+}
+
+// 32 x 32 bit-matrix transpose across a warp: lane i holds row i on entry
+// (bit j = element (i, j)) and column i on exit (bit j = element (j, i)).
+// Five butterfly stages exchange ever smaller blocks between lane pairs.
+__device__ __forceinline__ uint32_t warp_transpose32(uint32_t x) {
+  const int lane = threadIdx.x & 31;
+  const uint32_t masks[5] = {0x0000FFFFu, 0x00FF00FFu, 0x0F0F0F0Fu, 0x33333333u, 0x55555555u};
+#pragma unroll
+  for (int k = 0; k < 5; ++k) {
+    const int sft = 16 >> k;
+    const uint32_t m = masks[k];
+    const uint32_t y = __shfl_xor_sync(0xffffffffu, x, sft);
+    x = (lane & sft) ? ((x & ~m) | ((y >> sft) & m)) : ((x & m) | ((y << sft) & ~m));
+  }
+  return x;
+}
+
 // Shared-memory matrix descriptor for a K-major operand tile written with the
 // 64-byte swizzle: rows of 32 bf16 (64 B), 8-row core-matrix groups 512 B apart.
 __device__ __forceinline__ uint64_t smem_desc_sw64(uint32_t addr) {
@@ -245,6 +353,29 @@ __device__ __forceinline__ uint64_t smem_desc_sw64(uint32_t addr) {
   d |= (uint64_t)1 << 46;                        // descriptor version (sm_100 family)
   d |= (uint64_t)4 << 61;                        // layout: 64-byte swizzle
   return d;
+}
+
+// K-major operand tiles with BK bf16 of K per row: BK = 32 uses the 64-byte
+// swizzle (8-row groups 512 B apart), BK = 64 the 128-byte swizzle (1024 B).
+template <int BK>
+__device__ __forceinline__ uint64_t smem_desc_kmajor(uint32_t addr) {
+  static_assert(BK == 32 || BK == 64, "BK");
+  uint64_t d = 0;
+  d |= (uint64_t)((addr >> 4) & 0x3FFF);           // start address
+  d |= (uint64_t)(16 >> 4) << 16;                   // leading byte offset (unused here)
+  d |= (uint64_t)((BK * 2 * 8) >> 4) << 32;         // stride byte offset: 8 rows
+  d |= (uint64_t)1 << 46;                           // descriptor version (sm_100 family)
+  d |= (uint64_t)(BK == 32 ? 4 : 2) << 61;          // layout: 64- or 128-byte swizzle
+  return d;
+}
+
+// Byte offset of 16-byte chunk j of row r in a BK-wide swizzled tile (the
+// layout TMA writes with the matching CU_TENSOR_MAP_SWIZZLE_*): the chunk
+// index is XORed with the row's position inside the swizzle period.
+template <int BK>
+__device__ __forceinline__ uint32_t swz_offset(int r, int j) {
+  if (BK == 32) return (uint32_t)(r * 64 + ((j ^ ((r >> 1) & 3)) << 4));
+  return (uint32_t)(r * 128 + ((j ^ (r & 7)) << 4));
 }
 
 // Instruction descriptor: kind::f16, A = B = bf16, D = fp32, both K-major.

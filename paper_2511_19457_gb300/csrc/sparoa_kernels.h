@@ -18,10 +18,13 @@ struct IgemmArgs {
   int M = 0, N = 0;
   // conv = 0: A = x[M, K] row-major, loaded by TMA.  K = Ktot, K % 8 == 0.
   // conv = 1: A gathered from NHWC x (implicit GEMM over (tap, channel)).
+  // conv = 2: A loaded by 4-D TMA boxes over a spatial output tile (Cp % 32 == 0).
   int conv = 0;
   const __nv_bfloat16* x = nullptr;
-  int H = 1, W = 1, Cp = 0;          // conv input geometry; Cp = channel pitch (% 8 == 0)
+  int Nimg = 1, H = 1, W = 1, Cp = 0;  // conv input geometry; Cp = channel pitch (% 8 == 0)
   int Ho = 1, Wo = 1, kh = 1, kw = 1, stride = 1, pad = 0;
+  int bw = 0, bh = 0, bn = 0;        // conv = 2: output tile of bw x bh pixels in bn images
+  int tw = 0, th = 0;                // conv = 2: tiles along W and H
   int Ktot = 0;                      // GEMM K, or kh*kw*Cp
   const __nv_bfloat16* w = nullptr;  // [N, Ktot] K-major
   EpiDev ep{};
@@ -42,6 +45,9 @@ struct IgemmArgs {
 
 // Picks the N tile, encodes the tensor maps and launches.
 cudaError_t launch_igemm(const IgemmArgs& a, cudaStream_t s);
+
+// conv = 2: the bw x bh x bn (= 128) output tile with the fewest padded pixels.
+void choose_spatial_tile(IgemmArgs& a);
 
 // ----------------------------------------------------------------------------
 // Column-compacting zero-skip FC for few rows (M <= 128 per row block)
