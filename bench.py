@@ -43,7 +43,8 @@ def parse_args():
     p.add_argument("--steps", type=int, default=60000)
     p.add_argument("--warmup", type=int, default=400)
     p.add_argument("--impl", default="sparoa", choices=["sparoa", "reference"])
-    p.add_argument("--workload", default="conv", choices=["conv", "fc", "resnet18", "mobilenet_v2"])
+    p.add_argument("--workload", default="conv",
+                   choices=["conv", "fc", "resnet18", "mobilenet_v2", "mlp_sweep"])
     p.add_argument("--batch", type=int, default=32)
     p.add_argument("--no-cpu-baseline", action="store_true")
     return p.parse_args()
@@ -433,6 +434,101 @@ def conv_occupied_fraction(occ, N, H, W, C, k=3, pad=1):
     return occupied / total if total else 1.0
 
 
+def run_fc(args, rank, local_rank, world, peaks):
+    """Single FC operator [64, 512] x [512, 512]^T (column-sparse ReLU input),
+    fp32 output: stats + dispatch + the chosen kernel, CUDA-graph replays."""
+    import torch
+
+    from paper_2511_19457_gb300 import sparoa as sp
+    from paper_2511_19457_gb300 import synth
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    ctx = sp.Context(local_rank)
+    d = synth.fc_layer(seed=0)
+    M, K, N = d["M"], d["K"], d["N"]
+    nb = NBUF
+    xs = [sp.bits_to_device(d["x"]).view(M, K).clone() for _ in range(nb)]
+    w = sp.bits_to_device(d["w"]).view(N, K)
+    wkn = sp.bits_to_device(d["w_kn"]).view(K, N)
+    bias = torch.from_numpy(d["bias"]).to(dev)
+    ys = [torch.empty(M, N, dtype=torch.float32, device=dev) for _ in range(nb)]
+    xo = [sp.OccupancyBuffer(M, K) for _ in range(nb)]
+
+    def step(j):
+        sp.sparoa_op_stats(ctx, xs[j], (M, K), occ=xo[j], host=False)
+        sp.sparoa_gemm(ctx, xs[j], w, ys[j], W_kn=wkn, bias=bias, x_occ=xo[j])
+
+    st = sp.sparoa_gemm(ctx, xs[0], w, ys[0], W_kn=wkn, bias=bias, host=True)
+    for j in range(max(args.warmup, 3)):
+        step(j % nb)
+    g = graph_of(step, nb)
+    g.replay()
+    reps = max(1, args.steps // nb)
+    ms = time_graph(g, reps) / (reps * nb)
+    ms = max_over_ranks(ms, world, dev)
+    flops = 2 * M * K * N
+    ctx.close()
+    return {"metric": METRIC, "value": flops * world / (ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+            "n_gpus": world, "steps": reps * nb, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic", "config": {"workload": "fc [64,512]x[512,512] fp32 out, column-sparse "
+                                            "ReLU input (rho ~0.7), stats + dispatch",
+                                            "path": "zero-skip" if st.path == sp.PATH_SKIP else "dense",
+                                            "rho": st.sparsity}}
+
+
+def run_mlp_sweep(args, rank, local_rank, world, peaks):
+    """Down projection of a 768 -> 3072 -> 768 ReLU MLP, h [M, 3072] x W2 [768, 3072]^T,
+    at activation sparsity 0..0.95: dense tcgen05 vs zero-skip time per point, the
+    crossover sparsity where zero-skip wins, and what the rule (s_thr 0.5) picks."""
+    import torch
+
+    from paper_2511_19457_gb300 import sparoa as sp
+    from paper_2511_19457_gb300 import synth
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    ctx = sp.Context(local_rank)
+    wts = synth.mlp_weights(seed=0)
+    w2 = sp.bits_to_device(wts["w2"]).view(768, 3072)
+    rhos = [round(0.05 * i, 2) for i in range(20)]
+    table = []
+    cross = {}
+    for M in (256, 1024, 4096):
+        for structure in ("unstructured", "block32"):
+            nb = 4 if M == 4096 else 8
+            y = torch.empty(M, 768, dtype=torch.bfloat16, device=dev)
+            crossover = None
+            for rho in rhos:
+                hs = [sp.bits_to_device(synth.mlp_hidden(M, rho, structure, seed=j)).view(M, 3072)
+                      for j in range(nb)]
+                occ = [sp.OccupancyBuffer(M, 3072) for _ in range(nb)]
+                for j in range(nb):
+                    sp.sparoa_op_stats(ctx, hs[j], (M, 3072), occ=occ[j], host=False)
+                times = {}
+                for force in (1, 2):
+                    thr = sp.thresholds(force_path=force)
+                    g = graph_of(lambda j: sp.sparoa_gemm(ctx, hs[j], w2, y, thr=thr, x_occ=occ[j]), nb)
+                    g.replay()
+                    times[force] = time_graph(g, 10) / (10 * nb)
+                rule = sp.sparoa_gemm(ctx, hs[0], w2, y, x_occ=occ[0], host=True)
+                fl = 2 * M * 3072 * 768
+                row = {"M": M, "structure": structure, "rho": rho, "measured_rho": rule.sparsity,
+                       "dense_us": times[1] * 1e3, "skip_us": times[2] * 1e3,
+                       "dense_tflops": fl / (times[1] * 1e-3) / 1e12,
+                       "skip_eff_tflops": fl / (times[2] * 1e-3) / 1e12,
+                       "rule_path": "zero-skip" if rule.path == sp.PATH_SKIP else "dense"}
+                table.append(row)
+                if crossover is None and times[2] < times[1]:
+                    crossover = rho
+                del hs, occ
+            cross[f"M{M}_{structure}"] = crossover
+    ctx.close()
+    return {"metric": METRIC, "value": None, "unit": "us per down-projection", "n_gpus": world,
+            "higher_is_better": False, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "MLP down projection [M,3072]x[768,3072]^T sparsity sweep"},
+            "crossover_rho": cross, "table": table}
+
+
 def run_graph_workload(args, rank, local_rank, world, peaks, name):
     """CNN images/s through sparoa_run_graph (not the default bench line)."""
     import torch
@@ -484,6 +580,10 @@ def main():
             line["cpu_baseline"] = cpu_baseline_conv()
     elif args.workload in ("resnet18", "mobilenet_v2"):
         line = run_graph_workload(args, rank, local_rank, world, peaks, args.workload)
+    elif args.workload == "fc":
+        line = run_fc(args, rank, local_rank, world, peaks)
+    elif args.workload == "mlp_sweep":
+        line = run_mlp_sweep(args, rank, local_rank, world, peaks)
     else:
         raise SystemExit(f"workload {args.workload} is not wired into bench.py")
     if rank == 0:

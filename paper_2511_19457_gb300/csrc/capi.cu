@@ -394,6 +394,10 @@ sparoa_status run_conv(sparoa_ctx* ctx, const ConvPlan& c) {
   if (c.yo) a.out_occ = to_dev(*c.yo);
   a.emit = c.yo ? 1 : 0;
   a.err = ctx->d_err();
+  if (!pointwise && conv3_supported(a)) {
+    SP_CUDA(launch_conv3(a, ctx->stream));
+    return SPAROA_OK;
+  }
   if (a.conv == 2) choose_spatial_tile(a);
   SP_CUDA(launch_igemm(a, ctx->stream));
   return SPAROA_OK;

@@ -631,6 +631,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (et == 0) bulk_wait_all();
   }
 
+  __syncwarp();  // lanes that finished early wait for their warp's working lane
   tc_fence_before();
   __syncthreads();
   if (warp == 8) {
@@ -720,6 +721,9 @@ cudaError_t launch_cfg(const IgemmArgs& a, const CUtensorMap& tA, const CUtensor
 }
 
 }  // namespace
+
+PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() { return get_encode(); }
+int device_sm_count() { return num_sms(); }
 
 void choose_spatial_tile(IgemmArgs& a) {
   int64_t best = -1;

@@ -49,6 +49,12 @@ cudaError_t launch_igemm(const IgemmArgs& a, cudaStream_t s);
 // conv = 2: the bw x bh x bn (= 128) output tile with the fewest padded pixels.
 void choose_spatial_tile(IgemmArgs& a);
 
+// 3x3 stride-1 pad-1 convolution with resident weights and per-tile input
+// slabs (k_conv3.cu); the same IgemmArgs (conv geometry, epilogue, dispatch,
+// occupancy).  conv3_supported() says whether the shape fits.
+bool conv3_supported(const IgemmArgs& a);
+cudaError_t launch_conv3(const IgemmArgs& a, cudaStream_t s);
+
 // ----------------------------------------------------------------------------
 // Column-compacting zero-skip FC for few rows (M <= 128 per row block)
 // ----------------------------------------------------------------------------

@@ -328,3 +328,59 @@ def test_invalid_arguments_return_status(sp, ctx):
                        thr=sp.thresholds(force_path=7))
     assert e.value.status == sp.ERR_INVALID_ARG
     ctx.sync()   # the context stays usable
+
+
+# 3x3 stride-1 convolutions with resident weights and per-tile input slabs
+CONV3_CASES = [
+    # N, H, W, Cin, Cout, act, residual
+    (1, 7, 9, 64, 64, 1, True),
+    (2, 30, 17, 32, 128, 2, False),
+    (1, 20, 112, 64, 64, 1, False),
+    (3, 5, 5, 16, 64, 0, True),
+]
+
+
+@pytest.mark.parametrize("case", CONV3_CASES)
+@pytest.mark.parametrize("force", [1, 2])
+def test_conv3x3_slab_kernel(sp, ctx, case, force):
+    N, H, W, Cin, Cout, act, use_res = case
+    g = torch.Generator().manual_seed(H * W + Cin + Cout)
+    xb = _bits((N, H, W, Cin), H * 31 + W, zero_p=0.5, dist="abs")
+    wb = synth.to_bf16_bits(synth.he_normal((Cout, 3, 3, Cin), Cin * 9, g))
+    bn = synth.random_bn(Cout, g)
+    bias = (0.1 * torch.randn(Cout, generator=g)).numpy().astype(np.float32)
+    resb = _bits((N, H, W, Cout), Cout + 1, zero_p=0.2) if use_res else None
+    y = torch.empty(N, H, W, Cout, dtype=torch.bfloat16, device="cuda")
+    yo = sp.OccupancyBuffer(N * H * W, Cout)
+    st = sp.sparoa_conv2d(ctx, _dev(sp, xb, (N, H, W, Cin)), _dev(sp, wb, (Cout, 3, 3, Cin)), y,
+                          stride=1, pad=1, bias=torch.from_numpy(bias).cuda(),
+                          bn=torch.from_numpy(bn).cuda(), act=act,
+                          residual=_dev(sp, resb, (N, H, W, Cout)) if use_res else None,
+                          thr=sp.thresholds(force_path=force), y_occ=yo, host=True)
+    assert st.path == force
+    ref = orc.conv2d(xb, N, H, W, Cin, wb, Cout, 3, 3, 1, 1, bias=bias, bn=bn, residual_bits=resb,
+                     act=act)
+    assert_close(_f64(y), ref, what=f"conv3 {case} force={force}")
+    assert_occ_equal(yo.to_host(), orc.stats(sp.device_to_bits(y), N * H * W, Cout), "conv3 y_occ")
+
+
+def test_conv3x3_slab_kernel_skips_zero_regions(sp, ctx):
+    """Top half of every image and one whole image all zero: the zero-skip path
+    leaves out those taps' MMAs and still matches the oracle (including tiles
+    whose every tap is unoccupied)."""
+    N, H, W, C = 3, 24, 24, 64
+    g = torch.Generator().manual_seed(8)
+    x = torch.randn(N, H, W, C, generator=g).abs()
+    x[:, :12] = 0.0
+    x[1] = 0.0
+    xb = synth.to_bf16_bits(x)
+    wb = synth.to_bf16_bits(synth.he_normal((64, 3, 3, C), 9 * C, g))
+    outs = []
+    for force in (1, 2):
+        y = torch.empty(N, H, W, 64, dtype=torch.bfloat16, device="cuda")
+        sp.sparoa_conv2d(ctx, _dev(sp, xb, (N, H, W, C)), _dev(sp, wb, (64, 3, 3, C)), y, stride=1,
+                         pad=1, act=1, thr=sp.thresholds(force_path=force), host=True)
+        outs.append(_f64(y))
+    ref = orc.conv2d(xb, N, H, W, C, wb, 64, 3, 3, 1, 1, act=1)
+    assert_close(outs[0], ref, what="dense")
+    assert_close(outs[1], ref, what="skip")
