@@ -373,8 +373,8 @@ def run_conv(args, rank, local_rank, world, peaks):
     stats_bytes = R * C * 2 + int(sp._lib.sparoa_occupancy_bytes(R, C))
     roof = {"bound": "tensor", "achieved": achieved_tf, "peak": peaks["bf16_tflops"],
             "unit": "TFLOP/s", "frac": achieved_tf / peaks["bf16_tflops"],
-            "traffic": ncu_traffic("igemm_conv3x3_8x56x56x64"),
-            "kernel": "igemm_kernel<64> (" + path + ")", "kernel_us": conv_us,
+            "traffic": ncu_traffic("conv3_kernel_8x56x56x64"),
+            "kernel": "conv3_kernel<64> (" + path + ")", "kernel_us": conv_us,
             "algorithmic_flops": alg_flops, "algorithmic_bytes": conv_bytes,
             "hbm_view": {"achieved_gbs": conv_bytes / (conv_us * 1e-6) / 1e9,
                          "frac": conv_bytes / (conv_us * 1e-6) / 1e9 / peaks["hbm_gbs"]},

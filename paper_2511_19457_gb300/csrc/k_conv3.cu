@@ -157,7 +157,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     int j = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++j) {
-      if (!skip && t_ != 0) break;  // dense path: one thread streams the slabs
+      if (!skip && warp != 0) break;  // dense path: warp 0 walks the tiles, lane 0 streams the slabs
       const int b = j & 1;
       const int mb = j % 3;  // mask buffer: the MMAs of tile j - 3 are issued by now
       const int img = t / G.tiles_per_img;
@@ -199,7 +199,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (!skip) {
-        if (!ok) break;
+        if (__shfl_sync(0xffffffffu, ok ? 1 : 0, 0) == 0) break;
         continue;
       }
       // all masks written (and s_pos free for the next tile); uniform abort decision
@@ -208,18 +208,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 8) {
     // -------------------------------------------------------------- MMA issue
-    if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(kBM, CO);
-      bool ok = mbar_wait(bar_w, 0u, err, s_abort, kErrTimeoutFull);
-      tc_fence_after();
-      const int cbn = C / 64;
-      int j = 0;
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++j) {
-        const int b = j & 1;
+    // The whole warp walks the tiles so that it stays converged between tiles;
+    // lane 0 waits, issues the MMAs and commits.
+    constexpr uint32_t idesc = idesc_bf16_f32(kBM, CO);
+    bool ok = true;
+    if (lane == 0) ok = mbar_wait(bar_w, 0u, err, s_abort, kErrTimeoutFull);
+    ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+    tc_fence_after();
+    int j = 0;
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++j) {
+      const int b = j & 1;
+      if (lane == 0) {
+        ok = mbar_wait(bar_acce + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutAcc) &&
+             mbar_wait(bar_full + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutFull);
+      }
+      if (lane == 0 && ok) {
         const int q0 = (t - (t / G.tiles_per_img) * G.tiles_per_img) * kBM;
         const int qoff = q0 - (q0 / Wp) * Wp;
-        if (!mbar_wait(bar_acce + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutAcc)) break;
-        if (!mbar_wait(bar_full + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutFull)) break;
         tc_fence_after();
         const uint32_t d = tmem + (uint32_t)(b * CO);
         const uint32_t slab = sSlab + (uint32_t)(b * G.slab_bytes);
@@ -227,31 +232,55 @@ __global__ void __launch_bounds__(kThreads, 1)
         // in the start-address field (byte offset >> 4), which never carries out
         const uint64_t adesc0 = smem_desc_kmajor<64>(slab + (uint32_t)(qoff * 128));
         const uint64_t bdesc0 = smem_desc_kmajor<64>(sW);
-        const unsigned long long* tm = &s_tap[(j % 3) * 16];
-        bool first = true;
+        // Occupied taps as a 9-bit mask (one 64-channel block: C == 64). The
+        // lane issuing MMAs is slow at anything else, so the dense case is a
+        // straight run of 36 MMAs and the zero-skip case one branch per tap;
+        // every accumulate flag is a constant (the first occupied tap's first
+        // k-step is the only non-accumulating MMA).
+        uint32_t tapmask = 0x1FFu;
+        if (skip) {
+          const unsigned long long* tm = &s_tap[(j % 3) * 16];
+          tapmask = 0u;
 #pragma unroll
-        for (int tap = 0; tap < 9; ++tap) {
-          const unsigned long long tmask = skip ? tm[tap] : ~0ull;
-          const uint64_t arow = (uint64_t)((((tap / 3) * Wp + (tap % 3)) * 128) >> 4);
-          for (int cb = 0; cb < cbn; ++cb) {
-            if (!((tmask >> cb) & 1ull)) continue;  // all-zero 64-channel tile for this tap
-            const uint64_t ad = adesc0 + arow + (uint64_t)((cb * G.chunk_stride) >> 4);
-            const uint64_t bd = bdesc0 + (uint64_t)(((tap * cbn + cb) * CO * 128) >> 4);
-#pragma unroll
-            for (int ks = 0; ks < 4; ++ks) {
-              tc_mma_bf16(d, ad + (uint64_t)(2 * ks), bd + (uint64_t)(2 * ks), idesc, first ? 0u : 1u);
-              first = false;
-            }
-          }
+          for (int tap = 0; tap < 9; ++tap) tapmask |= (tm[tap] & 1ull) ? (1u << tap) : 0u;
         }
-        if (first) {
-          // no (tap, channel tile) is occupied: tap 0's activations are all zero,
-          // so one non-accumulating MMA on them writes the zero accumulator
+        if (tapmask == 0x1FFu) {
           tc_mma_bf16(d, adesc0, bdesc0, idesc, 0u);
+#pragma unroll
+          for (int i = 1; i < 36; ++i) {
+            const int tap = i >> 2, ks = i & 3;
+            tc_mma_bf16(d, adesc0 + (uint64_t)((((tap / 3) * Wp + (tap % 3)) * 128) >> 4) + (uint64_t)(2 * ks),
+                        bdesc0 + (uint64_t)((tap * CO * 128) >> 4) + (uint64_t)(2 * ks), idesc, 1u);
+          }
+        } else if (tapmask == 0u) {
+          // no tap is occupied: tap 0's activations are all zero, so one
+          // non-accumulating MMA on them writes the zero accumulator
+          tc_mma_bf16(d, adesc0, bdesc0, idesc, 0u);
+        } else {
+          const int ftap = __ffs((int)tapmask) - 1;
+          tapmask &= ~(1u << ftap);
+          {
+            const uint64_t ad = adesc0 + (uint64_t)((((ftap / 3) * Wp + (ftap % 3)) * 128) >> 4);
+            const uint64_t bd = bdesc0 + (uint64_t)((ftap * CO * 128) >> 4);
+            tc_mma_bf16(d, ad, bd, idesc, 0u);
+#pragma unroll
+            for (int ks = 1; ks < 4; ++ks)
+              tc_mma_bf16(d, ad + (uint64_t)(2 * ks), bd + (uint64_t)(2 * ks), idesc, 1u);
+          }
+#pragma unroll
+          for (int tap = 0; tap < 9; ++tap) {
+            if (!((tapmask >> tap) & 1u)) continue;  // all-zero activations, or the peeled tap
+            const uint64_t ad = adesc0 + (uint64_t)((((tap / 3) * Wp + (tap % 3)) * 128) >> 4);
+            const uint64_t bd = bdesc0 + (uint64_t)((tap * CO * 128) >> 4);
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks)
+              tc_mma_bf16(d, ad + (uint64_t)(2 * ks), bd + (uint64_t)(2 * ks), idesc, 1u);
+          }
         }
         tc_commit(bar_empty + 8 * b);  // slab free once these MMAs are done
         tc_commit(bar_accf + 8 * b);
       }
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
     }
   } else {
     // -------------------------------------------------------------- epilogue
@@ -393,7 +422,9 @@ cudaError_t launch_co(const CUtensorMap& tX, const CUtensorMap& tW, const IgemmA
 
 bool conv3_supported(const IgemmArgs& a) {
   if (a.kh != 3 || a.kw != 3 || a.stride != 1 || a.pad != 1) return false;
-  if (a.Cp % 64 != 0 || (a.N != 64 && a.N != 128) || a.W + 2 > 256) return false;
+  // one 64-channel block in and out: the weights (72 KB) stay resident next to
+  // two halo slabs
+  if (a.Cp != 64 || a.N != 64 || a.W + 2 > 256) return false;
   const int w_bytes = 9 * a.Cp * a.N * 2;
   const int Wp = a.W + 2;
   return w_bytes <= 96 * 1024 && conv3_smem(a.Cp, a.N, a.W) <= 220 * 1024 &&
@@ -439,8 +470,8 @@ cudaError_t launch_conv3(const IgemmArgs& a, cudaStream_t s) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
   }
-  if (g.Co == 64) return launch_co<64>(tX, tW, a, g, smem, s);
-  return launch_co<128>(tX, tW, a, g, smem, s);
+  if (g.C != 64 || g.Co != 64) return cudaErrorInvalidValue;
+  return launch_co<64>(tX, tW, a, g, smem, s);
 }
 
 }  // namespace sparoa

@@ -419,10 +419,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           const bool last = stage_last[slot] != 0;
           const uint32_t a = sA + slot * C::kAStage;
           const uint32_t bb = sB + slot * C::kBStage;
+          // k-steps advance the start-address field by 32 B (2 units); the
+          // accumulate flags are constants on both branches (a per-MMA flag
+          // computed at run time roughly halves the issue rate)
+          const uint64_t ad = smem_desc_kmajor<BK>(a), bd = smem_desc_kmajor<BK>(bb);
+          if (first) {
+            tc_mma_bf16(d, ad, bd, idesc, 0u);
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k)
-            tc_mma_bf16(d, smem_desc_kmajor<BK>(a + 32 * k), smem_desc_kmajor<BK>(bb + 32 * k),
-                        idesc, (!first || k > 0) ? 1u : 0u);
+            for (int k = 1; k < BK / 16; ++k)
+              tc_mma_bf16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc, 1u);
+          } else {
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k)
+              tc_mma_bf16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc, 1u);
+          }
           first = false;
           tc_commit(bar_empty + 8 * slot);
           ++it;

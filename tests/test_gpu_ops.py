@@ -337,6 +337,7 @@ CONV3_CASES = [
     (2, 30, 17, 32, 128, 2, False),
     (1, 20, 112, 64, 64, 1, False),
     (3, 5, 5, 16, 64, 0, True),
+    (8, 56, 56, 64, 64, 1, True),   # 208 tiles: several per persistent CTA
 ]
 
 
