@@ -193,6 +193,14 @@ sparoa_status sparoa_destroy(sparoa_ctx *ctx);
 /* Change the stream later calls enqueue on. */
 sparoa_status sparoa_set_stream(sparoa_ctx *ctx, void *stream);
 
+/* Launch overlap (default on): each kernel of a call is launched with CUDA's
+ * programmatic stream serialization, so that its on-chip prologue (barrier
+ * initialisation, tensor-memory allocation) runs while the kernel before it
+ * on the stream finishes.  No kernel reads or writes global memory before the
+ * previous grid has completed, so results do not depend on this setting.
+ * enable = 0 launches plainly.  Errors: INVALID_ARG (ctx == NULL). */
+sparoa_status sparoa_set_overlap(sparoa_ctx *ctx, int32_t enable);
+
 /* Wait for the stream; report (and clear) a device-side timeout. */
 sparoa_status sparoa_sync(sparoa_ctx *ctx);
 

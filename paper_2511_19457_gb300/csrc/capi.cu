@@ -11,6 +11,14 @@
 #include "../../include/sparoa.h"
 #include "sparoa_kernels.h"
 
+namespace sparoa {
+namespace {
+thread_local bool t_pdl = true;
+}  // namespace
+bool pdl_enabled() { return t_pdl; }
+void set_pdl_enabled(bool on) { t_pdl = on; }
+}  // namespace sparoa
+
 using namespace sparoa;
 
 namespace {
@@ -31,6 +39,7 @@ struct sparoa_ctx {
   DevBuf pad_x, pad_w;
   DevBuf arena;       // sparoa_run_graph activations, occupancies, paths
   std::vector<sparoa_occupancy> graph_occ;
+  int overlap = 1;    // programmatic dependent launch between consecutive kernels
   uint32_t* d_err() const { return reinterpret_cast<uint32_t*>(small.p); }
   int32_t* d_path() const { return reinterpret_cast<int32_t*>(reinterpret_cast<char*>(small.p) + 16); }
 };
@@ -65,14 +74,19 @@ sparoa_status fail(sparoa_ctx* ctx, sparoa_status st, const char* fmt, ...) {
     if (s_ != SPAROA_OK) return s_;        \
   } while (0)
 
-// Make `device` current for the duration of a call and restore the caller's.
+// Make `device` current for the duration of a call and restore the caller's;
+// launches made meanwhile follow the context's overlap setting.
 struct DeviceGuard {
   int prev = -1;
   bool changed = false;
-  explicit DeviceGuard(int dev) {
+  bool pdl_prev = true;
+  explicit DeviceGuard(int dev, int overlap = 1) {
     if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) changed = cudaSetDevice(dev) == cudaSuccess;
+    pdl_prev = pdl_enabled();
+    set_pdl_enabled(overlap != 0);
   }
   ~DeviceGuard() {
+    set_pdl_enabled(pdl_prev);
     if (changed) cudaSetDevice(prev);
   }
 };
@@ -154,21 +168,35 @@ sparoa_status check_occ(sparoa_ctx* ctx, const sparoa_occupancy* o, int64_t R, i
   return SPAROA_OK;
 }
 
-// Clear an occupancy block (fields may be spread when the library carved them).
-sparoa_status occ_clear(sparoa_ctx* ctx, const sparoa_occupancy& o) {
-  const OccLayout l = occ_layout(o.R, o.C);
-  char* b = reinterpret_cast<char*>(o.nnz);
-  if (reinterpret_cast<char*>(o.blk_mask) == b + l.blk) {
-    SP_CUDA(cudaMemsetAsync(b, 0, l.total, ctx->stream));
-  } else {
-    const int64_t T = (o.C + 63) / 64, W64 = (T + 63) / 64, RB = (o.R + 127) / 128,
-                  C32 = (o.C + 31) / 32;
-    SP_CUDA(cudaMemsetAsync(o.nnz, 0, 8, ctx->stream));
-    SP_CUDA(cudaMemsetAsync(o.col_nnz, 0, 4 * (size_t)o.C, ctx->stream));
-    SP_CUDA(cudaMemsetAsync(o.tile_nnz, 0, 4 * (size_t)T, ctx->stream));
-    SP_CUDA(cudaMemsetAsync(o.row_bm, 0, 8 * (size_t)(o.R * W64), ctx->stream));
-    SP_CUDA(cudaMemsetAsync(o.blk_mask, 0, 4 * (size_t)(RB * C32), ctx->stream));
+// Clear an occupancy block with the clear kernel (a kernel, not a memset, so
+// that consecutive launches keep overlapping).  counters_only: the Eq. 1
+// counters alone (the stats kernel writes the bitmaps whole).
+sparoa_status occ_clear(sparoa_ctx* ctx, const sparoa_occupancy& o, bool counters_only = false) {
+  const int64_t T = (o.C + 63) / 64, W64 = (T + 63) / 64, RB = (o.R + 127) / 128,
+                C32 = (o.C + 31) / 32;
+  ClearArgs a = {};
+  a.p[0] = reinterpret_cast<uint32_t*>(o.nnz);
+  a.words[0] = 2;
+  a.p[1] = o.col_nnz;
+  a.words[1] = o.C;
+  a.p[2] = o.tile_nnz;
+  a.words[2] = T;
+  if (!counters_only) {
+    a.p[3] = reinterpret_cast<uint32_t*>(o.row_bm);
+    a.words[3] = 2 * o.R * W64;
+    a.p[4] = o.blk_mask;
+    a.words[4] = RB * C32;
   }
+  SP_CUDA(launch_clear(a, ctx->stream));
+  return SPAROA_OK;
+}
+
+// Eq. 1 count and bitmaps of x [R, C] into `o` (counters cleared first; the
+// stats kernel writes the bitmaps whole).
+sparoa_status run_stats(sparoa_ctx* ctx, const void* x, int64_t R, int64_t C,
+                        const sparoa_occupancy& o) {
+  SP_TRY(occ_clear(ctx, o, true));
+  SP_CUDA(launch_stats(static_cast<const __nv_bfloat16*>(x), R, (int)C, to_dev(o), ctx->stream));
   return SPAROA_OK;
 }
 
@@ -177,9 +205,7 @@ sparoa_status measure(sparoa_ctx* ctx, const void* x, int64_t R, int64_t C, spar
   const OccLayout l = occ_layout(R, C);
   SP_TRY(ensure(ctx, ctx->occ, l.total));
   occ_carve(ctx->occ.p, R, C, out);
-  SP_CUDA(cudaMemsetAsync(ctx->occ.p, 0, l.total, ctx->stream));
-  SP_CUDA(launch_stats(static_cast<const __nv_bfloat16*>(x), R, (int)C, to_dev(*out), ctx->stream));
-  return SPAROA_OK;
+  return run_stats(ctx, x, R, C, *out);
 }
 
 // ---------------------------------------------------------------------------
@@ -456,11 +482,17 @@ sparoa_status sparoa_create(sparoa_ctx** out, int device, void* stream) {
 
 sparoa_status sparoa_destroy(sparoa_ctx* ctx) {
   if (!ctx) return SPAROA_OK;
-  DeviceGuard g(ctx->device);
+  DeviceGuard g(ctx->device, ctx->overlap);
   cudaStreamSynchronize(ctx->stream);
   for (DevBuf* b : {&ctx->small, &ctx->occ, &ctx->pad_x, &ctx->pad_w, &ctx->arena})
     if (b->p) cudaFree(b->p);
   delete ctx;
+  return SPAROA_OK;
+}
+
+sparoa_status sparoa_set_overlap(sparoa_ctx* ctx, int32_t enable) {
+  if (!ctx) return SPAROA_ERR_INVALID_ARG;
+  ctx->overlap = enable ? 1 : 0;
   return SPAROA_OK;
 }
 
@@ -472,7 +504,7 @@ sparoa_status sparoa_set_stream(sparoa_ctx* ctx, void* stream) {
 
 sparoa_status sparoa_sync(sparoa_ctx* ctx) {
   if (!ctx) return SPAROA_ERR_INVALID_ARG;
-  DeviceGuard g(ctx->device);
+  DeviceGuard g(ctx->device, ctx->overlap);
   return read_device_error(ctx);
 }
 
@@ -500,12 +532,11 @@ sparoa_status sparoa_op_stats(sparoa_ctx* ctx, const void* x, int64_t N, int64_t
   if (R > 0 && (C % 8) == 0 && !aligned16(x))
     return fail(ctx, SPAROA_ERR_INVALID_ARG, "op_stats: x must be 16-byte aligned");
   SP_TRY(check_occ(ctx, occ, R, C, "op_stats"));
-  DeviceGuard g(ctx->device);
+  DeviceGuard g(ctx->device, ctx->overlap);
   sparoa_occupancy o;
   if (occ) {
     o = *occ;
-    SP_TRY(occ_clear(ctx, o));
-    SP_CUDA(launch_stats(static_cast<const __nv_bfloat16*>(x), R, (int)C, to_dev(o), ctx->stream));
+    SP_TRY(run_stats(ctx, x, R, C, o));
   } else {
     SP_TRY(measure(ctx, x, R, C, &o));
   }
@@ -556,7 +587,7 @@ sparoa_status sparoa_gemm(sparoa_ctx* ctx, const void* x, int64_t M, int64_t K, 
   SP_TRY(check_ep(ctx, ep));
   SP_TRY(check_occ(ctx, x_occ, M, K, "gemm x_occ"));
   SP_TRY(check_occ(ctx, y_occ, M, N, "gemm y_occ"));
-  DeviceGuard g(ctx->device);
+  DeviceGuard g(ctx->device, ctx->overlap);
   const Work w = fc_work(M, K, N);
   GemmPlan p;
   p.x = x;
@@ -621,7 +652,7 @@ sparoa_status sparoa_conv2d(sparoa_ctx* ctx, const void* x, int64_t N, int64_t H
     return fail(ctx, SPAROA_ERR_UNSUPPORTED, "conv2d: depthwise needs C %% 8 == 0 and a 3x3 kernel");
   if (!depthwise && (C_out % 8))
     return fail(ctx, SPAROA_ERR_INVALID_ARG, "conv2d: C_out must be a multiple of 8");
-  DeviceGuard g(ctx->device);
+  DeviceGuard g(ctx->device, ctx->overlap);
   const Work wk = conv_work(N, H, W, C_in, C_out, kh, kw, Ho, Wo, groups);
   sparoa_occupancy xo;
   const bool need_x_occ = !depthwise || host_out;
@@ -719,7 +750,7 @@ sparoa_status sparoa_maxpool2d(sparoa_ctx* ctx, const void* x, int64_t N, int64_
   if (N > 0 && (!x || !y || !aligned16(x) || !aligned16(y)))
     return fail(ctx, SPAROA_ERR_INVALID_ARG, "maxpool: NULL or misaligned tensor");
   SP_TRY(check_occ(ctx, y_occ, N * Ho * Wo, C, "maxpool y_occ"));
-  DeviceGuard g(ctx->device);
+  DeviceGuard g(ctx->device, ctx->overlap);
   if (y_occ) SP_TRY(occ_clear(ctx, *y_occ));
   OccDev o{};
   if (y_occ) o = to_dev(*y_occ);
@@ -739,7 +770,7 @@ sparoa_status sparoa_avgpool_global(sparoa_ctx* ctx, const void* x, int64_t N, i
   if (N > 0 && (!x || !y || !aligned16(x) || !aligned16(y)))
     return fail(ctx, SPAROA_ERR_INVALID_ARG, "avgpool: NULL or misaligned tensor");
   SP_TRY(check_occ(ctx, y_occ, N, C, "avgpool y_occ"));
-  DeviceGuard g(ctx->device);
+  DeviceGuard g(ctx->device, ctx->overlap);
   if (y_occ) SP_TRY(occ_clear(ctx, *y_occ));
   OccDev o{};
   if (y_occ) o = to_dev(*y_occ);
@@ -757,7 +788,7 @@ sparoa_status sparoa_bn_act(sparoa_ctx* ctx, const void* x, int64_t R, int64_t C
     return fail(ctx, SPAROA_ERR_INVALID_ARG, "bn_act: NULL or misaligned tensor");
   SP_TRY(check_ep(ctx, ep));
   SP_TRY(check_occ(ctx, y_occ, R, C, "bn_act y_occ"));
-  DeviceGuard g(ctx->device);
+  DeviceGuard g(ctx->device, ctx->overlap);
   if (y_occ) SP_TRY(occ_clear(ctx, *y_occ));
   OccDev o{};
   if (y_occ) o = to_dev(*y_occ);
@@ -886,7 +917,7 @@ sparoa_status sparoa_run_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_
     return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: y holds %llu bytes, output needs %llu",
                 (unsigned long long)y_bytes, (unsigned long long)out_bytes);
   if (y && !aligned16(y)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: misaligned y");
-  DeviceGuard g(ctx->device);
+  DeviceGuard g(ctx->device, ctx->overlap);
   SP_TRY(ensure(ctx, ctx->arena, off));
   char* base = static_cast<char*>(ctx->arena.p);
   ctx->graph_occ.assign(vals.size(), sparoa_occupancy{});
@@ -897,10 +928,14 @@ sparoa_status sparoa_run_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_
     return v == 0 ? const_cast<void*>(x) : static_cast<void*>(base + vals[(size_t)v].act_off);
   };
   // ---- execute
-  SP_CUDA(cudaMemsetAsync(base + nnz_off, 0, occ_end - nnz_off + align_up(sizeof(int32_t) * (size_t)n_ops),
-                          ctx->stream));
-  SP_CUDA(launch_stats(static_cast<const __nv_bfloat16*>(x), N * H * W, (int)C,
-                       to_dev(ctx->graph_occ[0]), ctx->stream));
+  {
+    // every occupancy block and path slot of the walk, cleared in one launch
+    ClearArgs z = {};
+    z.p[0] = reinterpret_cast<uint32_t*>(base + nnz_off);
+    z.words[0] = (int64_t)((occ_end - nnz_off + align_up(sizeof(int32_t) * (size_t)n_ops)) / 4);
+    SP_CUDA(launch_clear(z, ctx->stream));
+  }
+  SP_TRY(run_stats(ctx, x, N * H * W, C, ctx->graph_occ[0]));
   for (int i = 0; i < n_ops; ++i) {
     const sparoa_op& op = ops[i];
     const Val& in = vals[(size_t)op.input];
@@ -995,8 +1030,7 @@ sparoa_status sparoa_run_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_
         p.yo = yo;
         if (aux[(size_t)i].fc_view) {
           occ_carve(base + aux[(size_t)i].fcocc, M, K, &p.xo);
-          SP_CUDA(launch_stats(static_cast<const __nv_bfloat16*>(p.x), M, (int)K, to_dev(p.xo),
-                               ctx->stream));
+          SP_TRY(run_stats(ctx, p.x, M, K, p.xo));
         } else {
           p.xo = xo;
         }

@@ -36,7 +36,6 @@
 namespace sparoa {
 
 PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder();  // k_igemm.cu
-int device_sm_count();                              // k_igemm.cu
 
 namespace {
 // Slab rows: a tile's 128 positions plus the two extra rows and two columns
@@ -96,17 +95,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t bar_acce = sCtl + 56;
   volatile int* s_abort = reinterpret_cast<volatile int*>(ctl + 72);
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(ctl + 76);
-  unsigned long long* s_tap = reinterpret_cast<unsigned long long*>(ctl + 128);  // [3][16]
+  uint32_t* s_tapm = reinterpret_cast<uint32_t*>(ctl + 128);  // [3] 9-bit occupied-tap masks
   float* s_scale = reinterpret_cast<float*>(ctl + 512);                          // [CO]
   float* s_shift = s_scale + CO;                                                 // [CO]
   uint32_t* s_cnt = reinterpret_cast<uint32_t*>(s_shift + CO);                   // [4][CO]
   uint32_t* s_acc = s_cnt + 4 * CO;                                              // [CO]
-  unsigned long long* s_pos = reinterpret_cast<unsigned long long*>(s_acc + CO + (CO & 1));  // [kMaxPos]
+  uint8_t* s_pos = reinterpret_cast<uint8_t*>(s_acc + CO);  // [kMaxPos] 1 = input pixel has a non-zero
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int path = decide_path(P.disp);
-  record_path(P.disp, path);
-  const bool skip = path == 2;
   const int N = G.N, H = G.H, W = G.W, C = G.C, Wp = G.Wp;
   const int tiles = N * G.tiles_per_img;
   const int act = P.ep.act;
@@ -116,20 +112,29 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* const err = P.err;
   const int emit = P.emit;
 
+  // on-chip prologue, overlapping the previous grid on the stream
   if (threadIdx.x == 0) {
     mbar_init(bar_w, 1u);
     for (int b = 0; b < 2; ++b) {
-      mbar_init(bar_full + 8 * b, skip ? 129u : 1u);
       mbar_init(bar_empty + 8 * b, 1u);
       mbar_init(bar_accf + 8 * b, 1u);
       mbar_init(bar_acce + 8 * b, 128u);
     }
     *s_abort = 0;
-    fence_mbar_init();
     prefetch_tmap(&tmX);
     prefetch_tmap(&tmW);
   }
   if (warp == 8) tmem_alloc(smem_u32(s_tmem), (uint32_t)(2 * CO));
+  pdl_wait();
+  pdl_trigger();
+  const int path = decide_path(P.disp);
+  record_path(P.disp, path);
+  const bool skip = path == 2;
+  if (threadIdx.x == 0) {
+    // zero-skip slabs complete on 128 mask arrivals + the TMA's arrival
+    for (int b = 0; b < 2; ++b) mbar_init(bar_full + 8 * b, skip ? 129u : 1u);
+    fence_mbar_init();
+  }
   if (warp >= 4 && warp < 8) {
     const int et = threadIdx.x - 128;
     for (int c = et; c < CO; c += 128) {
@@ -163,30 +168,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int img = t / G.tiles_per_img;
       const int q0 = (t - img * G.tiles_per_img) * kBM;
       const int oh0 = q0 / Wp;
-      if (skip) {
-        // zero-skip masks of this tile, computed before waiting for its slab
-        // buffer: per tap, OR of the row bitmaps of the tile's 128 shifted pixels
-        const int npos = G.R * Wp;
-        for (int pp = t_; pp < npos && pp < kMaxPos; pp += 128) {
-          const int pr = oh0 - 1 + pp / Wp, pc = pp % Wp - 1;  // input pixel of slab position pp
-          unsigned long long w = 0ull;
-          if (pr >= 0 && pr < H && pc >= 0 && pc < W)
-            w = in_rowbm[(((int64_t)img * H + pr) * W + pc) * in_W64];
-          s_pos[pp] = w;
-        }
-        if (t_ < 16) s_tap[mb * 16 + t_] = in_W64 > 1 ? ~0ull : 0ull;
-        named_bar_sync(1, 128);
-        const int qoff = q0 - oh0 * Wp;
-        const bool rvalid = q0 + t_ < H * Wp;
-#pragma unroll
-        for (int tap = 0; tap < 9; ++tap) {
-          const int pp = qoff + t_ + (tap / 3) * Wp + (tap % 3);
-          unsigned long long w = (rvalid && pp < kMaxPos) ? s_pos[pp] : 0ull;
-#pragma unroll
-          for (int s = 16; s > 0; s >>= 1) w |= __shfl_xor_sync(0xffffffffu, w, s);
-          if (lane == 0 && w) atomicOr(&s_tap[mb * 16 + tap], w);
-        }
-      }
+      // the slab first, so that its load overlaps the mask computation below
       bool ok = true;
       if (t_ == 0) {
         ok = mbar_wait(bar_empty + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutEmpty);
@@ -197,6 +179,40 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_4d(dst + (uint32_t)(cb * G.chunk_stride), &tmX, bar_full + 8 * b, cb * 64, -1,
                         oh0 - 1, img);
         }
+      }
+      if (skip) {
+        // zero-skip masks of this tile: per tap, OR of the row bitmaps of the
+        // tile's 128 shifted pixels (the mask buffer of tile j - 3 is free: the
+        // empty-slot wait of tile j - 1 saw those MMAs complete)
+        // One 64-channel block (C == 64): a pixel's row bitmap word is its bit 0.
+        // All of this thread's bitmap loads are issued before any is used.
+        const int npos = G.R * Wp < kMaxPos ? G.R * Wp : kMaxPos;
+        uint32_t nzb = 0u;  // bit k: slab position t_ + 128 k is a non-zero pixel
+#pragma unroll
+        for (int k = 0; k < kMaxPos / 128; ++k) {
+          const int pp = t_ + 128 * k;
+          const int prr = pp / Wp;
+          const int pr = oh0 - 1 + prr, pc = pp - prr * Wp - 1;  // input pixel of slab position pp
+          unsigned long long w = 0ull;
+          if (pp < npos && pr >= 0 && pr < H && pc >= 0 && pc < W)
+            w = in_rowbm[(((int64_t)img * H + pr) * W + pc) * in_W64];
+          nzb |= (uint32_t)(w & 1ull) << k;
+        }
+#pragma unroll
+        for (int k = 0; k < kMaxPos / 128; ++k)
+          if (t_ + 128 * k < npos) s_pos[t_ + 128 * k] = (uint8_t)((nzb >> k) & 1u);
+        if (t_ == 0) s_tapm[mb] = 0u;
+        named_bar_sync(1, 128);
+        const int qoff = q0 - oh0 * Wp;
+        const bool rvalid = q0 + t_ < H * Wp;
+        uint32_t tb = 0u;  // bit tap: this output position reads a non-zero pixel under that tap
+#pragma unroll
+        for (int tap = 0; tap < 9; ++tap) {
+          const int pp = qoff + t_ + (tap / 3) * Wp + (tap % 3);
+          if (rvalid && pp < kMaxPos && s_pos[pp]) tb |= 1u << tap;
+        }
+        tb = __reduce_or_sync(0xffffffffu, tb);
+        if (lane == 0 && tb) atomicOr(&s_tapm[mb], tb);
       }
       if (!skip) {
         if (__shfl_sync(0xffffffffu, ok ? 1 : 0, 0) == 0) break;
@@ -237,13 +253,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // straight run of 36 MMAs and the zero-skip case one branch per tap;
         // every accumulate flag is a constant (the first occupied tap's first
         // k-step is the only non-accumulating MMA).
-        uint32_t tapmask = 0x1FFu;
-        if (skip) {
-          const unsigned long long* tm = &s_tap[(j % 3) * 16];
-          tapmask = 0u;
-#pragma unroll
-          for (int tap = 0; tap < 9; ++tap) tapmask |= (tm[tap] & 1ull) ? (1u << tap) : 0u;
-        }
+        uint32_t tapmask = skip ? s_tapm[j % 3] : 0x1FFu;
         if (tapmask == 0x1FFu) {
           tc_mma_bf16(d, adesc0, bdesc0, idesc, 0u);
 #pragma unroll
@@ -414,7 +424,8 @@ cudaError_t launch_co(const CUtensorMap& tX, const CUtensorMap& tW, const IgemmA
   }
   const int tiles = g.N * g.tiles_per_img;
   const int grid = tiles < device_sm_count() ? tiles : device_sm_count();
-  conv3_kernel<CO><<<grid, kThreads, smem, s>>>(tX, tW, a, g);
+  cudaError_t e = launch_kernel(conv3_kernel<CO>, dim3(grid), dim3(kThreads), (size_t)smem, s, tX, tW, a, g);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

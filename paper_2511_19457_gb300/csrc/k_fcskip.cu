@@ -28,6 +28,8 @@ __global__ void __launch_bounds__(kThreads) fcskip_kernel(const FcSkipArgs a) {
   int* s_cnt = reinterpret_cast<int*>(s_nz + 128);
   int* cols = s_cnt + 4;                                    // [K]
 
+  pdl_wait();
+  pdl_trigger();
   const int path = decide_path(a.disp);
   if (path != 2) return;  // the dense kernel of this launch runs instead
   record_path(a.disp, path);
@@ -172,8 +174,7 @@ cudaError_t launch_fcskip(const FcSkipArgs& a, cudaStream_t s) {
     attr = smem;
   }
   dim3 grid((a.N + 63) / 64, (a.M + 127) / 128);
-  fcskip_kernel<<<grid, kThreads, smem, s>>>(a);
-  return cudaGetLastError();
+  return launch_kernel(fcskip_kernel, grid, dim3(kThreads), smem, s, a);
 }
 
 }  // namespace sparoa

@@ -198,10 +198,6 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int path = decide_path(P.disp);
-  if (P.dense_only && path == 2) return;  // the zero-skip kernel of this launch runs instead
-  record_path(P.disp, path);
-  const bool skip = (path == 2);
   const int kblocks = (p.Ktot + BK - 1) / BK;
   const int nt = (p.N + BN - 1) / BN;
   const int mtiles = p.conv == 2 ? ((p.Nimg + p.bn - 1) / p.bn) * p.th * p.tw : (p.M + kBM - 1) / kBM;
@@ -229,8 +225,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *s_tmem;
+  pdl_wait();
+  pdl_trigger();
+  const int path = decide_path(P.disp);
+  // with dense_only the zero-skip kernel of this launch runs instead
+  const bool run = !(P.dense_only && path == 2);
+  if (run) record_path(P.disp, path);
+  const bool skip = (path == 2);
 
-  if (warp < 4) {
+  if (!run) {
+    // nothing to do; fall through to the common exit (TMEM is freed there)
+  } else if (warp < 4) {
     // ------------------------------------------------------------------ producers
     const int r = threadIdx.x;
     const int cb_per_tap = p.Cp / BK;
@@ -709,7 +714,7 @@ int num_sms() {
     int dev = 0;
     cudaGetDevice(&dev);
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-      n = 148;
+      n = 152;
   }
   return n;
 }
@@ -726,7 +731,9 @@ cudaError_t launch_cfg(const IgemmArgs& a, const CUtensorMap& tA, const CUtensor
     attr = true;
   }
   const int64_t grid = tiles < num_sms() ? tiles : num_sms();
-  igemm_kernel<BN, BK><<<(unsigned)grid, kThreads, Cfg<BN, BK>::kSmem, s>>>(tA, tB, tY, a);
+  cudaError_t e = launch_kernel(igemm_kernel<BN, BK>, dim3((unsigned)grid), dim3(kThreads),
+                                (size_t)Cfg<BN, BK>::kSmem, s, tA, tB, tY, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

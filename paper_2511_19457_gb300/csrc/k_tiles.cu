@@ -146,39 +146,102 @@ __device__ __forceinline__ void cta_done(const OccDev& o, const uint32_t* s_acc,
   for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
 
 // ---------------------------------------------------------------------------
+// Eq. 1 count and bitmaps of an existing tensor.  A CTA owns whole 128-row
+// blocks (every column tile of them), so it writes their row bitmap words and
+// block masks with plain stores; only the counters need clearing beforehand.
+// Column counts gather in shared memory (C words, dynamic) and reach global
+// memory once per CTA.
 __global__ void __launch_bounds__(kTileThreads) stats_kernel(const __nv_bfloat16* __restrict__ x,
                                                              int64_t R, int C, OccDev o_param) {
   const OccDev o = o_param;  // registers, not parameter-space loads
+  extern __shared__ uint32_t s_acc[];  // [C] when acc
   __shared__ uint32_t s_cnt[8 * 64];
-  __shared__ uint32_t s_acc[kMaxAccCols];
   const bool acc = C <= kMaxAccCols;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
   const bool vec = (C & 7) == 0;
-  acc_init(s_acc, C, acc);
-  TileEmit e;
-  e.init();
-  SPAROA_TILE_LOOP(R, C) {
-    const int64_t row0 = (tile / ctn) * 128;
-    const int col0 = (int)(tile % ctn) * 64;
-    const int c0 = col0 + cg * 8;
-    uint32_t m[4];
+  const int ctn = (C + 63) / 64;
+  const int64_t nrb = (R + 127) / 128;
+  if (acc)
+    for (int c = threadIdx.x; c < C; c += kTileThreads) s_acc[c] = 0u;
+  __syncthreads();
+  pdl_wait();
+  pdl_trigger();
+  for (int64_t rb = blockIdx.x; rb < nrb; rb += gridDim.x) {
+    const int64_t row0 = rb * 128;
+    unsigned long long rw[4] = {0ull, 0ull, 0ull, 0ull};  // row bitmap word being built, per owned row
+    for (int ct = 0; ct < ctn; ++ct) {
+      const int col0 = ct * 64;
+      const int c0 = col0 + cg * 8;
+      uint32_t m[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int64_t r = row0 + rs + 32 * i;
-      m[i] = 0;
-      if (r < R && c0 < C) {
-        const __nv_bfloat16* p = x + r * C + c0;
-        if (vec) {
-          m[i] = nz_mask8(__ldg(reinterpret_cast<const uint4*>(p)));
-        } else {
-          for (int j = 0; j < 8 && c0 + j < C; ++j)
-            if (bf16_nz(__bfloat16_as_ushort(p[j]))) m[i] |= 1u << j;
+      for (int i = 0; i < 4; ++i) {
+        const int64_t r = row0 + rs + 32 * i;
+        m[i] = 0u;
+        if (r < R && c0 < C) {
+          const __nv_bfloat16* p = x + r * C + c0;
+          if (vec) {
+            m[i] = nz_mask8(__ldg(reinterpret_cast<const uint4*>(p)));
+          } else {
+            for (int j = 0; j < 8 && c0 + j < C; ++j)
+              if (bf16_nz(__bfloat16_as_ushort(p[j]))) m[i] |= 1u << j;
+          }
         }
       }
-    }
+      // row bits: lanes 8k..8k+7 share a row
+      uint32_t cnt[8];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) e.row(m[i], row0 + rs + 32 * i, col0, o);
-    e.tile_done(row0, col0, o, s_cnt, s_acc, acc);
+      for (int j = 0; j < 8; ++j) cnt[j] = 0u;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const uint32_t bl = __ballot_sync(0xffffffffu, m[i] != 0u);
+        if ((bl >> (lane & ~7)) & 0xFFu) rw[i] |= 1ull << (ct & 63);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) cnt[j] += (m[i] >> j) & 1u;
+      }
+      if ((ct & 63) == 63 || ct == ctn - 1) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int64_t r = row0 + rs + 32 * i;
+          if (cg == 0 && r < R) o.row_bm[r * o.W64 + (ct >> 6)] = rw[i];
+          rw[i] = 0ull;
+        }
+      }
+      // column counts of the tile: 8 warps x 64 columns through shared memory
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        cnt[j] += __shfl_xor_sync(0xffffffffu, cnt[j], 8);
+        cnt[j] += __shfl_xor_sync(0xffffffffu, cnt[j], 16);
+      }
+      if (lane < 8) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) s_cnt[warp * 64 + cg * 8 + j] = cnt[j];
+      }
+      __syncthreads();
+      if (threadIdx.x < 64) {
+        uint32_t c = 0;
+#pragma unroll
+        for (int w = 0; w < kTileThreads / 32; ++w) c += s_cnt[w * 64 + threadIdx.x];
+        const int col = col0 + threadIdx.x;
+        const uint32_t word = __ballot_sync(0xffffffffu, c != 0u);
+        const int w = (col0 >> 5) + (threadIdx.x >> 5);
+        if (lane == 0 && w < o.C32) o.blk_mask[rb * o.C32 + w] = word;  // this CTA owns the block
+        if (acc) {
+          if (col < C) s_acc[col] += c;
+        } else {
+          // c is 0 for columns past C; all 32 lanes of both warps take part
+          if (c) atomicAdd(&o.col_nnz[col], c);
+          uint32_t sum = c;
+#pragma unroll
+          for (int s = 16; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
+          if (lane == 0 && sum) {
+            atomicAdd(&o.tile_nnz[ct], sum);
+            atomicAdd(o.nnz, (unsigned long long)sum);
+          }
+        }
+      }
+      __syncthreads();
+    }
   }
   cta_done(o, s_acc, acc);
 }
@@ -186,6 +249,8 @@ __global__ void __launch_bounds__(kTileThreads) stats_kernel(const __nv_bfloat16
 // ---------------------------------------------------------------------------
 __global__ void pad_kernel(const __nv_bfloat16* __restrict__ x, int64_t P, int C, int Cp,
                            __nv_bfloat16* __restrict__ y) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= P * Cp) return;
   const int64_t p = i / Cp;
@@ -198,13 +263,15 @@ __global__ void pad_kernel(const __nv_bfloat16* __restrict__ x, int64_t P, int C
 __global__ void __launch_bounds__(kTileThreads) dwconv_kernel(const DwArgs a_param) {
   const DwArgs a = a_param;  // registers, not parameter-space loads
   __shared__ uint32_t s_cnt[8 * 64];
-  __shared__ uint32_t s_acc[kMaxAccCols];
+  extern __shared__ uint32_t s_acc[];  // [C] when acc (dynamic)
   __shared__ __align__(16) float s_w[9][64];
   const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
   const int64_t R = (int64_t)a.N * a.Ho * a.Wo;
   const bool acc = a.emit && a.C <= kMaxAccCols;
-  if (a.path_out && blockIdx.x == 0 && threadIdx.x == 0) *a.path_out = 3;
   acc_init(s_acc, a.C, acc);
+  pdl_wait();
+  pdl_trigger();
+  if (a.path_out && blockIdx.x == 0 && threadIdx.x == 0) *a.path_out = 3;
   TileEmit e;
   e.init();
   const int hw = a.Ho * a.Wo;
@@ -281,11 +348,13 @@ __global__ void __launch_bounds__(kTileThreads)
                    int emit) {
   const OccDev o = o_param;
   __shared__ uint32_t s_cnt[8 * 64];
-  __shared__ uint32_t s_acc[kMaxAccCols];
+  extern __shared__ uint32_t s_acc[];  // [C] when acc (dynamic)
   const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
   const int64_t R = (int64_t)N * Ho * Wo;
   const bool acc = emit && C <= kMaxAccCols;
   acc_init(s_acc, C, acc);
+  pdl_wait();
+  pdl_trigger();
   TileEmit e;
   e.init();
   SPAROA_TILE_LOOP(R, C) {
@@ -333,10 +402,12 @@ __global__ void __launch_bounds__(kTileThreads)
                    __nv_bfloat16* __restrict__ y, OccDev o_param, int emit) {
   const OccDev o = o_param;
   __shared__ uint32_t s_cnt[8 * 64];
-  __shared__ uint32_t s_acc[kMaxAccCols];
+  extern __shared__ uint32_t s_acc[];  // [C] when acc (dynamic)
   const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
   const bool acc = emit && C <= kMaxAccCols;
   acc_init(s_acc, C, acc);
+  pdl_wait();
+  pdl_trigger();
   TileEmit e;
   e.init();
   SPAROA_TILE_LOOP((int64_t)N, C) {
@@ -375,10 +446,12 @@ __global__ void __launch_bounds__(kTileThreads)
   const OccDev o = o_param;
   const EpiDev ep = ep_param;
   __shared__ uint32_t s_cnt[8 * 64];
-  __shared__ uint32_t s_acc[kMaxAccCols];
+  extern __shared__ uint32_t s_acc[];  // [C] when acc (dynamic)
   const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
   const bool acc = emit && C <= kMaxAccCols;
   acc_init(s_acc, C, acc);
+  pdl_wait();
+  pdl_trigger();
   TileEmit e;
   e.init();
   SPAROA_TILE_LOOP(R, C) {
@@ -412,17 +485,28 @@ __global__ void __launch_bounds__(kTileThreads)
   if (emit) cta_done(o, s_acc, acc);
 }
 
+// Dynamic shared memory of a tile kernel: the per-CTA column counters.
+size_t acc_smem(int emit, int C) {
+  return (emit && C <= kMaxAccCols) ? sizeof(uint32_t) * (size_t)C : 0;
+}
+
+// Zero the word ranges of a ClearArgs (grid-stride over the longest range).
+__global__ void __launch_bounds__(256) clear_kernel(const ClearArgs a) {
+  pdl_wait();
+  pdl_trigger();
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+#pragma unroll
+  for (int k = 0; k < 5; ++k) {
+    uint32_t* p = a.p[k];
+    const int64_t n = a.words[k];
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) p[i] = 0u;
+  }
+}
+
 // Grid-stride over 128 x 64 tiles with at most 4 CTAs per SM.
 unsigned tile_grid(int64_t R, int C) {
-  static int sms = 0;
-  if (!sms) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
-      sms = 148;
-  }
   const int64_t tiles = ((R + 127) / 128) * ((C + 63) / 64);
-  const int64_t cap = 4LL * sms;
+  const int64_t cap = 4LL * device_sm_count();
   return (unsigned)(tiles < cap ? tiles : cap);
 }
 
@@ -430,23 +514,34 @@ unsigned tile_grid(int64_t R, int C) {
 
 cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev& o, cudaStream_t s) {
   if (R <= 0 || C <= 0) return cudaSuccess;
-  stats_kernel<<<tile_grid(R, C), kTileThreads, 0, s>>>(x, R, C, o);
-  return cudaGetLastError();
+  const int64_t nrb = (R + 127) / 128;
+  const int64_t cap = 4LL * device_sm_count();  // 4 CTAs per SM
+  const unsigned grid = (unsigned)(nrb < cap ? nrb : cap);
+  const size_t smem = C <= kMaxAccCols ? sizeof(uint32_t) * (size_t)C : 0;
+  return launch_kernel(stats_kernel, dim3(grid), dim3(kTileThreads), smem, s, x, R, C, o);
+}
+
+cudaError_t launch_clear(const ClearArgs& a, cudaStream_t s) {
+  int64_t mx = 0;
+  for (int k = 0; k < 5; ++k) mx = a.words[k] > mx ? a.words[k] : mx;
+  if (mx <= 0) return cudaSuccess;
+  const int64_t blocks = (mx + 255) / 256;
+  const int64_t cap = 2LL * device_sm_count();
+  return launch_kernel(clear_kernel, dim3((unsigned)(blocks < cap ? blocks : cap)), dim3(256), 0, s, a);
 }
 
 cudaError_t launch_pad_channels(const __nv_bfloat16* x, int64_t P, int C, int Cp,
                                 __nv_bfloat16* y, cudaStream_t s) {
   const int64_t n = P * Cp;
   if (n <= 0) return cudaSuccess;
-  pad_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(x, P, C, Cp, y);
-  return cudaGetLastError();
+  return launch_kernel(pad_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, x, P, C, Cp, y);
 }
 
 cudaError_t launch_dwconv(const DwArgs& a, cudaStream_t s) {
   const int64_t R = (int64_t)a.N * a.Ho * a.Wo;
   if (R <= 0) return cudaSuccess;
-  dwconv_kernel<<<tile_grid(R, a.C), kTileThreads, 0, s>>>(a);
-  return cudaGetLastError();
+  return launch_kernel(dwconv_kernel, dim3(tile_grid(R, a.C)), dim3(kTileThreads),
+                       acc_smem(a.emit, a.C), s, a);
 }
 
 cudaError_t launch_maxpool(const __nv_bfloat16* x, int N, int H, int W, int C, int k, int stride,
@@ -454,23 +549,22 @@ cudaError_t launch_maxpool(const __nv_bfloat16* x, int N, int H, int W, int C, i
                            cudaStream_t s) {
   const int64_t R = (int64_t)N * Ho * Wo;
   if (R <= 0) return cudaSuccess;
-  maxpool_kernel<<<tile_grid(R, C), kTileThreads, 0, s>>>(x, N, H, W, C, k, stride, pad, Ho, Wo,
-                                                          y, o, emit);
-  return cudaGetLastError();
+  return launch_kernel(maxpool_kernel, dim3(tile_grid(R, C)), dim3(kTileThreads), acc_smem(emit, C),
+                       s, x, N, H, W, C, k, stride, pad, Ho, Wo, y, o, emit);
 }
 
 cudaError_t launch_avgpool(const __nv_bfloat16* x, int N, int HW, int C, __nv_bfloat16* y,
                            const OccDev& o, int emit, cudaStream_t s) {
   if (N <= 0) return cudaSuccess;
-  avgpool_kernel<<<tile_grid(N, C), kTileThreads, 0, s>>>(x, N, HW, C, y, o, emit);
-  return cudaGetLastError();
+  return launch_kernel(avgpool_kernel, dim3(tile_grid(N, C)), dim3(kTileThreads), acc_smem(emit, C),
+                       s, x, N, HW, C, y, o, emit);
 }
 
 cudaError_t launch_bn_act(const __nv_bfloat16* x, int64_t R, int C, const EpiDev& ep,
                           __nv_bfloat16* y, const OccDev& o, int emit, cudaStream_t s) {
   if (R <= 0) return cudaSuccess;
-  bn_act_kernel<<<tile_grid(R, C), kTileThreads, 0, s>>>(x, R, C, ep, y, o, emit);
-  return cudaGetLastError();
+  return launch_kernel(bn_act_kernel, dim3(tile_grid(R, C)), dim3(kTileThreads), acc_smem(emit, C),
+                       s, x, R, C, ep, y, o, emit);
 }
 
 }  // namespace sparoa

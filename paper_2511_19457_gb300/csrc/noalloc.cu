@@ -91,7 +91,7 @@ extern "C" sparoa_status sparoa_gemm_noalloc(void* stream, const void* x, int64_
   if (!(t.s_thr == t.s_thr) || !(t.c_thr == t.c_thr) || t.intensity_mode < 0 ||
       t.intensity_mode > 1 || t.force_path < 0 || t.force_path > 2)
     return SPAROA_ERR_INVALID_ARG;
-  // the input occupancy must fit the static array
+  // the control words and the input occupancy must fit the static array
   const size_t occ_bytes = carve(nullptr, M, K, nullptr);
   if (kCtrlBytes + occ_bytes > kStaticScratchBytes) return SPAROA_ERR_UNSUPPORTED;
 
@@ -116,7 +116,14 @@ extern "C" sparoa_status sparoa_gemm_noalloc(void* stream, const void* x, int64_
   int32_t* path_slot = reinterpret_cast<int32_t*>(b + 16);
   OccDev xo;
   carve(b + kCtrlBytes, M, K, &xo);
-  if (cudaMemsetAsync(b, 0, kCtrlBytes + occ_bytes, s) != cudaSuccess) return SPAROA_ERR_CUDA;
+  {
+    // control words and the Eq. 1 counters (which start the occupancy block);
+    // the stats kernel writes the bitmaps whole
+    ClearArgs z = {};
+    z.p[0] = reinterpret_cast<uint32_t*>(b);
+    z.words[0] = (int64_t)((kCtrlBytes + (reinterpret_cast<char*>(xo.row_bm) - (b + kCtrlBytes))) / 4);
+    if (launch_clear(z, s) != cudaSuccess) return SPAROA_ERR_CUDA;
+  }
 
   const uint64_t flops = (uint64_t)2 * M * K * N;
   const uint64_t in_bytes = (uint64_t)M * K * 2;

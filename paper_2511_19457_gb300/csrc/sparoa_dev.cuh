@@ -204,6 +204,17 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
+// Programmatic dependent launch.  Every kernel of the library runs its
+// on-chip prologue (barrier init, TMEM allocation, tensor-map prefetch), then
+// pdl_wait(): the grid launched before it on the stream has completed and its
+// memory is visible.  No global memory is read or written before that wait.
+// pdl_trigger() right after lets the next grid start its own prologue while
+// this one works.  Both are no-ops for a launch without the attribute.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // Make generic-proxy writes to shared memory visible to the async proxy
 // (tensor cores / TMA).
 __device__ __forceinline__ void fence_proxy_async_smem() {

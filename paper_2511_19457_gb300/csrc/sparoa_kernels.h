@@ -10,6 +10,37 @@
 
 namespace sparoa {
 
+// Whether launches made by the calling host thread carry the programmatic
+// stream serialization attribute (set per C-ABI call from its context).
+bool pdl_enabled();
+void set_pdl_enabled(bool on);
+
+// Launch `kernel` on `s`, overlapping its prologue with the previous grid on
+// the stream when enabled (the kernel must call pdl_wait() before touching
+// global memory).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                          cudaStream_t s, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl_enabled() ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
+// Zero up to five word ranges (the fields of an occupancy block) in one launch.
+struct ClearArgs {
+  uint32_t* p[5];
+  int64_t words[5];
+};
+cudaError_t launch_clear(const ClearArgs& a, cudaStream_t s);
+
 // ----------------------------------------------------------------------------
 // Implicit-GEMM tensor-core kernel (dense path and zero-skip path)
 // ----------------------------------------------------------------------------
@@ -46,6 +77,9 @@ struct IgemmArgs {
 // Picks the N tile, encodes the tensor maps and launches.
 cudaError_t launch_igemm(const IgemmArgs& a, cudaStream_t s);
 
+// Streaming multiprocessors of the current device (cached per process).
+int device_sm_count();
+
 // conv = 2: the bw x bh x bn (= 128) output tile with the fewest padded pixels.
 void choose_spatial_tile(IgemmArgs& a);
 
@@ -76,7 +110,9 @@ cudaError_t launch_fcskip(const FcSkipArgs& a, cudaStream_t s);
 // ----------------------------------------------------------------------------
 // Memory-bound kernels (128-row x 64-channel tiles, occupancy fused)
 // ----------------------------------------------------------------------------
-// Eq. 1 statistics and bitmaps of x viewed as [R, C].
+// Eq. 1 statistics and bitmaps of x viewed as [R, C].  The row bitmaps and
+// block masks are written whole; the counters (nnz, col_nnz, tile_nnz) are
+// accumulated and must be zero on entry.
 cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev& o, cudaStream_t s);
 
 // Copy [P, C] to [P, Cp] with zero channels C..Cp-1.

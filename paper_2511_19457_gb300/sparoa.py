@@ -80,6 +80,7 @@ def _sig(name, args):
 _sig("sparoa_create", [ctypes.POINTER(_P), ctypes.c_int, _P])
 _sig("sparoa_destroy", [_P])
 _sig("sparoa_set_stream", [_P, _P])
+_sig("sparoa_set_overlap", [_P, _I32])
 _sig("sparoa_sync", [_P])
 _lib.sparoa_status_str.restype = ctypes.c_char_p
 _lib.sparoa_status_str.argtypes = [ctypes.c_int]
@@ -105,7 +106,7 @@ _sig("sparoa_run_graph", [_P, ctypes.POINTER(Op), _I32, _P, _I64, _I64, _I64, _I
 _sig("sparoa_gemm_noalloc", [_P, _P, _I64, _I64, _P, _P, _I64, ctypes.POINTER(Epilogue),
                              ctypes.POINTER(Thresholds), _P, _I32, ctypes.POINTER(Stats)])
 
-EXPORTED = ["sparoa_create", "sparoa_destroy", "sparoa_set_stream", "sparoa_sync",
+EXPORTED = ["sparoa_create", "sparoa_destroy", "sparoa_set_stream", "sparoa_set_overlap", "sparoa_sync",
             "sparoa_status_str", "sparoa_last_error", "sparoa_occupancy_bytes",
             "sparoa_occupancy_init", "sparoa_op_stats", "sparoa_gemm", "sparoa_conv2d",
             "sparoa_maxpool2d", "sparoa_avgpool_global", "sparoa_bn_act", "sparoa_run_graph",
@@ -163,6 +164,10 @@ class Context:
 
     def sync(self):
         self._check(_lib.sparoa_sync(self.h))
+
+    def set_overlap(self, enable: bool):
+        """Programmatic dependent launch between consecutive kernels (default on)."""
+        self._check(_lib.sparoa_set_overlap(self.h, 1 if enable else 0))
 
 
 class OccupancyBuffer:

@@ -68,6 +68,23 @@ def test_stats_bit_exact(sp, ctx, R, C, zp):
     assert_occ_equal(occ.to_host(), ref, f"stats {R}x{C}")
 
 
+def test_stats_needs_no_cleared_output_and_repeats(sp, ctx):
+    """The stats kernel writes every occupancy field (a buffer full of junk
+    comes out exact), and back-to-back launches on one context agree with the
+    oracle each time (its column accumulator is left clean), including more
+    row blocks than CTAs."""
+    for (R, C, zp, seed) in [(100352, 64, 0.5, 1), (100352, 64, 0.8, 2), (777, 136, 0.3, 3),
+                             (300, 4104, 0.6, 4)]:
+        bits = _bits((R, C), seed, zero_p=zp)
+        x = _dev(sp, bits, (R, C))
+        occ = sp.OccupancyBuffer(R, C)
+        occ.buf.fill_(0xA5)
+        st = sp.sparoa_op_stats(ctx, x, (R, C), occ=occ, host=True)
+        ref = orc.stats(bits, R, C)
+        assert st.nnz == ref.nnz
+        assert_occ_equal(occ.to_host(), ref, f"stats junk-filled {R}x{C}")
+
+
 def test_stats_reports_consumer_work(sp, ctx):
     d = synth.conv_layer(seed=0)
     x = _dev(sp, d["x"], (8, 56, 56, 64))
