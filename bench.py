@@ -35,6 +35,7 @@ if ROOT not in sys.path:
 
 METRIC = "effective TFLOP/s & % roofline per op; synthetic CNN images/s at batch 1/32"
 NBUF = 40   # rotating input/output sets per step, 40 x 6.6 MB > 129 MB L2
+LAUNCHES_PER_CONV_STEP = 4
 
 
 def parse_args():
@@ -397,7 +398,8 @@ def run_conv(args, rank, local_rank, world, peaks):
             "roofline": roof, "stats_kernel": stats_kernel,
             "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": R * C * 2,
                     "d2h_bytes_per_step": R * Co * 2, "steps": e2e_steps},
-            "gpu_launches": 2 * args.steps,
+            # per step: counter clear + stats kernel (input), clear + conv kernel (output)
+            "gpu_launches": LAUNCHES_PER_CONV_STEP * args.steps,
             "clocks": clocks.summary()}
     ctx.close()
     return line

@@ -24,8 +24,9 @@
 // whose activations are all zero.  Epilogue: bias / batch norm / residual /
 // activation, bf16 store, output occupancy.
 //
-// Warp roles (288 threads, persistent CTAs): warps 0-3 producers (thread 0
-// issues TMA; all compute skip masks), warps 4-7 epilogue, warp 8 MMA.
+// Warp roles (416 threads, persistent CTAs): warps 0-3 producers (thread 0
+// issues TMA; all compute skip masks), warps 4-11 epilogue (two per TMEM lane
+// quarter, 32 columns each), warp 12 MMA.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -50,7 +51,10 @@ int conv3_smem(int C, int Co, int W) {
 
 namespace {
 
-constexpr int kThreads = 288;
+constexpr int kEpiWarps = 8;                      // two per TMEM lane quarter, 32 columns each
+constexpr int kEpiThreads = 32 * kEpiWarps;
+constexpr int kMmaWarp = 4 + kEpiWarps;
+constexpr int kThreads = 32 * (kMmaWarp + 1);     // 4 producer warps, epilogue warps, MMA warp
 constexpr int kBM = 128;
 constexpr int kMaxPos = 1024;  // slab positions for the skip masks
 
@@ -101,6 +105,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* s_cnt = reinterpret_cast<uint32_t*>(s_shift + CO);                   // [4][CO]
   uint32_t* s_acc = s_cnt + 4 * CO;                                              // [CO]
   uint8_t* s_pos = reinterpret_cast<uint8_t*>(s_acc + CO);  // [kMaxPos] 1 = input pixel has a non-zero
+  unsigned long long* s_rowbm = reinterpret_cast<unsigned long long*>(s_pos + kMaxPos);  // [128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int N = G.N, H = G.H, W = G.W, C = G.C, Wp = G.Wp;
@@ -118,13 +123,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int b = 0; b < 2; ++b) {
       mbar_init(bar_empty + 8 * b, 1u);
       mbar_init(bar_accf + 8 * b, 1u);
-      mbar_init(bar_acce + 8 * b, 128u);
+      mbar_init(bar_acce + 8 * b, (uint32_t)kEpiThreads);
     }
     *s_abort = 0;
     prefetch_tmap(&tmX);
     prefetch_tmap(&tmW);
   }
-  if (warp == 8) tmem_alloc(smem_u32(s_tmem), (uint32_t)(2 * CO));
+  if (warp == kMmaWarp) tmem_alloc(smem_u32(s_tmem), (uint32_t)(2 * CO));
   pdl_wait();
   pdl_trigger();
   const int path = decide_path(P.disp);
@@ -135,15 +140,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int b = 0; b < 2; ++b) mbar_init(bar_full + 8 * b, skip ? 129u : 1u);
     fence_mbar_init();
   }
-  if (warp >= 4 && warp < 8) {
+  if (warp >= 4 && warp < kMmaWarp) {
     const int et = threadIdx.x - 128;
-    for (int c = et; c < CO; c += 128) {
+    for (int c = et; c < CO; c += kEpiThreads) {
       float sc = 1.f, sh = 0.f;
       if (c < G.Co) epi_affine(P.ep, G.Co, c, sc, sh);
       s_scale[c] = sc;
       s_shift[c] = sh;
       s_acc[c] = 0u;
     }
+    for (int i = et; i < kBM; i += kEpiThreads) s_rowbm[i] = 0ull;
   }
   tc_fence_before();
   __syncthreads();
@@ -222,7 +228,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (named_bar_or(1, 128, !ok)) break;
       mbar_arrive(bar_full + 8 * b);  // 128 mask arrivals + the TMA's expect_tx arrival
     }
-  } else if (warp == 8) {
+  } else if (warp == kMmaWarp) {
     // -------------------------------------------------------------- MMA issue
     // The whole warp walks the tiles so that it stays converged between tiles;
     // lane 0 waits, issues the MMAs and commits.
@@ -294,9 +300,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // -------------------------------------------------------------- epilogue
+    // warp w reads TMEM lanes 32 (w % 4).. (its quarter of the tile's rows) and
+    // the 32 accumulator columns 32 ((w - 4) / 4)..
     const int q = warp & 3, r = q * 32 + lane, et = threadIdx.x - 128;
+    const int c0 = ((warp - 4) >> 2) * 32;
     const OccDev o = P.out_occ;
     const bool acc_smem = emit != 0;
+    const bool affine = P.ep.bias != nullptr || P.ep.bn != nullptr;  // else the column affine is 1, 0
     int j = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++j) {
       const int b = j & 1;
@@ -305,17 +315,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int oh = qq / Wp, ow = qq - (qq / Wp) * Wp;
       const bool mvalid = oh < H && ow < W;
       const int64_t m = ((int64_t)img * H + oh) * W + ow;
-      bool ok = mbar_wait(bar_accf + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutAcc);
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok) break;
+      const bool ok = mbar_wait(bar_accf + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutAcc);
+      // the same abort decision for every epilogue warp (one that left alone
+      // would strand the others at the occupancy barrier)
+      if (named_bar_or(2, kEpiThreads, !ok)) break;
       tc_fence_after();
       const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * CO);
       const int blk = mvalid ? (int)(m >> 7) : -1;
       const uint32_t grp = __match_any_sync(0xffffffffu, blk);
       const bool leader = (__ffs(grp) - 1) == lane;
       unsigned long long tl = 0ull;
-#pragma unroll 1
-      for (int c0 = 0; c0 < CO; c0 += 32) {
+      {
         uint32_t raw[32];
         tmem_ld32_nowait(tbase + (uint32_t)c0, raw);
         tmem_wait_ld32(raw);
@@ -324,14 +334,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int h = 0; h < 2; ++h) {
           const int cc = c0 + h * 16;
           float v[16];
+          if (affine) {
 #pragma unroll
-          for (int q4 = 0; q4 < 4; ++q4) {
-            const float4 sc = reinterpret_cast<const float4*>(s_scale + cc)[q4];
-            const float4 sh = reinterpret_cast<const float4*>(s_shift + cc)[q4];
-            v[4 * q4 + 0] = fmaf(__uint_as_float(raw[h * 16 + 4 * q4 + 0]), sc.x, sh.x);
-            v[4 * q4 + 1] = fmaf(__uint_as_float(raw[h * 16 + 4 * q4 + 1]), sc.y, sh.y);
-            v[4 * q4 + 2] = fmaf(__uint_as_float(raw[h * 16 + 4 * q4 + 2]), sc.z, sh.z);
-            v[4 * q4 + 3] = fmaf(__uint_as_float(raw[h * 16 + 4 * q4 + 3]), sc.w, sh.w);
+            for (int q4 = 0; q4 < 4; ++q4) {
+              const float4 sc = reinterpret_cast<const float4*>(s_scale + cc)[q4];
+              const float4 sh = reinterpret_cast<const float4*>(s_shift + cc)[q4];
+              v[4 * q4 + 0] = fmaf(__uint_as_float(raw[h * 16 + 4 * q4 + 0]), sc.x, sh.x);
+              v[4 * q4 + 1] = fmaf(__uint_as_float(raw[h * 16 + 4 * q4 + 1]), sc.y, sh.y);
+              v[4 * q4 + 2] = fmaf(__uint_as_float(raw[h * 16 + 4 * q4 + 2]), sc.z, sh.z);
+              v[4 * q4 + 3] = fmaf(__uint_as_float(raw[h * 16 + 4 * q4 + 3]), sc.w, sh.w);
+            }
+          } else {
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj) v[jj] = __uint_as_float(raw[h * 16 + jj]);
           }
           if (residual && mvalid) {
             const uint4* rp = reinterpret_cast<const uint4*>(residual + m * G.Co + cc);
@@ -381,17 +396,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_before();
       mbar_arrive(bar_acce + 8 * b);
       if (emit) {
-        if (mvalid && tl) atomicOr(&o.row_bm[m * o.W64], tl);
-        named_bar_sync(2, 128);
-        for (int c = et; c < CO; c += 128)
+        // both column halves of a row meet in shared memory; the tile owns its
+        // output rows, so the half-0 thread stores the word once
+        if (tl) atomicOr(&s_rowbm[r], tl);
+        named_bar_sync(2, kEpiThreads);
+        if (c0 == 0) {
+          const unsigned long long v = s_rowbm[r];
+          s_rowbm[r] = 0ull;
+          if (mvalid) o.row_bm[m * o.W64] = v;
+        }
+        for (int c = et; c < CO; c += kEpiThreads)
           s_acc[c] += s_cnt[c] + s_cnt[CO + c] + s_cnt[2 * CO + c] + s_cnt[3 * CO + c];
-        named_bar_sync(2, 128);
+        named_bar_sync(2, kEpiThreads);
       }
     }
     if (emit && acc_smem) {
       unsigned long long total = 0ull;
-      for (int c0 = 0; c0 < CO; c0 += 128) {
-        const int c = c0 + et;
+      for (int cb0 = 0; cb0 < CO; cb0 += kEpiThreads) {
+        const int c = cb0 + et;
         const uint32_t cnt = c < CO ? s_acc[c] : 0u;
         if (cnt) atomicAdd(&o.col_nnz[c], cnt);
         uint32_t sum = cnt;
@@ -407,7 +429,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncwarp();  // lanes that finished early wait for their warp's working lane
   tc_fence_before();
   __syncthreads();
-  if (warp == 8) {
+  if (warp == kMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, (uint32_t)(2 * CO));
   }

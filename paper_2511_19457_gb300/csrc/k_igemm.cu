@@ -31,9 +31,10 @@
 // The epilogue applies bias / batch norm / residual / activation, stores y and
 // writes y's Eq. 1 count and occupancy bitmaps for the next operator.
 //
-// Warp roles (288 threads): warps 0-3 producers (the skip masks; thread 0
-// issues TMA; all 128 gather in mode 1), warps 4-7 epilogue (TMEM lane
-// quarters), warp 8 TMEM allocation and MMA issue (lane 0).
+// Warp roles (416 threads): warps 0-3 producers (the skip masks; thread 0
+// issues TMA; all 128 gather in mode 1), warps 4-11 epilogue (two per TMEM
+// lane quarter, each taking 32 of every 64 accumulator columns), warp 12 TMEM
+// allocation and MMA issue (lane 0).
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -45,11 +46,15 @@ namespace sparoa {
 
 namespace {
 
-constexpr int kThreads = 288;
+constexpr int kEpiWarps = 8;                   // two per TMEM lane quarter, 32 of each 64 columns
+constexpr int kEpiThreads = 32 * kEpiWarps;
+constexpr int kMmaWarp = 4 + kEpiWarps;
+constexpr int kThreads = 32 * (kMmaWarp + 1);  // 4 producer warps, epilogue warps, MMA warp
 constexpr int kBM = 128;
 constexpr int kMaxKWords = 128;  // K-block occupancy bits: up to 4096 blocks
 constexpr int kMaxTaps = 64;
-constexpr int kStgBytes = 128 * 128;  // one 128-row x 128-byte output staging tile
+constexpr int kStgBytes = 128 * 128;  // output staging: per epilogue warp 2 blocks of 32 rows x 64 bytes
+constexpr int kWarpStgBytes = 32 * 64;
 constexpr int kMaxAccCols = 2048;     // per-CTA column counters (output occupancy)
 
 template <int BN, int BK>
@@ -70,10 +75,12 @@ struct Cfg {
   static constexpr int kKBitsOff = (kFlagOff + (kStages + 8) * 4 + 15) & ~15;
   static constexpr int kTapOff = kKBitsOff + kMaxKWords * 4;
   static constexpr int kScaleOff = kTapOff + kMaxTaps * 8;
-  static constexpr int kShiftOff = kScaleOff + BN * 4;
-  static constexpr int kCntOff = kShiftOff + BN * 4;
+  static constexpr int kShiftOff = kScaleOff + 2 * BN * 4;  // scale / shift: [2 accumulators][BN]
+  static constexpr int kCntOff = kShiftOff + 2 * BN * 4;
   static constexpr int kAccOff = kCntOff + 4 * BN * 4;
-  static constexpr int kBytes = kAccOff + kMaxAccCols * 4 + 16;
+  static constexpr int kRowOff = kAccOff + kMaxAccCols * 4;   // [128] row bits of the tile
+  static constexpr int kBlkOff = kRowOff + kBM * 8;           // [BN / 32] block-mask words
+  static constexpr int kBytes = kBlkOff + (BN / 32) * 4 + 16;
   static constexpr int kSmem = kBytes + 1024;  // slack for 1024-byte alignment
   static_assert(kStages >= 2, "stages");
   static_assert(kSmem <= 227 * 1024, "shared memory");
@@ -192,6 +199,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t sShift = sbase + C::kShiftOff;
   uint32_t* s_cnt = reinterpret_cast<uint32_t*>(smem + C::kCntOff);  // [4][BN]
   uint32_t* s_acc = reinterpret_cast<uint32_t*>(smem + C::kAccOff);  // [N] non-zeros per column
+  unsigned long long* s_rowbm = reinterpret_cast<unsigned long long*>(smem + C::kRowOff);
+  uint32_t* s_blk = reinterpret_cast<uint32_t*>(smem + C::kBlkOff);
   // Column counts of all tiles a CTA handles are summed here and flushed once
   // (atomics on one address from every tile would serialise in L2).
   const bool acc_smem = emit && p.N <= kMaxAccCols;
@@ -210,7 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(bar_accf + 8 * b, 1u);
-      mbar_init(bar_acce + 8 * b, 128u);
+      mbar_init(bar_acce + 8 * b, (uint32_t)kEpiThreads);
     }
     *s_abort = 0;
     fence_mbar_init();
@@ -218,9 +227,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tmap(&tmB);
     if (!y_f32) prefetch_tmap(&tmY);
   }
-  if (warp == 8) tmem_alloc(smem_u32(s_tmem), (uint32_t)(2 * BN));
-  if (acc_smem && warp >= 4 && warp < 8)
-    for (int c = threadIdx.x - 128; c < p.N; c += 128) s_acc[c] = 0u;
+  if (warp == kMmaWarp) tmem_alloc(smem_u32(s_tmem), (uint32_t)(2 * BN));
+  if (acc_smem && warp >= 4 && warp < kMmaWarp)
+    for (int c = threadIdx.x - 128; c < p.N; c += kEpiThreads) s_acc[c] = 0u;
+  if (warp >= 4 && warp < kMmaWarp) {
+    for (int i = threadIdx.x - 128; i < kBM; i += kEpiThreads) s_rowbm[i] = 0ull;
+    for (int i = threadIdx.x - 128; i < BN / 32; i += kEpiThreads) s_blk[i] = 0u;
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -399,7 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       fence_proxy_async_smem();
       for (int q = pending; q > 0; --q) mbar_arrive(bar_full + 8 * ((it - q) % S));
     }
-  } else if (warp == 8) {
+  } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------------ MMA issue
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(kBM, BN);
@@ -448,29 +461,51 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------------ epilogue
+    // Each epilogue warp owns a 32-row x 32-column block of every 64-column
+    // group (rows from its TMEM lane quarter, columns from its half) and
+    // stores it on its own: staging in shared memory with the 64-byte swizzle
+    // and one TMA store per block, so the warps never wait for each other
+    // inside a tile.  The only barrier per tile publishes the column affine
+    // (double-buffered by accumulator), plus one for the output occupancy.
     const int q = warp & 3;            // TMEM lane quarter of this warp
+    const int hf = (warp - 4) >> 2;    // which 32 columns of each 64-column group
+    const int ew = warp - 4;           // epilogue warp index
     const int r = q * 32 + lane;       // tile row
-    const int et = threadIdx.x - 128;  // 0..127
+    const int et = threadIdx.x - 128;  // 0..kEpiThreads-1
     const bool vec = (p.N % 8) == 0;
+    const bool affine = ep.bias != nullptr || ep.bn != nullptr;  // else the column affine is 1, 0
+    // this warp's 32-row sub-box of the tile: {32 channels, bw', bh', bn'} for
+    // spatial tiles, 32 consecutive rows otherwise
+    int sw_ = 0, sh_ = 0, sn_ = 0;
+    if (p.conv == 2) {
+      const int rho = q * 32;
+      sw_ = rho % p.bw;
+      sh_ = (rho / p.bw) % p.bh;
+      sn_ = rho / (p.bw * p.bh);
+    }
+    const uint32_t stg_base = sStg + (uint32_t)(ew * 2 * kWarpStgBytes);
     int j = 0;
-    int stg_count = 0;  // staging tiles handed to TMA so far
+    int stg_count = 0;  // blocks this warp handed to TMA so far
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++j) {
       const int b = j & 1;
       const TileGeo g = tile_geo(p, t, nt, BN);
       bool mvalid;
       int img, oh, ow;
       const int64_t m = tile_row(p, g, r, mvalid, img, oh, ow);
-      // per-tile column affine (the previous tile's readers are past its last barrier)
-      for (int c = et; c < BN; c += 128) {
+      float* const scb = s_scale + b * BN;
+      float* const shb = s_shift + b * BN;
+      // column affine of this tile into buffer b (its readers of tile j - 2
+      // passed tile j - 1's barrier before any thread gets here)
+      for (int c = et; c < BN; c += kEpiThreads) {
         float sc = 1.f, sh = 0.f;
         if (g.n0 + c < p.N) epi_affine(ep, p.N, g.n0 + c, sc, sh);
-        s_scale[c] = sc;
-        s_shift[c] = sh;
+        scb[c] = sc;
+        shb[c] = sh;
       }
-      bool ok = mbar_wait(bar_accf + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutAcc);
-      ok = __all_sync(0xffffffffu, ok);
-      named_bar_sync(2, 128);
-      if (!ok) break;
+      const bool ok = mbar_wait(bar_accf + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutAcc);
+      // publishes the affine, and makes the abort decision the same for every
+      // epilogue warp (a warp that left alone would strand the others at a barrier)
+      if (named_bar_or(2, kEpiThreads, !ok)) break;
       tc_fence_after();
       const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * BN);
       const OccDev o = P.out_occ;  // registers, not parameter-space loads
@@ -484,129 +519,159 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int gcol = 0; gcol < BN / 64; ++gcol) {
         const int nbase = g.n0 + gcol * 64;
         if (nbase >= p.N) break;  // uniform across the epilogue warps
+        const int ncol0 = nbase + hf * 32;  // first column of this warp's block
         uint32_t stg = 0;
         if (!y_f32) {
-          stg = sStg + (uint32_t)((stg_count & 1) * kStgBytes);
-          if (et == 0) bulk_wait_read<1>();  // the store that used this buffer has read it
-          named_bar_sync(2, 128);
+          stg = stg_base + (uint32_t)((stg_count & 1) * kWarpStgBytes);
+          if (lane == 0) bulk_wait_read<1>();  // the store that used this buffer has read it
+          __syncwarp();
         }
-        uint32_t raw2[2][32];
-        tmem_ld32_nowait(tbase + (uint32_t)(gcol * 64), raw2[0]);
-        tmem_ld32_nowait(tbase + (uint32_t)(gcol * 64 + 32), raw2[1]);
-        tmem_wait_ld32(raw2[0]);
-        tmem_wait_ld32(raw2[1]);
-        uint32_t rwg[2] = {0u, 0u};  // non-zero bits of this row in the group's two 32-column words
+        uint32_t raw[32];
+        tmem_ld32_nowait(tbase + (uint32_t)(gcol * 64 + hf * 32), raw);
+        tmem_wait_ld32(raw);
+        uint32_t rw = 0u;  // non-zero bits of this row in the warp's 32 columns
+        const float* scg = scb + gcol * 64 + hf * 32;
+        const float* shg = shb + gcol * 64 + hf * 32;
 #pragma unroll
-        for (int half = 0; half < 2; ++half) {
-#pragma unroll
-          for (int c16s = 0; c16s < 2; ++c16s) {
-            const int cg0 = half * 32 + c16s * 16;  // column inside the group
-            const int nb = nbase + cg0;
-            const bool full = vec && (nb + 16 <= p.N);
-            const float4* sc4 = reinterpret_cast<const float4*>(s_scale + gcol * 64 + cg0);
-            const float4* sh4 = reinterpret_cast<const float4*>(s_shift + gcol * 64 + cg0);
-            float o32[16];
+        for (int c16s = 0; c16s < 2; ++c16s) {
+          const int nb = ncol0 + c16s * 16;
+          const bool full = vec && (nb + 16 <= p.N);
+          const float4* sc4 = reinterpret_cast<const float4*>(scg + c16s * 16);
+          const float4* sh4 = reinterpret_cast<const float4*>(shg + c16s * 16);
+          float o32[16];
+          if (affine) {
 #pragma unroll
             for (int q4 = 0; q4 < 4; ++q4) {
               const float4 sc = sc4[q4];
               const float4 sh = sh4[q4];
-              o32[4 * q4 + 0] = fmaf(__uint_as_float(raw2[half][c16s * 16 + 4 * q4 + 0]), sc.x, sh.x);
-              o32[4 * q4 + 1] = fmaf(__uint_as_float(raw2[half][c16s * 16 + 4 * q4 + 1]), sc.y, sh.y);
-              o32[4 * q4 + 2] = fmaf(__uint_as_float(raw2[half][c16s * 16 + 4 * q4 + 2]), sc.z, sh.z);
-              o32[4 * q4 + 3] = fmaf(__uint_as_float(raw2[half][c16s * 16 + 4 * q4 + 3]), sc.w, sh.w);
+              o32[4 * q4 + 0] = fmaf(__uint_as_float(raw[c16s * 16 + 4 * q4 + 0]), sc.x, sh.x);
+              o32[4 * q4 + 1] = fmaf(__uint_as_float(raw[c16s * 16 + 4 * q4 + 1]), sc.y, sh.y);
+              o32[4 * q4 + 2] = fmaf(__uint_as_float(raw[c16s * 16 + 4 * q4 + 2]), sc.z, sh.z);
+              o32[4 * q4 + 3] = fmaf(__uint_as_float(raw[c16s * 16 + 4 * q4 + 3]), sc.w, sh.w);
             }
-            if (residual && mvalid) {
-              const __nv_bfloat16* rp = residual + m * p.N + nb;
-              if (full) {
-                const uint4 r0 = *reinterpret_cast<const uint4*>(rp);
-                const uint4 r1 = *reinterpret_cast<const uint4*>(rp + 8);
-                const __nv_bfloat162* h0 = reinterpret_cast<const __nv_bfloat162*>(&r0);
-                const __nv_bfloat162* h1 = reinterpret_cast<const __nv_bfloat162*>(&r1);
+          } else {
 #pragma unroll
-                for (int jj = 0; jj < 4; ++jj) {
-                  const float2 a0 = __bfloat1622float2(h0[jj]);
-                  const float2 a1 = __bfloat1622float2(h1[jj]);
-                  o32[2 * jj] += a0.x;
-                  o32[2 * jj + 1] += a0.y;
-                  o32[8 + 2 * jj] += a1.x;
-                  o32[8 + 2 * jj + 1] += a1.y;
-                }
-              } else {
-                for (int jj = 0; jj < 16; ++jj)
-                  if (nb + jj < p.N) o32[jj] += __bfloat162float(rp[jj]);
-              }
-            }
-            if (act == 1) {
+            for (int jj = 0; jj < 16; ++jj) o32[jj] = __uint_as_float(raw[c16s * 16 + jj]);
+          }
+          if (residual && mvalid) {
+            const __nv_bfloat16* rp = residual + m * p.N + nb;
+            if (full) {
+              const uint4 r0 = *reinterpret_cast<const uint4*>(rp);
+              const uint4 r1 = *reinterpret_cast<const uint4*>(rp + 8);
+              const __nv_bfloat162* h0 = reinterpret_cast<const __nv_bfloat162*>(&r0);
+              const __nv_bfloat162* h1 = reinterpret_cast<const __nv_bfloat162*>(&r1);
 #pragma unroll
-              for (int jj = 0; jj < 16; ++jj) o32[jj] = o32[jj] > 0.f ? o32[jj] : 0.f;
-            } else if (act == 2) {
-#pragma unroll
-              for (int jj = 0; jj < 16; ++jj) o32[jj] = o32[jj] > 0.f ? (o32[jj] < 6.f ? o32[jj] : 6.f) : 0.f;
-            }
-            if (y_f32) {
-              if (mvalid) {
-                float* yp = reinterpret_cast<float*>(yout) + m * p.N + nb;
-                if (full && (p.N % 4) == 0) {
-#pragma unroll
-                  for (int jj = 0; jj < 16; jj += 4)
-                    *reinterpret_cast<float4*>(yp + jj) = make_float4(o32[jj], o32[jj + 1], o32[jj + 2], o32[jj + 3]);
-                } else {
-                  for (int jj = 0; jj < 16; ++jj)
-                    if (nb + jj < p.N) yp[jj] = o32[jj];
-                }
+              for (int jj = 0; jj < 4; ++jj) {
+                const float2 a0 = __bfloat1622float2(h0[jj]);
+                const float2 a1 = __bfloat1622float2(h1[jj]);
+                o32[2 * jj] += a0.x;
+                o32[2 * jj + 1] += a0.y;
+                o32[8 + 2 * jj] += a1.x;
+                o32[8 + 2 * jj + 1] += a1.y;
               }
             } else {
-              uint32_t pk[8];
-              uint32_t nzbits = 0;
+              for (int jj = 0; jj < 16; ++jj)
+                if (nb + jj < p.N) o32[jj] += __bfloat162float(rp[jj]);
+            }
+          }
+          if (act == 1) {
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj) o32[jj] = fmaxf(o32[jj], 0.f);
+          } else if (act == 2) {
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj) o32[jj] = fminf(fmaxf(o32[jj], 0.f), 6.f);
+          }
+          if (y_f32) {
+            if (mvalid) {
+              float* yp = reinterpret_cast<float*>(yout) + m * p.N + nb;
+              if (full && (p.N % 4) == 0) {
+#pragma unroll
+                for (int jj = 0; jj < 16; jj += 4)
+                  *reinterpret_cast<float4*>(yp + jj) = make_float4(o32[jj], o32[jj + 1], o32[jj + 2], o32[jj + 3]);
+              } else {
+                for (int jj = 0; jj < 16; ++jj)
+                  if (nb + jj < p.N) yp[jj] = o32[jj];
+              }
+            }
+          } else {
+            uint32_t pk[8];
+#pragma unroll
+            for (int jj = 0; jj < 8; ++jj) {
+              const __nv_bfloat162 h2 = __floats2bfloat162_rn(o32[2 * jj], o32[2 * jj + 1]);
+              pk[jj] = *reinterpret_cast<const uint32_t*>(&h2);
+            }
+            if (emit) {
+              uint32_t nzbits = 0u;
 #pragma unroll
               for (int jj = 0; jj < 8; ++jj) {
-                const __nv_bfloat162 h2 = __floats2bfloat162_rn(o32[2 * jj], o32[2 * jj + 1]);
-                pk[jj] = *reinterpret_cast<const uint32_t*>(&h2);
                 nzbits |= ((pk[jj] & 0x7FFFu) ? 1u : 0u) << (2 * jj);
                 nzbits |= ((pk[jj] & 0x7FFF0000u) ? 1u : 0u) << (2 * jj + 1);
               }
               const int nvalid = p.N - nb;  // columns of this chunk inside the tensor
-              if (!mvalid) nzbits = 0;
+              if (!mvalid) nzbits = 0u;
               else if (nvalid < 16) nzbits &= nvalid > 0 ? ((1u << nvalid) - 1u) : 0u;
-              rwg[half] |= nzbits << (c16s * 16);
-              // staging tile: 128 rows x 128 bytes with the 128-byte swizzle the TMA store reads
-              const uint32_t row_addr = stg + (uint32_t)r * 128u;
-              const int j0 = (half * 2 + c16s) * 2;
-              sts_u4(row_addr + (uint32_t)((j0 ^ (r & 7)) << 4), make_uint4(pk[0], pk[1], pk[2], pk[3]));
-              sts_u4(row_addr + (uint32_t)(((j0 + 1) ^ (r & 7)) << 4), make_uint4(pk[4], pk[5], pk[6], pk[7]));
+              rw |= nzbits << (c16s * 16);
             }
+            // staging block: 32 rows x 64 bytes, 16-byte chunk k of row `lane` at
+            // chunk k ^ ((lane >> 1) & 3) (the TMA 64-byte swizzle)
+            const uint32_t row_addr = stg + (uint32_t)lane * 64u;
+            const int k0 = c16s * 2;
+            const int sx = (lane >> 1) & 3;
+            sts_u4(row_addr + (uint32_t)((k0 ^ sx) << 4), make_uint4(pk[0], pk[1], pk[2], pk[3]));
+            sts_u4(row_addr + (uint32_t)(((k0 + 1) ^ sx) << 4), make_uint4(pk[4], pk[5], pk[6], pk[7]));
           }
         }
         if (!y_f32) {
           fence_proxy_async_smem();
-          named_bar_sync(2, 128);
-          if (et == 0) {
-            if (p.conv == 2) tma_store_4d(&tmY, stg, nbase, g.tw0, g.th0, g.tn0);
-            else tma_store_2d(&tmY, stg, nbase, g.m0);
+          __syncwarp();
+          if (lane == 0) {
+            if (p.conv == 2)
+              tma_store_4d(&tmY, stg, ncol0, g.tw0 + sw_, g.th0 + sh_, g.tn0 + sn_);
+            else
+              tma_store_2d(&tmY, stg, ncol0, g.m0 + q * 32);
             bulk_commit();
           }
           ++stg_count;
         }
         if (emit) {
-          // this group's share of the output occupancy
-          if (rwg[0] | rwg[1]) tl |= 1ull << ((nbase >> 6) & 63);
-#pragma unroll
-          for (int w = 0; w < 2; ++w) {
-            const uint32_t bits = __reduce_or_sync(grp, rwg[w]);
-            const int word = (nbase >> 5) + w;
-            if (leader && blk >= 0 && bits && word < o.C32) atomicOr(&o.blk_mask[blk * o.C32 + word], bits);
-            // lane j: non-zeros of column 32w + j of this group in the warp's 32 rows
-            s_cnt[q * BN + gcol * 64 + w * 32 + lane] = __popc(warp_transpose32(rwg[w]));
+          // this block's share of the output occupancy
+          if (rw) tl |= 1ull << ((nbase >> 6) & 63);
+          const uint32_t bits = __reduce_or_sync(grp, rw);
+          const int word = (nbase >> 5) + hf;
+          if (leader && blk >= 0 && bits && word < o.C32) {
+            if (p.conv == 2) atomicOr(&o.blk_mask[blk * o.C32 + word], bits);
+            else atomicOr(&s_blk[gcol * 2 + hf], bits);  // the tile is the whole block
           }
+          // lane j: non-zeros of column 32 hf + j of this group in the warp's 32 rows
+          s_cnt[q * BN + gcol * 64 + hf * 32 + lane] = __popc(warp_transpose32(rw));
         }
       }
       // accumulator b is free for the MMA of tile j + 2
       tc_fence_before();
       mbar_arrive(bar_acce + 8 * b);
       if (emit) {
-        if (mvalid && tl) atomicOr(&o.row_bm[m * o.W64 + ((g.n0 >> 6) >> 6)], tl);
-        named_bar_sync(2, 128);
-        for (int c = et; c < BN; c += 128) {
+        // both column halves of a row meet in shared memory; the half-0 thread of
+        // the row then writes it once (a plain store when the tile spans every
+        // column of the row's bitmap word, i.e. the word is this tile's alone)
+        if (tl) atomicOr(&s_rowbm[r], tl);
+        named_bar_sync(2, kEpiThreads);
+        if (hf == 0) {
+          const unsigned long long v = s_rowbm[r];
+          s_rowbm[r] = 0ull;
+          if (mvalid) {
+            unsigned long long* dst = &o.row_bm[m * o.W64 + ((g.n0 >> 6) >> 6)];
+            if (nt == 1) *dst = v;
+            else if (v) atomicOr(dst, v);
+          }
+        }
+        if (p.conv != 2 && et < BN / 32) {
+          const uint32_t v = s_blk[et];
+          s_blk[et] = 0u;
+          const int word = (g.n0 >> 5) + et;
+          // rows m0.. m0+127 are one whole block and columns n0.. are this tile's
+          if (word < o.C32) o.blk_mask[(g.m0 >> 7) * o.C32 + word] = v;
+        }
+        for (int c = et; c < BN; c += kEpiThreads) {
           const bool live = g.n0 + c < o.C;
           const uint32_t cnt =
               live ? s_cnt[c] + s_cnt[BN + c] + s_cnt[2 * BN + c] + s_cnt[3 * BN + c] : 0u;
@@ -624,14 +689,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      named_bar_sync(2, 128);  // s_scale / s_cnt / staging reuse by the next tile
     }
     if (acc_smem) {
       // flush the CTA's column counts: per column, per 64-column tile, total
-      named_bar_sync(2, 128);
+      named_bar_sync(2, kEpiThreads);
       const OccDev& o = P.out_occ;
       unsigned long long total = 0ull;
-      for (int c0 = 0; c0 < p.N; c0 += 128) {
+      for (int c0 = 0; c0 < p.N; c0 += kEpiThreads) {
         const int c = c0 + et;
         const uint32_t cnt = c < p.N ? s_acc[c] : 0u;
         if (cnt) atomicAdd(&o.col_nnz[c], cnt);
@@ -643,13 +707,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (lane == 0 && total) atomicAdd(o.nnz, total);
     }
-    if (et == 0) bulk_wait_all();
+    if (lane == 0) bulk_wait_all();
   }
 
   __syncwarp();  // lanes that finished early wait for their warp's working lane
   tc_fence_before();
   __syncthreads();
-  if (warp == 8) {
+  if (warp == kMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, (uint32_t)(2 * BN));
   }
@@ -791,9 +855,14 @@ cudaError_t launch_igemm(const IgemmArgs& a, cudaStream_t s) {
   if (!make_tmap_2d(&tB, a.w, (uint64_t)a.N, (uint64_t)a.Ktot, (uint32_t)bk, (uint32_t)bn))
     return cudaErrorInvalidValue;
   if (!a.y_f32) {
+    // one epilogue warp's block: 32 columns x 32 tile rows (for spatial tiles
+    // the sub-box {bw', bh', bn'} of 32 pixels that the rows form)
+    const int sbw = a.bw < 32 ? a.bw : 32;
+    const int sbh = a.bh < 32 / sbw ? a.bh : 32 / sbw;
+    const int sbn = 32 / (sbw * sbh);
     bool okY = a.conv == 2
-                   ? make_tmap_nhwc(&tY, a.y, a.Nimg, a.Ho, a.Wo, a.N, 64, a.bw, a.bh, a.bn, 1)
-                   : make_tmap_2d(&tY, a.y, (uint64_t)a.M, (uint64_t)a.N, 64, kBM);
+                   ? make_tmap_nhwc(&tY, a.y, a.Nimg, a.Ho, a.Wo, a.N, 32, sbw, sbh, sbn, 1)
+                   : make_tmap_2d(&tY, a.y, (uint64_t)a.M, (uint64_t)a.N, 32, 32);
     if (!okY) return cudaErrorInvalidValue;
   }
   if (a.conv == 1) tA = tB;  // unused by the gather producers

@@ -216,6 +216,11 @@ CONV_CASES = [
     (2, 9, 11, 144, 32, 1, 1, 0, 2, False),    # K = 144 (ragged 32-block)
     (2, 10, 10, 24, 144, 3, 1, 1, 2, False),   # C_in 24: blocks straddle taps
     (1, 7, 7, 512, 512, 3, 1, 1, 1, True),
+    # spatial output tiles whose 32-row epilogue blocks are {4 w, 4 h, 2 images},
+    # {32 of 128 w}, and several whole images
+    (8, 6, 6, 64, 64, 3, 2, 1, 1, False),
+    (1, 8, 128, 64, 128, 3, 1, 1, 1, True),
+    (32, 8, 8, 64, 64, 3, 2, 1, 0, False),
 ]
 
 
