@@ -38,6 +38,7 @@ struct sparoa_ctx {
   DevBuf occ;         // occupancy of inputs measured inside a call
   DevBuf pad_x, pad_w;
   DevBuf arena;       // sparoa_run_graph activations, occupancies, paths
+  DevBuf splitk;      // split-K arrival counters (kept zero) + fp32 partial tiles
   std::vector<sparoa_occupancy> graph_occ;
   int overlap = 1;    // programmatic dependent launch between consecutive kernels
   uint32_t* d_err() const { return reinterpret_cast<uint32_t*>(small.p); }
@@ -188,6 +189,22 @@ sparoa_status occ_clear(sparoa_ctx* ctx, const sparoa_occupancy& o, bool counter
     a.words[4] = RB * C32;
   }
   SP_CUDA(launch_clear(a, ctx->stream));
+  return SPAROA_OK;
+}
+
+// Split-K scratch offered to the implicit-GEMM kernel: 65536 arrival counters
+// (zeroed once when allocated; every launch leaves them zero) and 64 MiB of
+// fp32 partial tiles.  Allocated with the context.
+constexpr int kSplitCounters = 65536;
+constexpr size_t kSplitCntBytes = sizeof(unsigned) * kSplitCounters;
+constexpr size_t kSplitWsBytes = (size_t)64 << 20;
+
+sparoa_status offer_splitk(sparoa_ctx* ctx, IgemmArgs* a) {
+  if (!ctx->splitk.p) return SPAROA_OK;  // no split K
+  a->ws_cnt = static_cast<unsigned*>(ctx->splitk.p);
+  a->ws_cnt_len = kSplitCounters;
+  a->ws = reinterpret_cast<float*>(static_cast<char*>(ctx->splitk.p) + kSplitCntBytes);
+  a->ws_bytes = kSplitWsBytes;
   return SPAROA_OK;
 }
 
@@ -353,6 +370,7 @@ sparoa_status run_gemm(sparoa_ctx* ctx, const GemmPlan& g) {
     a.out_occ = yo;
     a.emit = g.yo ? 1 : 0;
     a.err = ctx->d_err();
+    SP_TRY(offer_splitk(ctx, &a));
     SP_CUDA(launch_igemm(a, ctx->stream));
   }
   if (small_skip && force != 1) {
@@ -425,6 +443,7 @@ sparoa_status run_conv(sparoa_ctx* ctx, const ConvPlan& c) {
     return SPAROA_OK;
   }
   if (a.conv == 2) choose_spatial_tile(a);
+  SP_TRY(offer_splitk(ctx, &a));
   SP_CUDA(launch_igemm(a, ctx->stream));
   return SPAROA_OK;
 }
@@ -476,6 +495,21 @@ sparoa_status sparoa_create(sparoa_ctx** out, int device, void* stream) {
     delete ctx;
     return SPAROA_ERR_CUDA;
   }
+  // the split-K scratch is allocated here, not on first use, so that a
+  // context's first conv/GEMM can be recorded by stream capture
+  if (cudaMalloc(&ctx->splitk.p, kSplitCntBytes + kSplitWsBytes) != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(ctx->small.p);
+    delete ctx;
+    return SPAROA_ERR_OOM;
+  }
+  ctx->splitk.bytes = kSplitCntBytes + kSplitWsBytes;
+  if (cudaMemset(ctx->splitk.p, 0, kSplitCntBytes) != cudaSuccess || cudaStreamSynchronize(0) != cudaSuccess) {
+    cudaFree(ctx->splitk.p);
+    cudaFree(ctx->small.p);
+    delete ctx;
+    return SPAROA_ERR_CUDA;
+  }
   *out = ctx;
   return SPAROA_OK;
 }
@@ -484,7 +518,7 @@ sparoa_status sparoa_destroy(sparoa_ctx* ctx) {
   if (!ctx) return SPAROA_OK;
   DeviceGuard g(ctx->device, ctx->overlap);
   cudaStreamSynchronize(ctx->stream);
-  for (DevBuf* b : {&ctx->small, &ctx->occ, &ctx->pad_x, &ctx->pad_w, &ctx->arena})
+  for (DevBuf* b : {&ctx->small, &ctx->occ, &ctx->pad_x, &ctx->pad_w, &ctx->arena, &ctx->splitk})
     if (b->p) cudaFree(b->p);
   delete ctx;
   return SPAROA_OK;

@@ -190,6 +190,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   int* flags = reinterpret_cast<int*>(smem + C::kFlagOff);
   int* stage_last = flags;                // [S]: 1 = last stage of its tile
   volatile int* s_abort = flags + S;      // CTA-wide abort request
+  volatile int* s_last = flags + S + 2;   // [2] split K: this unit finishes its tile
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(flags + S + 1);
   uint32_t* s_kbits = reinterpret_cast<uint32_t*>(smem + C::kKBitsOff);
   unsigned long long* s_tap = reinterpret_cast<unsigned long long*>(smem + C::kTapOff);
@@ -211,6 +212,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nt = (p.N + BN - 1) / BN;
   const int mtiles = p.conv == 2 ? ((p.Nimg + p.bn - 1) / p.bn) * p.th * p.tw : (p.M + kBM - 1) / kBM;
   const int tiles = mtiles * nt;
+  // split K: work unit u = (tile u / KS, K range u % KS); KS consecutive units
+  // (run by neighbouring CTAs at the same time) share one output tile
+  const int KS = P.ksplit > 1 ? P.ksplit : 1;
+  const int units = tiles * KS;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -255,12 +260,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     int it = 0;        // stages filled so far (ring position)
     int pending = 0;   // mode 1: filled stages whose A arrivals are still owed
     bool ok = true;
-    for (int t = blockIdx.x; t < tiles; t += gridDim.x) {
+    for (int u = blockIdx.x; u < units; u += gridDim.x) {
+      const int t = u / KS, ks = u - (u / KS) * KS;
+      const int kb0 = (int)((int64_t)ks * kblocks / KS);
+      const int kb1 = (int)((int64_t)(ks + 1) * kblocks / KS);
       const TileGeo g = tile_geo(p, t, nt, BN);
       bool rvalid;
       int img, oh, ow;
       tile_row(p, g, r, rvalid, img, oh, ow);
-      int last = kblocks - 1;
+      int last = kb1 - 1;
       if (skip) {
         // ---- occupied K blocks of this tile
         named_bar_sync(1, 128);  // thread 0 is done with the previous tile's bits
@@ -324,14 +332,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         named_bar_sync(1, 128);
-        // last occupied block; a tile with none still runs block 0 (its data is all zero)
-        last = 0;
-        const int wtop = (kblocks - 1) >> 5;
-        for (int w = wtop; w >= 0; --w) {
-          uint32_t bits = w < kMaxKWords ? s_kbits[w] : 0xffffffffu;
-          if (w == wtop) bits &= 0xffffffffu >> (31 - ((kblocks - 1) & 31));
-          if (bits) {
-            last = w * 32 + 31 - __clz(bits);
+        // last occupied block of this unit's K range; a range with none still
+        // runs its first block (whose data is all zero)
+        last = kb0;
+        for (int kb = kb1 - 1; kb > kb0; --kb) {
+          if (kb >= kMaxKWords * 32 || ((s_kbits[kb >> 5] >> (kb & 31)) & 1u)) {
+            last = kb;
             break;
           }
         }
@@ -339,28 +345,50 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) continue;  // keep the skip-mask barriers in step; issue nothing more
       if (p.conv != 1) {
         if (r == 0) {
-          for (int kb = 0; kb <= last; ++kb) {
-            if (skip && kb != last && kb < kMaxKWords * 32 && !((s_kbits[kb >> 5] >> (kb & 31)) & 1u))
-              continue;
-            const int slot = it % S;
-            const uint32_t ph = (uint32_t)((it / S) & 1);
-            if (!mbar_wait(bar_empty + 8 * slot, ph ^ 1u, err, s_abort, kErrTimeoutEmpty)) {
-              ok = false;
-              break;
+          // The issuing lane is slow at anything but issuing: ring slot, phase
+          // and the (tap, channel block) of each K block advance incrementally,
+          // with no divisions in the loop, and the ring's first lap (whose
+          // slots are free by construction) waits for nothing.
+          int slot = it % S;
+          uint32_t ph = (uint32_t)((it / S) & 1);
+          int cb = 0, rr = 0, ss = 0;  // conv = 2: channel block and tap of block kb
+          if (p.conv == 2) {
+            const int tap = kb0 / cb_per_tap;
+            cb = kb0 - tap * cb_per_tap;
+            rr = tap / p.kw;
+            ss = tap - rr * p.kw;
+          }
+          const int iy0 = g.th0 * p.stride - p.pad, ix0 = g.tw0 * p.stride - p.pad;
+          const uint32_t fb0 = bar_full, eb0 = bar_empty;
+          for (int kb = kb0; kb <= last; ++kb) {
+            const bool issue =
+                !(skip && kb != last && kb < kMaxKWords * 32 && !((s_kbits[kb >> 5] >> (kb & 31)) & 1u));
+            if (issue) {
+              if (it >= S && !mbar_wait(eb0 + 8 * slot, ph ^ 1u, err, s_abort, kErrTimeoutEmpty)) {
+                ok = false;
+                break;
+              }
+              const uint32_t fb = fb0 + 8 * slot;
+              stage_last[slot] = (kb == last) ? 1 : 0;
+              mbar_arrive_expect_tx(fb, (uint32_t)C::kStageBytes);
+              if (p.conv == 0)
+                tma_load_2d(sA + slot * C::kAStage, &tmA, fb, kb * BK, g.m0);
+              else
+                tma_load_4d(sA + slot * C::kAStage, &tmA, fb, cb * BK, ix0 + ss, iy0 + rr, g.tn0);
+              tma_load_2d(sB + slot * C::kBStage, &tmB, fb, kb * BK, g.n0);
+              ++it;
+              if (++slot == S) {
+                slot = 0;
+                ph ^= 1u;
+              }
             }
-            stage_last[slot] = (kb == last) ? 1 : 0;
-            mbar_arrive_expect_tx(bar_full + 8 * slot, (uint32_t)C::kStageBytes);
-            if (p.conv == 0) {
-              tma_load_2d(sA + slot * C::kAStage, &tmA, bar_full + 8 * slot, kb * BK, g.m0);
-            } else {
-              const int tap = kb / cb_per_tap;
-              const int cb = kb - tap * cb_per_tap;
-              const int rr = tap / p.kw, ss = tap - (tap / p.kw) * p.kw;
-              tma_load_4d(sA + slot * C::kAStage, &tmA, bar_full + 8 * slot, cb * BK,
-                          g.tw0 * p.stride - p.pad + ss, g.th0 * p.stride - p.pad + rr, g.tn0);
+            if (p.conv == 2 && ++cb == cb_per_tap) {
+              cb = 0;
+              if (++ss == p.kw) {
+                ss = 0;
+                ++rr;
+              }
             }
-            tma_load_2d(sB + slot * C::kBStage, &tmB, bar_full + 8 * slot, kb * BK, g.n0);
-            ++it;
           }
         }
       } else {
@@ -368,7 +396,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int ih0 = oh * p.stride - p.pad;
         const int iw0 = ow * p.stride - p.pad;
         const __nv_bfloat16* ximg = xin + (int64_t)img * p.H * p.W * p.Cp;
-        for (int kb = 0; kb <= last; ++kb) {
+        for (int kb = kb0; kb <= last; ++kb) {
           if (skip && kb != last && kb < kMaxKWords * 32 && !((s_kbits[kb >> 5] >> (kb & 31)) & 1u))
             continue;
           const int slot = it % S;
@@ -418,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t idesc = idesc_bf16_f32(kBM, BN);
       int it = 0, j = 0;
       bool ok = true;
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++j) {
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++j) {
         const int b = j & 1;
         if (!mbar_wait(bar_acce + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort,
                        kErrTimeoutAcc))
@@ -426,9 +454,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         const uint32_t d = tmem + (uint32_t)(b * BN);
         bool first = true;
+        int slot = it % S;
+        uint32_t ph = (uint32_t)((it / S) & 1);
         while (true) {
-          const int slot = it % S;
-          const uint32_t ph = (uint32_t)((it / S) & 1);
           if (!mbar_wait(bar_full + 8 * slot, ph, err, s_abort, kErrTimeoutFull)) {
             ok = false;
             break;
@@ -454,6 +482,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           first = false;
           tc_commit(bar_empty + 8 * slot);
           ++it;
+          if (++slot == S) {
+            slot = 0;
+            ph ^= 1u;
+          }
           if (last) break;
         }
         if (ok) tc_commit(bar_accf + 8 * b);
@@ -486,7 +518,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t stg_base = sStg + (uint32_t)(ew * 2 * kWarpStgBytes);
     int j = 0;
     int stg_count = 0;  // blocks this warp handed to TMA so far
-    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++j) {
+    for (int u = blockIdx.x; u < units; u += gridDim.x, ++j) {
+      const int t = u / KS, ks = u - (u / KS) * KS;
       const int b = j & 1;
       const TileGeo g = tile_geo(p, t, nt, BN);
       bool mvalid;
@@ -508,6 +541,35 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (named_bar_or(2, kEpiThreads, !ok)) break;
       tc_fence_after();
       const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * BN);
+      // split K: every unit stores its fp32 partial tile, then takes a ticket;
+      // the unit that arrives last adds the others' partials and finishes the
+      // tile (nobody waits for anybody)
+      float* const ws_tile = KS > 1 ? P.ws + (int64_t)t * KS * kBM * BN : nullptr;
+      if (KS > 1) {
+        float* const mine = ws_tile + ((int64_t)ks * kBM + r) * BN + hf * 32;
+#pragma unroll 1
+        for (int gcol = 0; gcol < BN / 64; ++gcol) {
+          uint32_t raw[32];
+          tmem_ld32_nowait(tbase + (uint32_t)(gcol * 64 + hf * 32), raw);
+          tmem_wait_ld32(raw);
+          float4* dst = reinterpret_cast<float4*>(mine + gcol * 64);
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            __stcg(dst + i, make_float4(__uint_as_float(raw[4 * i]), __uint_as_float(raw[4 * i + 1]),
+                                        __uint_as_float(raw[4 * i + 2]), __uint_as_float(raw[4 * i + 3])));
+        }
+        __threadfence();
+        named_bar_sync(2, kEpiThreads);
+        if (et == 0) s_last[b] = atomicAdd(&P.ws_cnt[t], 1u) == (unsigned)(KS - 1) ? 1 : 0;
+        named_bar_sync(2, kEpiThreads);
+        if (!s_last[b]) {
+          tc_fence_before();
+          mbar_arrive(bar_acce + 8 * b);  // this unit's share is in the partial
+          continue;
+        }
+        __threadfence();
+        if (et == 0) P.ws_cnt[t] = 0u;  // every unit of the tile has arrived: ready for reuse
+      }
       const OccDev o = P.out_occ;  // registers, not parameter-space loads
       const int blk = mvalid ? (int)(m >> 7) : -1;
       const uint32_t grp = p.conv == 2 ? __match_any_sync(0xffffffffu, blk) : 0xffffffffu;
@@ -529,6 +591,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t raw[32];
         tmem_ld32_nowait(tbase + (uint32_t)(gcol * 64 + hf * 32), raw);
         tmem_wait_ld32(raw);
+        if (KS > 1) {
+          // the other units' partials of this row's 32 columns
+          for (int k2 = 0; k2 < KS; ++k2) {
+            if (k2 == ks) continue;
+            const float4* src =
+                reinterpret_cast<const float4*>(ws_tile + ((int64_t)k2 * kBM + r) * BN + gcol * 64 + hf * 32);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              const float4 v = __ldcg(src + i);
+              raw[4 * i] = __float_as_uint(__uint_as_float(raw[4 * i]) + v.x);
+              raw[4 * i + 1] = __float_as_uint(__uint_as_float(raw[4 * i + 1]) + v.y);
+              raw[4 * i + 2] = __float_as_uint(__uint_as_float(raw[4 * i + 2]) + v.z);
+              raw[4 * i + 3] = __float_as_uint(__uint_as_float(raw[4 * i + 3]) + v.w);
+            }
+          }
+        }
         uint32_t rw = 0u;  // non-zero bits of this row in the warp's 32 columns
         const float* scg = scb + gcol * 64 + hf * 32;
         const float* shg = shb + gcol * 64 + hf * 32;
@@ -794,7 +872,8 @@ cudaError_t launch_cfg(const IgemmArgs& a, const CUtensorMap& tA, const CUtensor
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  const int64_t grid = tiles < num_sms() ? tiles : num_sms();
+  const int64_t units = tiles * (a.ksplit > 1 ? a.ksplit : 1);
+  const int64_t grid = units < num_sms() ? units : num_sms();
   cudaError_t e = launch_kernel(igemm_kernel<BN, BK>, dim3((unsigned)grid), dim3(kThreads),
                                 (size_t)Cfg<BN, BK>::kSmem, s, tA, tB, tY, a);
   if (e != cudaSuccess) return e;
@@ -829,16 +908,45 @@ void choose_spatial_tile(IgemmArgs& a) {
   }
 }
 
-cudaError_t launch_igemm(const IgemmArgs& a, cudaStream_t s) {
+// N tile and K split, from a sweep of (BN, ksplit) on GB300 over GEMMs
+// (M 256..4096, K 768..3072) and 3x3 convs (ResNet stages at batch 1..32):
+// 128-wide tiles win or tie nearly everywhere, 256-wide ones when there are
+// still two tiles per SM, 64-wide ones when 128-wide tiles would fill under
+// half of the SMs; splitting K pays only while the
+// tiles leave SMs idle, at most 4 ways and with at least 8 K blocks per unit
+// (the tile's last unit reads the other partials alone).
+void choose_tiles(const IgemmArgs& a, int64_t mtiles, int* bn_out, int* ks_out) {
+  const int sms = num_sms();
+  int bn = a.N > 64 ? 128 : 64;
+  int64_t tiles = mtiles * ((a.N + bn - 1) / bn);
+  if (a.N > 128 && mtiles * ((a.N + 255) / 256) >= 2 * sms) {
+    bn = 256;  // plenty of tiles even at 256 wide: the wider epilogue amortises better
+    tiles = mtiles * ((a.N + bn - 1) / bn);
+  } else if (bn == 128 && tiles < sms / 2) {
+    bn = 64;
+    tiles = mtiles * ((a.N + bn - 1) / bn);
+  }
+  const int bk = (bn < 256 && (a.conv == 2 ? (a.Cp % 64 == 0) : (a.Ktot > 32))) ? 64 : 32;
+  const int kblocks = (a.Ktot + bk - 1) / bk;
+  int ks = 1;
+  if (a.ws && a.ws_cnt && tiles < sms && tiles <= a.ws_cnt_len) {
+    ks = (int)(sms / tiles);
+    if (ks > 4) ks = 4;
+    while (ks > 1 && (kblocks < 8 * ks || (size_t)tiles * ks * kBM * bn * 4 > a.ws_bytes)) --ks;
+  }
+  *bn_out = bn;
+  *ks_out = ks;
+}
+
+cudaError_t launch_igemm(const IgemmArgs& a_in, cudaStream_t s) {
+  IgemmArgs a = a_in;
   if (a.M <= 0 || a.N <= 0) return cudaSuccess;
   if (a.conv == 2 && (a.Cp % 32 != 0 || a.bw * a.bh * a.bn != 128)) return cudaErrorInvalidValue;
   const int64_t mtiles =
       a.conv == 2 ? (int64_t)((a.Nimg + a.bn - 1) / a.bn) * a.th * a.tw : (a.M + kBM - 1) / kBM;
-  int bn = 64;
-  if (a.N > 64) {
-    bn = 256;
-    while (bn > 64 && (bn / 2 >= a.N || mtiles * ((a.N + bn - 1) / bn) < num_sms())) bn /= 2;
-  }
+  int bn = 64, ks = 1;
+  choose_tiles(a, mtiles, &bn, &ks);
+  a.ksplit = ks;
   // K block: 64 (128-byte swizzle) when the channel layout allows it and the
   // stage ring still holds at least four stages; 32 otherwise
   const int bk = (bn < 256 && (a.conv == 2 ? (a.Cp % 64 == 0) : (a.Ktot > 32))) ? 64 : 32;

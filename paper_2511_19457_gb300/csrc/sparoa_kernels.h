@@ -72,9 +72,17 @@ struct IgemmArgs {
   OccDev out_occ{};
   int emit = 0;
   uint32_t* err = nullptr;
+  // split K (set by launch_igemm from the scratch offered here): fp32 partial
+  // tiles [tiles][ksplit][128][BN] in `ws` (ws_bytes), one zeroed arrival
+  // counter per output tile in `ws_cnt` (ws_cnt_len), left zero again
+  int ksplit = 1;
+  float* ws = nullptr;
+  size_t ws_bytes = 0;
+  unsigned* ws_cnt = nullptr;
+  int ws_cnt_len = 0;
 };
 
-// Picks the N tile, encodes the tensor maps and launches.
+// Picks the N tile and the K split, encodes the tensor maps and launches.
 cudaError_t launch_igemm(const IgemmArgs& a, cudaStream_t s);
 
 // Streaming multiprocessors of the current device (cached per process).
