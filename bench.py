@@ -45,7 +45,7 @@ def parse_args():
     p.add_argument("--warmup", type=int, default=400)
     p.add_argument("--impl", default="sparoa", choices=["sparoa", "reference"])
     p.add_argument("--workload", default="conv",
-                   choices=["conv", "fc", "resnet18", "mobilenet_v2", "mlp_sweep"])
+                   choices=["conv", "fc", "resnet18", "mobilenet_v2", "mlp_sweep", "ops"])
     p.add_argument("--batch", type=int, default=32)
     p.add_argument("--no-cpu-baseline", action="store_true")
     return p.parse_args()
@@ -601,6 +601,136 @@ def run_graph_workload(args, rank, local_rank, world, peaks, name):
     return line
 
 
+def run_ops(args, rank, local_rank, world, peaks):
+    """Per-operator roofline: every kernel of the path at the workloads' shapes,
+    timed as CUDA-graph replays over rotating input/output sets larger than L2;
+    achieved = algorithmic bytes (or dense-equivalent FLOPs) / time per call."""
+    import torch
+
+    from paper_2511_19457_gb300 import sparoa as sp
+    from paper_2511_19457_gb300 import synth
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    ctx = sp.Context(local_rank)
+    gen = torch.Generator(device=dev).manual_seed(0)
+    L2 = 129e6
+    hbm, tc = peaks["hbm_gbs"], peaks["bf16_tflops"]
+    occ_b = lambda R, C: int(sp._lib.sparoa_occupancy_bytes(R, C))
+
+    def act_like(*shape, zero_p=0.5):
+        v = torch.randn(*shape, device=dev, generator=gen).abs()
+        v[torch.rand(*shape, device=dev, generator=gen) < zero_p] = 0.0
+        return v.to(torch.bfloat16)
+
+    rows = []
+
+    def measure(name, make_set, call, set_bytes, alg_bytes=0.0, alg_flops=0.0, bound="hbm"):
+        nb = max(2, min(40, int(3 * L2 / max(set_bytes, 1)) + 1))
+        sets = [make_set() for _ in range(nb)]
+        for st in sets:
+            call(st)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for st in sets:
+                call(st)
+        g.replay()
+        reps = max(3, 200 // nb)
+        us = time_graph(g, reps) * 1e3 / (reps * nb)
+        if bound == "hbm":
+            ach = alg_bytes / (us * 1e-6) / 1e9
+            rows.append({"op": name, "us": round(us, 2), "bound": "hbm", "achieved": round(ach, 1),
+                         "unit": "GB/s", "peak": hbm, "frac": round(ach / hbm, 4),
+                         "algorithmic_bytes": int(alg_bytes), "rotating_sets": nb})
+        else:
+            ach = alg_flops / (us * 1e-6) / 1e12
+            rows.append({"op": name, "us": round(us, 2), "bound": "tensor", "achieved": round(ach, 1),
+                         "unit": "TFLOP/s", "peak": tc, "frac": round(ach / tc, 4),
+                         "algorithmic_flops": int(alg_flops), "rotating_sets": nb})
+        del sets
+        torch.cuda.empty_cache()
+
+    # a1 stats
+    for (R, C) in [(25088, 64), (4096, 3072), (401408, 64)]:
+        b = R * C * 2 + occ_b(R, C)
+        measure(f"stats [{R},{C}]",
+                lambda R=R, C=C: (act_like(R, C), sp.OccupancyBuffer(R, C)),
+                lambda st, R=R, C=C: sp.sparoa_op_stats(ctx, st[0], (R, C), occ=st[1], host=False),
+                b, alg_bytes=b)
+    # a6 depthwise (MobileNetV2 layers), BN + ReLU6, output occupancy
+    for (N, H, W, C, s) in [(32, 112, 112, 96, 2), (32, 56, 56, 144, 1)]:
+        Ho, Wo = (H + 2 - 3) // s + 1, (W + 2 - 3) // s + 1
+        w = (torch.randn(C, 3, 3, 1, device=dev, generator=gen) / 3).to(torch.bfloat16)
+        bnp = torch.tensor(synth.identity_bn(C), device=dev)
+        b = N * H * W * C * 2 + N * Ho * Wo * C * 2 + C * 9 * 2 + occ_b(N * Ho * Wo, C)
+        measure(f"depthwise 3x3 s{s} [{N},{H},{W},{C}]",
+                lambda N=N, H=H, W=W, C=C, Ho=Ho, Wo=Wo: (
+                    act_like(N, H, W, C), torch.empty(N, Ho, Wo, C, dtype=torch.bfloat16, device=dev),
+                    sp.OccupancyBuffer(N * Ho * Wo, C)),
+                lambda st, w=w, s=s, C=C, bnp=bnp: sp.sparoa_conv2d(
+                    ctx, st[0], w, st[1], stride=s, pad=1, groups=C, bn=bnp, act=sp.ACT_RELU6,
+                    y_occ=st[2]),
+                b, alg_bytes=b)
+    # a7 pooling and stand-alone BN/activation
+    b = 32 * 112 * 112 * 64 * 2 + 32 * 56 * 56 * 64 * 2 + occ_b(32 * 56 * 56, 64)
+    measure("maxpool 3x3/2 [32,112,112,64]",
+            lambda: (act_like(32, 112, 112, 64), torch.empty(32, 56, 56, 64, dtype=torch.bfloat16, device=dev),
+                     sp.OccupancyBuffer(32 * 56 * 56, 64)),
+            lambda st: sp.sparoa_maxpool2d(ctx, st[0], st[1], y_occ=st[2]), b, alg_bytes=b)
+    b = 32 * 7 * 7 * 1280 * 2 + 32 * 1280 * 2 + occ_b(32, 1280)
+    measure("avgpool global [32,7,7,1280]",
+            lambda: (act_like(32, 7, 7, 1280), torch.empty(32, 1, 1, 1280, dtype=torch.bfloat16, device=dev),
+                     sp.OccupancyBuffer(32, 1280)),
+            lambda st: sp.sparoa_avgpool_global(ctx, st[0], st[1], y_occ=st[2]), b, alg_bytes=b)
+    bnp64 = torch.tensor(synth.identity_bn(64), device=dev)
+    b = 2 * 32 * 56 * 56 * 64 * 2 + occ_b(32 * 56 * 56, 64)
+    measure("bn+relu [32,56,56,64]",
+            lambda: (act_like(32, 56, 56, 64, zero_p=0.0), torch.empty(32, 56, 56, 64, dtype=torch.bfloat16, device=dev),
+                     sp.OccupancyBuffer(32 * 56 * 56, 64)),
+            lambda st: sp.sparoa_bn_act(ctx, st[0], st[1], bn=bnp64, act=sp.ACT_RELU, y_occ=st[2]),
+            b, alg_bytes=b)
+    # a4 zero-skip FC (column-sparse input: only occupied weight rows are read)
+    d = synth.fc_layer(seed=0)
+    M, K, N = d["M"], d["K"], d["N"]
+    wfc = sp.bits_to_device(d["w"]).view(N, K)
+    wkn = sp.bits_to_device(d["w_kn"]).view(K, N)
+    x0 = sp.bits_to_device(d["x"]).view(M, K)
+    kocc = int((x0.float().abs().sum(0) != 0).sum().item())
+    b = kocc * N * 2 + M * K * 2 + M * N * 4
+    measure(f"fc zero-skip [{M},{K}]x[{K},{N}] (occupied K {kocc})",
+            lambda: (x0.clone(), torch.empty(M, N, dtype=torch.float32, device=dev), sp.OccupancyBuffer(M, K)),
+            lambda st: (sp.sparoa_op_stats(ctx, st[0], (M, K), occ=st[2], host=False),
+                        sp.sparoa_gemm(ctx, st[0], wfc, st[1], W_kn=wkn, x_occ=st[2])),
+            M * K * 2 + M * N * 4, alg_bytes=b)
+    # a5 dense GEMMs (MLP block) and the 3x3 conv
+    for (M, K, N) in [(4096, 768, 3072), (4096, 3072, 768)]:
+        w = (torch.randn(N, K, device=dev, generator=gen) / K ** 0.5).to(torch.bfloat16)
+        measure(f"gemm dense [{M},{K}]x[{N},{K}]^T",
+                lambda M=M, K=K, N=N: (act_like(M, K, zero_p=0.0), torch.empty(M, N, dtype=torch.bfloat16, device=dev),
+                                       sp.OccupancyBuffer(M, K)),
+                lambda st, w=w, M=M, K=K: (sp.sparoa_op_stats(ctx, st[0], (M, K), occ=st[2], host=False),
+                                           sp.sparoa_gemm(ctx, st[0], w, st[1], x_occ=st[2],
+                                                          thr=sp.thresholds(force_path=sp.PATH_DENSE))),
+                M * K * 2 + M * N * 2, alg_flops=2.0 * M * K * N, bound="tensor")
+    w3 = (torch.randn(64, 3, 3, 64, device=dev, generator=gen) / 24).to(torch.bfloat16)
+    for force, tag in [(sp.PATH_DENSE, "dense"), (sp.PATH_SKIP, "zero-skip")]:
+        measure(f"conv3x3 [32,56,56,64]->64 {tag}",
+                lambda: (act_like(32, 56, 56, 64), torch.empty(32, 56, 56, 64, dtype=torch.bfloat16, device=dev),
+                         sp.OccupancyBuffer(32 * 56 * 56, 64), sp.OccupancyBuffer(32 * 56 * 56, 64)),
+                lambda st, force=force: (sp.sparoa_op_stats(ctx, st[0], (32, 56, 56, 64), occ=st[2], host=False),
+                                         sp.sparoa_conv2d(ctx, st[0], w3, st[1], stride=1, pad=1, act=sp.ACT_RELU,
+                                                          thr=sp.thresholds(force_path=force), x_occ=st[2],
+                                                          y_occ=st[3])),
+                2 * 32 * 56 * 56 * 64 * 2, alg_flops=2.0 * 32 * 56 * 56 * 64 * 64 * 9, bound="tensor")
+    ctx.close()
+    return {"metric": METRIC, "value": None, "unit": "per-op roofline", "n_gpus": world,
+            "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "every kernel of the path at the workloads' shapes; the GEMM, FC and "
+                                   "conv rows include their input's stats kernel",
+                       "l2": "rotating sets totalling > 3 x 129 MB per graph"},
+            "ops": rows}
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -622,6 +752,8 @@ def main():
         line = run_fc(args, rank, local_rank, world, peaks)
     elif args.workload == "mlp_sweep":
         line = run_mlp_sweep(args, rank, local_rank, world, peaks)
+    elif args.workload == "ops":
+        line = run_ops(args, rank, local_rank, world, peaks)
     else:
         raise SystemExit(f"workload {args.workload} is not wired into bench.py")
     if rank == 0:

@@ -146,11 +146,36 @@ __device__ __forceinline__ void cta_done(const OccDev& o, const uint32_t* s_acc,
   for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
 
 // ---------------------------------------------------------------------------
-// Eq. 1 count and bitmaps of an existing tensor.  A CTA owns whole 128-row
-// blocks (every column tile of them), so it writes their row bitmap words and
-// block masks with plain stores; only the counters need clearing beforehand.
-// Column counts gather in shared memory (C words, dynamic) and reach global
-// memory once per CTA.
+// Eq. 1 count and bitmaps of an existing tensor.  A work item is a 128-row
+// block x a chunk of up to kStatsChunk 64-column tiles; the next tile's loads
+// are issued before the current one is reduced.  Block masks are owned by
+// their item (plain stores); a row's bitmap word is stored whole when one
+// chunk covers all of the row's tiles, else OR-ed in (the caller then clears
+// the row bitmaps too).  Column counts gather in shared memory (C words,
+// dynamic) and reach global memory once per CTA.
+constexpr int kStatsChunk = kStatsWholeRowCols / 64;
+
+__device__ __forceinline__ void stats_load(const __nv_bfloat16* __restrict__ x, int64_t R, int C,
+                                           bool vec, int64_t row0, int col0, int cg, int rs,
+                                           uint4 (&u)[4], uint32_t (&m)[4]) {
+  const int c0 = col0 + cg * 8;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int64_t r = row0 + rs + 32 * i;
+    m[i] = 0u;
+    u[i] = make_uint4(0u, 0u, 0u, 0u);
+    if (r < R && c0 < C) {
+      const __nv_bfloat16* p = x + r * C + c0;
+      if (vec) {
+        u[i] = __ldg(reinterpret_cast<const uint4*>(p));
+      } else {
+        for (int j = 0; j < 8 && c0 + j < C; ++j)
+          if (bf16_nz(__bfloat16_as_ushort(p[j]))) m[i] |= 1u << j;
+      }
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kTileThreads) stats_kernel(const __nv_bfloat16* __restrict__ x,
                                                              int64_t R, int C, OccDev o_param) {
   const OccDev o = o_param;  // registers, not parameter-space loads
@@ -161,49 +186,53 @@ __global__ void __launch_bounds__(kTileThreads) stats_kernel(const __nv_bfloat16
   const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
   const bool vec = (C & 7) == 0;
   const int ctn = (C + 63) / 64;
+  const int nch = (ctn + kStatsChunk - 1) / kStatsChunk;
+  const bool own_row = nch == 1;  // one chunk holds every tile of a row
   const int64_t nrb = (R + 127) / 128;
+  const int64_t items = nrb * nch;
   if (acc)
     for (int c = threadIdx.x; c < C; c += kTileThreads) s_acc[c] = 0u;
   __syncthreads();
   pdl_wait();
   pdl_trigger();
-  for (int64_t rb = blockIdx.x; rb < nrb; rb += gridDim.x) {
+  for (int64_t item = blockIdx.x; item < items; item += gridDim.x) {
+    const int64_t rb = item / nch;
+    const int ch = (int)(item - rb * nch);
     const int64_t row0 = rb * 128;
-    unsigned long long rw[4] = {0ull, 0ull, 0ull, 0ull};  // row bitmap word being built, per owned row
-    for (int ct = 0; ct < ctn; ++ct) {
+    const int ct0 = ch * kStatsChunk;
+    const int ct1 = ct0 + kStatsChunk < ctn ? ct0 + kStatsChunk : ctn;
+    unsigned long long rw[4] = {0ull, 0ull, 0ull, 0ull};  // row bitmap bits of this chunk, per owned row
+    uint4 u[4];
+    uint32_t m[4];
+    stats_load(x, R, C, vec, row0, ct0 * 64, cg, rs, u, m);
+    for (int ct = ct0; ct < ct1; ++ct) {
       const int col0 = ct * 64;
-      const int c0 = col0 + cg * 8;
-      uint32_t m[4];
+      if (vec) {
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int64_t r = row0 + rs + 32 * i;
-        m[i] = 0u;
-        if (r < R && c0 < C) {
-          const __nv_bfloat16* p = x + r * C + c0;
-          if (vec) {
-            m[i] = nz_mask8(__ldg(reinterpret_cast<const uint4*>(p)));
-          } else {
-            for (int j = 0; j < 8 && c0 + j < C; ++j)
-              if (bf16_nz(__bfloat16_as_ushort(p[j]))) m[i] |= 1u << j;
-          }
-        }
+        for (int i = 0; i < 4; ++i) m[i] = nz_mask8(u[i]);
       }
+      uint32_t mc[4] = {m[0], m[1], m[2], m[3]};
+      if (ct + 1 < ct1) stats_load(x, R, C, vec, row0, col0 + 64, cg, rs, u, m);  // next tile in flight
       // row bits: lanes 8k..8k+7 share a row
       uint32_t cnt[8];
 #pragma unroll
       for (int j = 0; j < 8; ++j) cnt[j] = 0u;
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        const uint32_t bl = __ballot_sync(0xffffffffu, m[i] != 0u);
+        const uint32_t bl = __ballot_sync(0xffffffffu, mc[i] != 0u);
         if ((bl >> (lane & ~7)) & 0xFFu) rw[i] |= 1ull << (ct & 63);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) cnt[j] += (m[i] >> j) & 1u;
+        for (int j = 0; j < 8; ++j) cnt[j] += (mc[i] >> j) & 1u;
       }
-      if ((ct & 63) == 63 || ct == ctn - 1) {
+      if ((ct & 63) == 63 || ct == ct1 - 1) {
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           const int64_t r = row0 + rs + 32 * i;
-          if (cg == 0 && r < R) o.row_bm[r * o.W64 + (ct >> 6)] = rw[i];
+          if (cg == 0 && r < R) {
+            unsigned long long* dst = &o.row_bm[r * o.W64 + (ct >> 6)];
+            if (own_row) *dst = rw[i];
+            else if (rw[i]) atomicOr(dst, rw[i]);
+          }
           rw[i] = 0ull;
         }
       }
@@ -225,7 +254,7 @@ __global__ void __launch_bounds__(kTileThreads) stats_kernel(const __nv_bfloat16
         const int col = col0 + threadIdx.x;
         const uint32_t word = __ballot_sync(0xffffffffu, c != 0u);
         const int w = (col0 >> 5) + (threadIdx.x >> 5);
-        if (lane == 0 && w < o.C32) o.blk_mask[rb * o.C32 + w] = word;  // this CTA owns the block
+        if (lane == 0 && w < o.C32) o.blk_mask[rb * o.C32 + w] = word;  // this item owns the word
         if (acc) {
           if (col < C) s_acc[col] += c;
         } else {
@@ -275,11 +304,16 @@ __global__ void __launch_bounds__(kTileThreads) dwconv_kernel(const DwArgs a_par
   TileEmit e;
   e.init();
   const int hw = a.Ho * a.Wo;
+  const int64_t img_elems = (int64_t)a.H * a.W * a.C;
   int cur_col0 = -1;
   float sc[8], sh[8];
-  SPAROA_TILE_LOOP(R, a.C) {
-    const int64_t row0 = (tile / ctn) * 128;
-    const int col0 = (int)(tile % ctn) * 64;
+  // channel slice major: a CTA's consecutive tiles share their weights and affine
+  const int ctn = (a.C + 63) / 64;
+  const int64_t nrt = (R + 127) / 128;
+  const int64_t ntiles = nrt * ctn;
+  for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+    const int64_t row0 = (tile % nrt) * 128;
+    const int col0 = (int)(tile / nrt) * 64;
     const int c0 = col0 + cg * 8;
     const bool cvalid = c0 < a.C;
     if (col0 != cur_col0) {  // (uniform) new channel slice: weights and affine
@@ -297,44 +331,62 @@ __global__ void __launch_bounds__(kTileThreads) dwconv_kernel(const DwArgs a_par
       __syncthreads();
       cur_col0 = col0;
     }
+    // Every tap's load is unconditional (its address clamped into the image;
+    // out-of-range taps are zeroed afterwards), so a row's 9 loads, and the
+    // next row's, are in flight together instead of one latency each.
+#pragma unroll 2
     for (int i = 0; i < 4; ++i) {
-      const int64_t mrow = row0 + rs + 32 * i;
+      const int64_t mrow_raw = row0 + rs + 32 * i;
+      const bool live = cvalid && mrow_raw < R;
+      const int64_t mrow = live ? mrow_raw : 0;
       uint32_t mask = 0;
-      if (cvalid && mrow < R) {
-        const int img = (int)(mrow / hw);
-        const int rem = (int)(mrow - (int64_t)img * hw);
-        const int oh = rem / a.Wo, ow = rem - (rem / a.Wo) * a.Wo;
-        const __nv_bfloat16* xi = a.x + (int64_t)img * a.H * a.W * a.C + c0;
+      {
+        // 32-bit index math (output rows and in-image offsets stay below 2^31;
+        // the launcher checks), 64-bit only for the image base
+        const uint32_t m32 = (uint32_t)mrow;
+        const uint32_t img = m32 / (uint32_t)hw;
+        const uint32_t rem = m32 - img * (uint32_t)hw;
+        const int oh = (int)(rem / (uint32_t)a.Wo), ow = (int)(rem - (rem / (uint32_t)a.Wo) * (uint32_t)a.Wo);
+        const __nv_bfloat16* xi = a.x + (int64_t)img * img_elems + (cvalid ? c0 : 0);
+        uint4 u[9];
+        uint32_t inb = 0u;
+#pragma unroll
+        for (int r = 0; r < 3; ++r) {
+          const int ih = oh * a.stride - a.pad + r;
+          const int ihc = ih < 0 ? 0 : (ih >= a.H ? a.H - 1 : ih);
+#pragma unroll
+          for (int s = 0; s < 3; ++s) {
+            const int iw = ow * a.stride - a.pad + s;
+            const int iwc = iw < 0 ? 0 : (iw >= a.W ? a.W - 1 : iw);
+            if (ih == ihc && iw == iwc) inb |= 1u << (r * 3 + s);
+            u[r * 3 + s] = __ldg(reinterpret_cast<const uint4*>(xi + (uint32_t)(ihc * a.W + iwc) * (uint32_t)a.C));
+          }
+        }
         float accv[8];
 #pragma unroll
         for (int j = 0; j < 8; ++j) accv[j] = 0.f;
 #pragma unroll
-        for (int r = 0; r < 3; ++r) {
-          const int ih = oh * a.stride - a.pad + r;
+        for (int t = 0; t < 9; ++t) {
+          float f[8];
+          unpack8(((inb >> t) & 1u) ? u[t] : make_uint4(0u, 0u, 0u, 0u), f);
+          const float4 w0 = *reinterpret_cast<const float4*>(&s_w[t][cg * 8]);
+          const float4 w1 = *reinterpret_cast<const float4*>(&s_w[t][cg * 8 + 4]);
+          const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
 #pragma unroll
-          for (int s = 0; s < 3; ++s) {
-            const int iw = ow * a.stride - a.pad + s;
-            if (ih >= 0 && ih < a.H && iw >= 0 && iw < a.W) {
-              float f[8];
-              unpack8(__ldg(reinterpret_cast<const uint4*>(xi + ((int64_t)ih * a.W + iw) * a.C)), f);
-              const float4 w0 = *reinterpret_cast<const float4*>(&s_w[r * 3 + s][cg * 8]);
-              const float4 w1 = *reinterpret_cast<const float4*>(&s_w[r * 3 + s][cg * 8 + 4]);
-              const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
-#pragma unroll
-              for (int j = 0; j < 8; ++j) accv[j] = fmaf(f[j], wv[j], accv[j]);
-            }
-          }
+          for (int j = 0; j < 8; ++j) accv[j] = fmaf(f[j], wv[j], accv[j]);
         }
         float rv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        if (a.ep.residual) unpack8(*reinterpret_cast<const uint4*>(a.ep.residual + mrow * a.C + c0), rv);
+        if (a.ep.residual && live) unpack8(*reinterpret_cast<const uint4*>(a.ep.residual + mrow * a.C + c0), rv);
         float o[8];
 #pragma unroll
         for (int j = 0; j < 8; ++j) o[j] = epi_act(fmaf(accv[j], sc[j], sh[j]) + rv[j], a.ep.act);
-        const uint4 u = pack8(o);
-        *reinterpret_cast<uint4*>(a.y + mrow * a.C + c0) = u;
-        mask = nz_mask8(u);
+        const uint4 uo = pack8(o);
+        if (live) {
+          *reinterpret_cast<uint4*>(a.y + mrow * a.C + c0) = uo;
+          mask = nz_mask8(uo);
+        }
       }
-      if (a.emit) e.row(mask, mrow, col0, a.out_occ);
+      if (a.emit) e.row(mask, mrow_raw, col0, a.out_occ);
     }
     if (a.emit) e.tile_done(row0, col0, a.out_occ, s_cnt, s_acc, acc);
   }
@@ -372,17 +424,45 @@ __global__ void __launch_bounds__(kTileThreads)
         float mx[8];
 #pragma unroll
         for (int j = 0; j < 8; ++j) mx[j] = -INFINITY;
-        for (int r = 0; r < k; ++r) {
-          const int ih = oh * stride - pad + r;
-          if (ih < 0 || ih >= H) continue;
-          for (int s = 0; s < k; ++s) {
-            const int iw = ow * stride - pad + s;
-            if (iw < 0 || iw >= W) continue;
+        if (k == 3) {
+          // 3x3: the 9 loads unconditional (addresses clamped into the image,
+          // out-of-range taps left out of the max), all in flight together
+          uint4 u[9];
+          uint32_t inb = 0u;
+#pragma unroll
+          for (int r = 0; r < 3; ++r) {
+            const int ih = oh * stride - pad + r;
+            const int ihc = ih < 0 ? 0 : (ih >= H ? H - 1 : ih);
+#pragma unroll
+            for (int s = 0; s < 3; ++s) {
+              const int iw = ow * stride - pad + s;
+              const int iwc = iw < 0 ? 0 : (iw >= W ? W - 1 : iw);
+              if (ih == ihc && iw == iwc) inb |= 1u << (r * 3 + s);
+              u[r * 3 + s] = __ldg(reinterpret_cast<const uint4*>(x + (((int64_t)img * H + ihc) * W + iwc) * C + c0));
+            }
+          }
+#pragma unroll
+          for (int t = 0; t < 9; ++t) {
+            if (!((inb >> t) & 1u)) continue;
             float f[8];
-            unpack8(__ldg(reinterpret_cast<const uint4*>(x + (((int64_t)img * H + ih) * W + iw) * C + c0)), f);
+            unpack8(u[t], f);
 #pragma unroll
             for (int j = 0; j < 8; ++j)
               if (f[j] > mx[j]) mx[j] = f[j];
+          }
+        } else {
+          for (int r = 0; r < k; ++r) {
+            const int ih = oh * stride - pad + r;
+            if (ih < 0 || ih >= H) continue;
+            for (int s = 0; s < k; ++s) {
+              const int iw = ow * stride - pad + s;
+              if (iw < 0 || iw >= W) continue;
+              float f[8];
+              unpack8(__ldg(reinterpret_cast<const uint4*>(x + (((int64_t)img * H + ih) * W + iw) * C + c0)), f);
+#pragma unroll
+              for (int j = 0; j < 8; ++j)
+                if (f[j] > mx[j]) mx[j] = f[j];
+            }
           }
         }
         const uint4 u = pack8(mx);
@@ -420,7 +500,8 @@ __global__ void __launch_bounds__(kTileThreads)
       if (n < N && c0 < C) {
         float a8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         const __nv_bfloat16* p = x + n * (int64_t)HW * C + c0;
-        for (int q = 0; q < HW; ++q) {
+#pragma unroll 8
+        for (int q = 0; q < HW; ++q) {  // unrolled: eight pixels' loads in flight
           float f[8];
           unpack8(__ldg(reinterpret_cast<const uint4*>(p + (int64_t)q * C)), f);
 #pragma unroll
@@ -514,9 +595,9 @@ unsigned tile_grid(int64_t R, int C) {
 
 cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev& o, cudaStream_t s) {
   if (R <= 0 || C <= 0) return cudaSuccess;
-  const int64_t nrb = (R + 127) / 128;
+  const int64_t items = ((R + 127) / 128) * ((((C + 63) / 64) + kStatsChunk - 1) / kStatsChunk);
   const int64_t cap = 4LL * device_sm_count();  // 4 CTAs per SM
-  const unsigned grid = (unsigned)(nrb < cap ? nrb : cap);
+  const unsigned grid = (unsigned)(items < cap ? items : cap);
   const size_t smem = C <= kMaxAccCols ? sizeof(uint32_t) * (size_t)C : 0;
   return launch_kernel(stats_kernel, dim3(grid), dim3(kTileThreads), smem, s, x, R, C, o);
 }
@@ -540,6 +621,8 @@ cudaError_t launch_pad_channels(const __nv_bfloat16* x, int64_t P, int C, int Cp
 cudaError_t launch_dwconv(const DwArgs& a, cudaStream_t s) {
   const int64_t R = (int64_t)a.N * a.Ho * a.Wo;
   if (R <= 0) return cudaSuccess;
+  // the kernel's 32-bit index math: output rows and one image's elements
+  if (R >= ((int64_t)1 << 31) || (int64_t)a.H * a.W * a.C >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;
   return launch_kernel(dwconv_kernel, dim3(tile_grid(R, a.C)), dim3(kTileThreads),
                        acc_smem(a.emit, a.C), s, a);
 }

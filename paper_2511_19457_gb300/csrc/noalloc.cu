@@ -118,10 +118,13 @@ extern "C" sparoa_status sparoa_gemm_noalloc(void* stream, const void* x, int64_
   carve(b + kCtrlBytes, M, K, &xo);
   {
     // control words and the Eq. 1 counters (which start the occupancy block);
-    // the stats kernel writes the bitmaps whole
+    // the stats kernel writes the block masks whole, and the row bitmaps too
+    // unless K is wide
     ClearArgs z = {};
     z.p[0] = reinterpret_cast<uint32_t*>(b);
-    z.words[0] = (int64_t)((kCtrlBytes + (reinterpret_cast<char*>(xo.row_bm) - (b + kCtrlBytes))) / 4);
+    const char* end = K <= kStatsWholeRowCols ? reinterpret_cast<char*>(xo.row_bm)
+                                              : reinterpret_cast<char*>(xo.blk_mask);
+    z.words[0] = (int64_t)((end - b) / 4);
     if (launch_clear(z, s) != cudaSuccess) return SPAROA_ERR_CUDA;
   }
 
