@@ -394,6 +394,186 @@ __global__ void __launch_bounds__(kTileThreads) dwconv_kernel(const DwArgs a_par
 }
 
 // ---------------------------------------------------------------------------
+// Depthwise 3x3, pad 1, stride S in {1, 2} (every MobileNetV2 depthwise layer)
+// on 2-D output tiles: a CTA computes kDwTH x kDwTW output pixels of one image
+// and one 64-channel slice.  The input tile with its halo is staged in shared
+// memory once (cp.async, zero-filled outside the image = the padding); each
+// thread then computes 4 horizontally adjacent pixels x 8 channels, reading
+// every input column it needs once per kernel row.  Tiles run channel-slice
+// major so a CTA's consecutive tiles keep their weights and affine.
+constexpr int kDwTH = 8, kDwTW = 16;
+
+template <int S>
+__global__ void __launch_bounds__(kTileThreads) dw3_kernel(const DwArgs a_param) {
+  const DwArgs a = a_param;  // registers, not parameter-space loads
+  constexpr int IH = (kDwTH - 1) * S + 3, IW = (kDwTW - 1) * S + 3;
+  constexpr int NCOL = 3 * S + 3;  // input columns a 4-pixel strip reads: (4 - 1) S + 3
+  extern __shared__ __align__(16) uint8_t dsm[];
+  __nv_bfloat16* s_in = reinterpret_cast<__nv_bfloat16*>(dsm);   // [IH][IW][64]
+  uint32_t* s_acc = reinterpret_cast<uint32_t*>(dsm + IH * IW * 128);  // [C] when acc
+  __shared__ __align__(16) float s_w[9][64];
+  __shared__ uint32_t s_cnt[8 * 64];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int cg = lane & 7, st = lane >> 3;  // channel group, 4-pixel strip of the warp's row
+  const bool acc = a.emit && a.C <= kMaxAccCols;
+  if (acc)
+    for (int c = threadIdx.x; c < a.C; c += kTileThreads) s_acc[c] = 0u;
+  __syncthreads();
+  pdl_wait();
+  pdl_trigger();
+  if (a.path_out && blockIdx.x == 0 && threadIdx.x == 0) *a.path_out = 3;
+  const OccDev o = a.out_occ;
+  const int ctn = (a.C + 63) / 64;
+  const int tiles_h = (a.Ho + kDwTH - 1) / kDwTH, tiles_w = (a.Wo + kDwTW - 1) / kDwTW;
+  const int per_slice = a.N * tiles_h * tiles_w;
+  const int64_t ntiles = (int64_t)per_slice * ctn;
+  const uint32_t s_in_u32 = smem_u32(s_in);
+  int cur_ct = -1;
+  float sc[8], sh[8];
+  for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+    const int ct = (int)(tile / per_slice);
+    int rest = (int)(tile - (int64_t)ct * per_slice);
+    const int n = rest / (tiles_h * tiles_w);
+    rest -= n * tiles_h * tiles_w;
+    const int ty = rest / tiles_w, tx = rest - (rest / tiles_w) * tiles_w;
+    const int col0 = ct * 64;
+    const int c0 = col0 + cg * 8;
+    const bool cvalid = c0 < a.C;
+    __syncthreads();  // the previous tile's readers of s_in / s_w are done
+    if (ct != cur_ct) {
+      for (int idx = threadIdx.x; idx < 9 * 64; idx += kTileThreads) {
+        const int t = idx / 64, c = idx % 64;
+        s_w[t][c] = (col0 + c < a.C) ? __bfloat162float(a.w[(int64_t)(col0 + c) * 9 + t]) : 0.f;
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        sc[j] = 1.f;
+        sh[j] = 0.f;
+        if (cvalid) epi_affine(a.ep, a.C, c0 + j, sc[j], sh[j]);
+      }
+      cur_ct = ct;
+    }
+    // stage the input tile: 16-byte chunks (8 channels) of IH x IW pixels
+    const int gy0 = ty * kDwTH * S - 1, gx0 = tx * kDwTW * S - 1;
+    const __nv_bfloat16* ximg = a.x + (int64_t)n * a.H * a.W * a.C;
+    for (int idx = threadIdx.x; idx < IH * IW * 8; idx += kTileThreads) {
+      const int p = idx >> 3, ch = idx & 7;
+      const int iy = p / IW, ix = p - (p / IW) * IW;
+      const int gy = gy0 + iy, gx = gx0 + ix;
+      const int cc = col0 + ch * 8;
+      const bool ok = gy >= 0 && gy < a.H && gx >= 0 && gx < a.W && cc < a.C;
+      const __nv_bfloat16* src = ok ? ximg + ((uint32_t)(gy * a.W + gx) * (uint32_t)a.C + cc) : a.x;
+      cp_async_16(s_in_u32 + (uint32_t)(p * 128 + ch * 16), src, ok ? 16u : 0u);
+    }
+    cp_async_commit();
+    cp_async_wait<0>();
+    __syncthreads();
+    // compute: warp = output row of the tile, strip st = pixels 4 st .. 4 st + 3
+    const int oy = warp, ox0 = st * 4;
+    float accv[4][8];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+#pragma unroll
+      for (int k = 0; k < 8; ++k) accv[j][k] = 0.f;
+#pragma unroll
+    for (int r = 0; r < 3; ++r) {
+      float wr[3][8];
+#pragma unroll
+      for (int c = 0; c < 3; ++c) {
+        const float4 w0 = *reinterpret_cast<const float4*>(&s_w[r * 3 + c][cg * 8]);
+        const float4 w1 = *reinterpret_cast<const float4*>(&s_w[r * 3 + c][cg * 8 + 4]);
+        wr[c][0] = w0.x; wr[c][1] = w0.y; wr[c][2] = w0.z; wr[c][3] = w0.w;
+        wr[c][4] = w1.x; wr[c][5] = w1.y; wr[c][6] = w1.z; wr[c][7] = w1.w;
+      }
+      const int iy = oy * S + r;
+#pragma unroll
+      for (int q = 0; q < NCOL; ++q) {  // input column ox0 * S + q
+        float f[8];
+        unpack8(*reinterpret_cast<const uint4*>(&s_in[((iy * IW) + ox0 * S + q) * 64 + cg * 8]), f);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int c = q - j * S;  // kernel column that pixel j applies to this input column
+          if (c >= 0 && c < 3) {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) accv[j][k] = fmaf(f[k], wr[c][k], accv[j][k]);
+          }
+        }
+      }
+    }
+    // epilogue: affine, residual, activation, store, occupancy
+    const int oh = ty * kDwTH + oy;
+    uint32_t cnt[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) cnt[k] = 0u;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int ow = tx * kDwTW + ox0 + j;
+      const bool live = cvalid && oh < a.Ho && ow < a.Wo;
+      const uint32_t mrow = ((uint32_t)n * a.Ho + (oh < a.Ho ? oh : 0)) * a.Wo + (ow < a.Wo ? ow : 0);
+      float rv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      if (a.ep.residual && live) unpack8(*reinterpret_cast<const uint4*>(a.ep.residual + (int64_t)mrow * a.C + c0), rv);
+      float ov[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) ov[k] = epi_act(fmaf(accv[j][k], sc[k], sh[k]) + rv[k], a.ep.act);
+      const uint4 uo = pack8(ov);
+      uint32_t mask = 0u;
+      if (live) {
+        *reinterpret_cast<uint4*>(a.y + (int64_t)mrow * a.C + c0) = uo;
+        mask = nz_mask8(uo);
+      }
+      if (a.emit) {
+        // row bitmap: the strip's 8 lanes hold this pixel's 64 channels
+        const uint32_t b = __ballot_sync(0xffffffffu, mask != 0u);
+        if (cg == 0 && ((b >> (8 * st)) & 0xFFu))
+          atomicOr(&o.row_bm[(int64_t)mrow * o.W64 + (col0 >> 12)], 1ull << ((col0 >> 6) & 63));
+        // block mask: lanes with the same (128-row block, 32-column word) combine first
+        const int blk = live ? (int)(mrow >> 7) : -1;
+        const int word = (col0 >> 5) + (cg >> 2);
+        const int key = blk < 0 ? -1 : blk * 4 + (cg >> 2);
+        const uint32_t grp = __match_any_sync(0xffffffffu, key);
+        const uint32_t bits = __reduce_or_sync(grp, mask << ((cg & 3) * 8));
+        if (blk >= 0 && bits && (__ffs(grp) - 1) == lane && word < o.C32)
+          atomicOr(&o.blk_mask[(int64_t)blk * o.C32 + word], bits);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) cnt[k] += (mask >> k) & 1u;
+      }
+    }
+    if (a.emit) {
+      // column counts: lanes cg, cg + 8, cg + 16, cg + 24 hold one channel group
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        cnt[k] += __shfl_xor_sync(0xffffffffu, cnt[k], 8);
+        cnt[k] += __shfl_xor_sync(0xffffffffu, cnt[k], 16);
+      }
+      if (lane < 8) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) s_cnt[warp * 64 + cg * 8 + k] = cnt[k];
+      }
+      __syncthreads();
+      if (threadIdx.x < 64) {
+        uint32_t c = 0;
+#pragma unroll
+        for (int w = 0; w < kTileThreads / 32; ++w) c += s_cnt[w * 64 + threadIdx.x];
+        const int col = col0 + threadIdx.x;
+        if (acc) {
+          if (col < a.C) s_acc[col] += c;
+        } else {
+          if (c && col < a.C) atomicAdd(&o.col_nnz[col], c);
+          uint32_t sum = col < a.C ? c : 0u;
+#pragma unroll
+          for (int sft = 16; sft > 0; sft >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, sft);
+          if (lane == 0 && sum) {
+            atomicAdd(&o.tile_nnz[col0 >> 6], sum);
+            atomicAdd(o.nnz, (unsigned long long)sum);
+          }
+        }
+      }
+    }
+  }
+  if (a.emit) cta_done(o, s_acc, acc);
+}
+
+// ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kTileThreads)
     maxpool_kernel(const __nv_bfloat16* __restrict__ x, int N, int H, int W, int C, int k,
                    int stride, int pad, int Ho, int Wo, __nv_bfloat16* __restrict__ y, OccDev o_param,
@@ -623,6 +803,25 @@ cudaError_t launch_dwconv(const DwArgs& a, cudaStream_t s) {
   if (R <= 0) return cudaSuccess;
   // the kernel's 32-bit index math: output rows and one image's elements
   if (R >= ((int64_t)1 << 31) || (int64_t)a.H * a.W * a.C >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;
+  if (a.kh == 3 && a.kw == 3 && a.pad == 1 && (a.stride == 1 || a.stride == 2) && (a.C % 8) == 0) {
+    // 2-D tiles with the input staged in shared memory
+    const int tiles = ((a.Ho + kDwTH - 1) / kDwTH) * ((a.Wo + kDwTW - 1) / kDwTW);
+    const int64_t ntiles = (int64_t)a.N * tiles * ((a.C + 63) / 64);
+    if (ntiles >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;
+    const int ih = (kDwTH - 1) * a.stride + 3, iw = (kDwTW - 1) * a.stride + 3;
+    const size_t smem = (size_t)ih * iw * 128 + acc_smem(a.emit, a.C);
+    const int64_t cap = 3LL * device_sm_count();
+    const unsigned grid = (unsigned)(ntiles < cap ? ntiles : cap);
+    auto kern = a.stride == 1 ? dw3_kernel<1> : dw3_kernel<2>;
+    static size_t attr1 = 0, attr2 = 0;
+    size_t& attr = a.stride == 1 ? attr1 : attr2;
+    if (smem > 48 * 1024 && smem > attr) {
+      cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e != cudaSuccess) return e;
+      attr = smem;
+    }
+    return launch_kernel(kern, dim3(grid), dim3(kTileThreads), smem, s, a);
+  }
   return launch_kernel(dwconv_kernel, dim3(tile_grid(R, a.C)), dim3(kTileThreads),
                        acc_smem(a.emit, a.C), s, a);
 }
