@@ -403,169 +403,213 @@ __global__ void __launch_bounds__(kTileThreads) dwconv_kernel(const DwArgs a_par
 // major so a CTA's consecutive tiles keep their weights and affine.
 constexpr int kDwTH = 8, kDwTW = 16;
 
+constexpr int kDwMaxBlk = 16;  // 128-row blocks one output tile can touch (Wo up to ~280)
+
 template <int S>
-__global__ void __launch_bounds__(kTileThreads) dw3_kernel(const DwArgs a_param) {
+__global__ void __launch_bounds__(kTileThreads) dw3_kernel(const DwArgs a_param, int inner) {
   const DwArgs a = a_param;  // registers, not parameter-space loads
   constexpr int IH = (kDwTH - 1) * S + 3, IW = (kDwTW - 1) * S + 3;
   constexpr int NCOL = 3 * S + 3;  // input columns a 4-pixel strip reads: (4 - 1) S + 3
   extern __shared__ __align__(16) uint8_t dsm[];
-  __nv_bfloat16* s_in = reinterpret_cast<__nv_bfloat16*>(dsm);   // [IH][IW][64]
-  uint32_t* s_acc = reinterpret_cast<uint32_t*>(dsm + IH * IW * 128);  // [C] when acc
-  __shared__ __align__(16) float s_w[9][64];
-  __shared__ uint32_t s_cnt[8 * 64];
+  const int Cp = ((a.C + 63) / 64) * 64;  // channels rounded up to whole slices
+  __nv_bfloat16* s_in = reinterpret_cast<__nv_bfloat16*>(dsm);  // [IH][IW][64]
+  float* s_wf = reinterpret_cast<float*>(dsm + IH * IW * 128);   // [9][Cp] weights
+  float* s_sc = s_wf + 9 * Cp;                                   // [Cp] affine scale
+  float* s_sh = s_sc + Cp;                                       // [Cp] affine shift
+  uint32_t* s_acc = reinterpret_cast<uint32_t*>(s_sh + Cp);      // [C] when acc
+  uint32_t* s_blk = s_acc + (a.emit && a.C <= kMaxAccCols ? ((a.C + 3) & ~3) : 0);  // [kDwMaxBlk][C32]
+  __shared__ unsigned long long s_rowbm[kDwTH * kDwTW];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int cg = lane & 7, st = lane >> 3;  // channel group, 4-pixel strip of the warp's row
   const bool acc = a.emit && a.C <= kMaxAccCols;
+  const OccDev o = a.out_occ;
+  // inner: a CTA runs every channel slice of its pixel tile, so it owns the
+  // tile's row-bitmap words (one plain store each) and gathers its block-mask
+  // words in shared memory; otherwise slices are separate work items
+  const bool own = inner != 0;
   if (acc)
     for (int c = threadIdx.x; c < a.C; c += kTileThreads) s_acc[c] = 0u;
-  __syncthreads();
+  if (own && a.emit) {
+    for (int i = threadIdx.x; i < kDwMaxBlk * o.C32; i += kTileThreads) s_blk[i] = 0u;
+    if (threadIdx.x < kDwTH * kDwTW) s_rowbm[threadIdx.x] = 0ull;
+  }
   pdl_wait();
   pdl_trigger();
   if (a.path_out && blockIdx.x == 0 && threadIdx.x == 0) *a.path_out = 3;
-  const OccDev o = a.out_occ;
+  // every channel's weights and affine, once per CTA
+  for (int idx = threadIdx.x; idx < 9 * Cp; idx += kTileThreads) {
+    const int c = idx / 9, t = idx - (idx / 9) * 9;
+    s_wf[t * Cp + c] = c < a.C ? __bfloat162float(a.w[(int64_t)c * 9 + t]) : 0.f;
+  }
+  for (int c = threadIdx.x; c < Cp; c += kTileThreads) {
+    float scv = 1.f, shv = 0.f;
+    if (c < a.C) epi_affine(a.ep, a.C, c, scv, shv);
+    s_sc[c] = scv;
+    s_sh[c] = shv;
+  }
+  __syncthreads();
   const int ctn = (a.C + 63) / 64;
   const int tiles_h = (a.Ho + kDwTH - 1) / kDwTH, tiles_w = (a.Wo + kDwTW - 1) / kDwTW;
-  const int per_slice = a.N * tiles_h * tiles_w;
-  const int64_t ntiles = (int64_t)per_slice * ctn;
+  const int nsp = a.N * tiles_h * tiles_w;
+  const int64_t items = own ? (int64_t)nsp : (int64_t)nsp * ctn;
   const uint32_t s_in_u32 = smem_u32(s_in);
-  int cur_ct = -1;
-  float sc[8], sh[8];
-  for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-    const int ct = (int)(tile / per_slice);
-    int rest = (int)(tile - (int64_t)ct * per_slice);
+  for (int64_t item = blockIdx.x; item < items; item += gridDim.x) {
+    const int ct_begin = own ? 0 : (int)(item / nsp);
+    const int ct_end = own ? ctn : ct_begin + 1;
+    int rest = (int)(own ? item : item - (int64_t)ct_begin * nsp);
     const int n = rest / (tiles_h * tiles_w);
     rest -= n * tiles_h * tiles_w;
     const int ty = rest / tiles_w, tx = rest - (rest / tiles_w) * tiles_w;
-    const int col0 = ct * 64;
-    const int c0 = col0 + cg * 8;
-    const bool cvalid = c0 < a.C;
-    __syncthreads();  // the previous tile's readers of s_in / s_w are done
-    if (ct != cur_ct) {
-      for (int idx = threadIdx.x; idx < 9 * 64; idx += kTileThreads) {
-        const int t = idx / 64, c = idx % 64;
-        s_w[t][c] = (col0 + c < a.C) ? __bfloat162float(a.w[(int64_t)(col0 + c) * 9 + t]) : 0.f;
+    // first 128-row block the tile touches (block-mask words gathered relative to it)
+    const int b0 = (int)((((uint32_t)n * a.Ho + ty * kDwTH) * a.Wo + tx * kDwTW) >> 7);
+    for (int ct = ct_begin; ct < ct_end; ++ct) {
+      const int col0 = ct * 64;
+      const int c0 = col0 + cg * 8;
+      const bool cvalid = c0 < a.C;
+      __syncthreads();  // the previous slice's readers of s_in are done
+      // stage the input tile: 16-byte chunks (8 channels) of IH x IW pixels
+      const int gy0 = ty * kDwTH * S - 1, gx0 = tx * kDwTW * S - 1;
+      const __nv_bfloat16* ximg = a.x + (int64_t)n * a.H * a.W * a.C;
+      for (int idx = threadIdx.x; idx < IH * IW * 8; idx += kTileThreads) {
+        const int p = idx >> 3, ch = idx & 7;
+        const int iy = p / IW, ix = p - (p / IW) * IW;
+        const int gy = gy0 + iy, gx = gx0 + ix;
+        const int cc = col0 + ch * 8;
+        const bool ok = gy >= 0 && gy < a.H && gx >= 0 && gx < a.W && cc < a.C;
+        const __nv_bfloat16* src = ok ? ximg + ((uint32_t)(gy * a.W + gx) * (uint32_t)a.C + cc) : a.x;
+        cp_async_16(s_in_u32 + (uint32_t)(p * 128 + ch * 16), src, ok ? 16u : 0u);
       }
+      cp_async_commit();
+      cp_async_wait<0>();
+      __syncthreads();
+      // compute: warp = output row of the tile, strip st = pixels 4 st .. 4 st + 3
+      const int oy = warp, ox0 = st * 4;
+      float accv[4][8];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        sc[j] = 1.f;
-        sh[j] = 0.f;
-        if (cvalid) epi_affine(a.ep, a.C, c0 + j, sc[j], sh[j]);
+      for (int j = 0; j < 4; ++j)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) accv[j][k] = 0.f;
+#pragma unroll
+      for (int r = 0; r < 3; ++r) {
+        float wr[3][8];
+#pragma unroll
+        for (int c = 0; c < 3; ++c) {
+          const float4 w0 = *reinterpret_cast<const float4*>(&s_wf[(r * 3 + c) * Cp + c0]);
+          const float4 w1 = *reinterpret_cast<const float4*>(&s_wf[(r * 3 + c) * Cp + c0 + 4]);
+          wr[c][0] = w0.x; wr[c][1] = w0.y; wr[c][2] = w0.z; wr[c][3] = w0.w;
+          wr[c][4] = w1.x; wr[c][5] = w1.y; wr[c][6] = w1.z; wr[c][7] = w1.w;
+        }
+        const int iy = oy * S + r;
+#pragma unroll
+        for (int q = 0; q < NCOL; ++q) {  // input column ox0 * S + q
+          float f[8];
+          unpack8(*reinterpret_cast<const uint4*>(&s_in[((iy * IW) + ox0 * S + q) * 64 + cg * 8]), f);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int c = q - j * S;  // kernel column that pixel j applies to this input column
+            if (c >= 0 && c < 3) {
+#pragma unroll
+              for (int k = 0; k < 8; ++k) accv[j][k] = fmaf(f[k], wr[c][k], accv[j][k]);
+            }
+          }
+        }
       }
-      cur_ct = ct;
-    }
-    // stage the input tile: 16-byte chunks (8 channels) of IH x IW pixels
-    const int gy0 = ty * kDwTH * S - 1, gx0 = tx * kDwTW * S - 1;
-    const __nv_bfloat16* ximg = a.x + (int64_t)n * a.H * a.W * a.C;
-    for (int idx = threadIdx.x; idx < IH * IW * 8; idx += kTileThreads) {
-      const int p = idx >> 3, ch = idx & 7;
-      const int iy = p / IW, ix = p - (p / IW) * IW;
-      const int gy = gy0 + iy, gx = gx0 + ix;
-      const int cc = col0 + ch * 8;
-      const bool ok = gy >= 0 && gy < a.H && gx >= 0 && gx < a.W && cc < a.C;
-      const __nv_bfloat16* src = ok ? ximg + ((uint32_t)(gy * a.W + gx) * (uint32_t)a.C + cc) : a.x;
-      cp_async_16(s_in_u32 + (uint32_t)(p * 128 + ch * 16), src, ok ? 16u : 0u);
-    }
-    cp_async_commit();
-    cp_async_wait<0>();
-    __syncthreads();
-    // compute: warp = output row of the tile, strip st = pixels 4 st .. 4 st + 3
-    const int oy = warp, ox0 = st * 4;
-    float accv[4][8];
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-#pragma unroll
-      for (int k = 0; k < 8; ++k) accv[j][k] = 0.f;
-#pragma unroll
-    for (int r = 0; r < 3; ++r) {
-      float wr[3][8];
-#pragma unroll
-      for (int c = 0; c < 3; ++c) {
-        const float4 w0 = *reinterpret_cast<const float4*>(&s_w[r * 3 + c][cg * 8]);
-        const float4 w1 = *reinterpret_cast<const float4*>(&s_w[r * 3 + c][cg * 8 + 4]);
-        wr[c][0] = w0.x; wr[c][1] = w0.y; wr[c][2] = w0.z; wr[c][3] = w0.w;
-        wr[c][4] = w1.x; wr[c][5] = w1.y; wr[c][6] = w1.z; wr[c][7] = w1.w;
+      // epilogue: affine, residual, activation, store, occupancy
+      const int oh = ty * kDwTH + oy;
+      float sc[8], sh[8];
+      {
+        const float4 a0 = *reinterpret_cast<const float4*>(&s_sc[c0]);
+        const float4 a1 = *reinterpret_cast<const float4*>(&s_sc[c0 + 4]);
+        const float4 b0v = *reinterpret_cast<const float4*>(&s_sh[c0]);
+        const float4 b1v = *reinterpret_cast<const float4*>(&s_sh[c0 + 4]);
+        sc[0] = a0.x; sc[1] = a0.y; sc[2] = a0.z; sc[3] = a0.w; sc[4] = a1.x; sc[5] = a1.y; sc[6] = a1.z; sc[7] = a1.w;
+        sh[0] = b0v.x; sh[1] = b0v.y; sh[2] = b0v.z; sh[3] = b0v.w; sh[4] = b1v.x; sh[5] = b1v.y; sh[6] = b1v.z; sh[7] = b1v.w;
       }
-      const int iy = oy * S + r;
+      uint32_t cnt[8];
 #pragma unroll
-      for (int q = 0; q < NCOL; ++q) {  // input column ox0 * S + q
-        float f[8];
-        unpack8(*reinterpret_cast<const uint4*>(&s_in[((iy * IW) + ox0 * S + q) * 64 + cg * 8]), f);
+      for (int k = 0; k < 8; ++k) cnt[k] = 0u;
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int c = q - j * S;  // kernel column that pixel j applies to this input column
-          if (c >= 0 && c < 3) {
+      for (int j = 0; j < 4; ++j) {
+        const int ow = tx * kDwTW + ox0 + j;
+        const bool live = cvalid && oh < a.Ho && ow < a.Wo;
+        const uint32_t mrow = ((uint32_t)n * a.Ho + (oh < a.Ho ? oh : 0)) * a.Wo + (ow < a.Wo ? ow : 0);
+        float rv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        if (a.ep.residual && live) unpack8(*reinterpret_cast<const uint4*>(a.ep.residual + (int64_t)mrow * a.C + c0), rv);
+        float ov[8];
 #pragma unroll
-            for (int k = 0; k < 8; ++k) accv[j][k] = fmaf(f[k], wr[c][k], accv[j][k]);
+        for (int k = 0; k < 8; ++k) ov[k] = epi_act(fmaf(accv[j][k], sc[k], sh[k]) + rv[k], a.ep.act);
+        const uint4 uo = pack8(ov);
+        uint32_t mask = 0u;
+        if (live) {
+          *reinterpret_cast<uint4*>(a.y + (int64_t)mrow * a.C + c0) = uo;
+          mask = nz_mask8(uo);
+        }
+        if (a.emit) {
+          // row bitmap: the strip's 8 lanes hold this pixel's 64 channels
+          const uint32_t b = __ballot_sync(0xffffffffu, mask != 0u);
+          if (cg == 0 && ((b >> (8 * st)) & 0xFFu)) {
+            const unsigned long long bit = 1ull << ((col0 >> 6) & 63);
+            if (own) atomicOr(&s_rowbm[oy * kDwTW + ox0 + j], bit);
+            else atomicOr(&o.row_bm[(int64_t)mrow * o.W64 + (col0 >> 12)], bit);
+          }
+          // block mask: OR over the 4 lanes of one 32-column word, then one add
+          uint32_t bits = mask << ((cg & 3) * 8);
+          bits |= __shfl_xor_sync(0xffffffffu, bits, 1);
+          bits |= __shfl_xor_sync(0xffffffffu, bits, 2);
+          const int word = (col0 >> 5) + (cg >> 2);
+          if ((cg & 3) == 0 && bits && word < o.C32) {
+            const int lb = (int)(mrow >> 7) - b0;
+            if (own && lb >= 0 && lb < kDwMaxBlk) atomicOr(&s_blk[lb * o.C32 + word], bits);
+            else atomicOr(&o.blk_mask[(int64_t)(mrow >> 7) * o.C32 + word], bits);
+          }
+#pragma unroll
+          for (int k = 0; k < 8; ++k) cnt[k] += (mask >> k) & 1u;
+        }
+      }
+      if (a.emit) {
+        // column counts: lanes cg, cg + 8, cg + 16, cg + 24 hold one channel
+        // group; its first lane adds them (shared-memory atomics, no barrier)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          cnt[k] += __shfl_xor_sync(0xffffffffu, cnt[k], 8);
+          cnt[k] += __shfl_xor_sync(0xffffffffu, cnt[k], 16);
+        }
+        if (lane < 8 && cvalid) {
+          if (acc) {
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+              if (cnt[k]) atomicAdd(&s_acc[c0 + k], cnt[k]);
+          } else {
+            uint32_t sum = 0u;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              if (cnt[k]) atomicAdd(&o.col_nnz[c0 + k], cnt[k]);
+              sum += cnt[k];
+            }
+            if (sum) {
+              atomicAdd(&o.tile_nnz[col0 >> 6], sum);
+              atomicAdd(o.nnz, (unsigned long long)sum);
+            }
           }
         }
       }
     }
-    // epilogue: affine, residual, activation, store, occupancy
-    const int oh = ty * kDwTH + oy;
-    uint32_t cnt[8];
-#pragma unroll
-    for (int k = 0; k < 8; ++k) cnt[k] = 0u;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int ow = tx * kDwTW + ox0 + j;
-      const bool live = cvalid && oh < a.Ho && ow < a.Wo;
-      const uint32_t mrow = ((uint32_t)n * a.Ho + (oh < a.Ho ? oh : 0)) * a.Wo + (ow < a.Wo ? ow : 0);
-      float rv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      if (a.ep.residual && live) unpack8(*reinterpret_cast<const uint4*>(a.ep.residual + (int64_t)mrow * a.C + c0), rv);
-      float ov[8];
-#pragma unroll
-      for (int k = 0; k < 8; ++k) ov[k] = epi_act(fmaf(accv[j][k], sc[k], sh[k]) + rv[k], a.ep.act);
-      const uint4 uo = pack8(ov);
-      uint32_t mask = 0u;
-      if (live) {
-        *reinterpret_cast<uint4*>(a.y + (int64_t)mrow * a.C + c0) = uo;
-        mask = nz_mask8(uo);
-      }
-      if (a.emit) {
-        // row bitmap: the strip's 8 lanes hold this pixel's 64 channels
-        const uint32_t b = __ballot_sync(0xffffffffu, mask != 0u);
-        if (cg == 0 && ((b >> (8 * st)) & 0xFFu))
-          atomicOr(&o.row_bm[(int64_t)mrow * o.W64 + (col0 >> 12)], 1ull << ((col0 >> 6) & 63));
-        // block mask: lanes with the same (128-row block, 32-column word) combine first
-        const int blk = live ? (int)(mrow >> 7) : -1;
-        const int word = (col0 >> 5) + (cg >> 2);
-        const int key = blk < 0 ? -1 : blk * 4 + (cg >> 2);
-        const uint32_t grp = __match_any_sync(0xffffffffu, key);
-        const uint32_t bits = __reduce_or_sync(grp, mask << ((cg & 3) * 8));
-        if (blk >= 0 && bits && (__ffs(grp) - 1) == lane && word < o.C32)
-          atomicOr(&o.blk_mask[(int64_t)blk * o.C32 + word], bits);
-#pragma unroll
-        for (int k = 0; k < 8; ++k) cnt[k] += (mask >> k) & 1u;
-      }
-    }
-    if (a.emit) {
-      // column counts: lanes cg, cg + 8, cg + 16, cg + 24 hold one channel group
-#pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        cnt[k] += __shfl_xor_sync(0xffffffffu, cnt[k], 8);
-        cnt[k] += __shfl_xor_sync(0xffffffffu, cnt[k], 16);
-      }
-      if (lane < 8) {
-#pragma unroll
-        for (int k = 0; k < 8; ++k) s_cnt[warp * 64 + cg * 8 + k] = cnt[k];
-      }
+    if (own && a.emit) {
+      // the tile's row words (owned: plain stores) and its block-mask words
       __syncthreads();
-      if (threadIdx.x < 64) {
-        uint32_t c = 0;
-#pragma unroll
-        for (int w = 0; w < kTileThreads / 32; ++w) c += s_cnt[w * 64 + threadIdx.x];
-        const int col = col0 + threadIdx.x;
-        if (acc) {
-          if (col < a.C) s_acc[col] += c;
-        } else {
-          if (c && col < a.C) atomicAdd(&o.col_nnz[col], c);
-          uint32_t sum = col < a.C ? c : 0u;
-#pragma unroll
-          for (int sft = 16; sft > 0; sft >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, sft);
-          if (lane == 0 && sum) {
-            atomicAdd(&o.tile_nnz[col0 >> 6], sum);
-            atomicAdd(o.nnz, (unsigned long long)sum);
-          }
+      if (threadIdx.x < kDwTH * kDwTW) {
+        const int oy = threadIdx.x / kDwTW, ox = threadIdx.x - (threadIdx.x / kDwTW) * kDwTW;
+        const int oh = ty * kDwTH + oy, ow = tx * kDwTW + ox;
+        if (oh < a.Ho && ow < a.Wo)
+          o.row_bm[(int64_t)(((uint32_t)n * a.Ho + oh) * a.Wo + ow) * o.W64] = s_rowbm[threadIdx.x];
+        s_rowbm[threadIdx.x] = 0ull;
+      }
+      for (int i = threadIdx.x; i < kDwMaxBlk * o.C32; i += kTileThreads) {
+        const uint32_t v = s_blk[i];
+        if (v) {
+          const int lb = i / o.C32, w = i - (i / o.C32) * o.C32;
+          atomicOr(&o.blk_mask[(int64_t)(b0 + lb) * o.C32 + w], v);
+          s_blk[i] = 0u;
         }
       }
     }
@@ -801,17 +845,25 @@ cudaError_t launch_pad_channels(const __nv_bfloat16* x, int64_t P, int C, int Cp
 cudaError_t launch_dwconv(const DwArgs& a, cudaStream_t s) {
   const int64_t R = (int64_t)a.N * a.Ho * a.Wo;
   if (R <= 0) return cudaSuccess;
-  // the kernel's 32-bit index math: output rows and one image's elements
+  // the kernels' 32-bit index math: output rows and one image's elements
   if (R >= ((int64_t)1 << 31) || (int64_t)a.H * a.W * a.C >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;
-  if (a.kh == 3 && a.kw == 3 && a.pad == 1 && (a.stride == 1 || a.stride == 2) && (a.C % 8) == 0) {
-    // 2-D tiles with the input staged in shared memory
-    const int tiles = ((a.Ho + kDwTH - 1) / kDwTH) * ((a.Wo + kDwTW - 1) / kDwTW);
-    const int64_t ntiles = (int64_t)a.N * tiles * ((a.C + 63) / 64);
-    if (ntiles >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;
-    const int ih = (kDwTH - 1) * a.stride + 3, iw = (kDwTW - 1) * a.stride + 3;
-    const size_t smem = (size_t)ih * iw * 128 + acc_smem(a.emit, a.C);
+  const bool shape3 = a.kh == 3 && a.kw == 3 && a.pad == 1 && (a.stride == 1 || a.stride == 2) && (a.C % 8) == 0;
+  const int tiles = ((a.Ho + kDwTH - 1) / kDwTH) * ((a.Wo + kDwTW - 1) / kDwTW);
+  const int64_t nsp = (int64_t)a.N * tiles;
+  const int64_t ntiles = nsp * ((a.C + 63) / 64);
+  const int ih = (kDwTH - 1) * a.stride + 3, iw = (kDwTW - 1) * a.stride + 3;
+  const int C32 = (a.C + 31) / 32;
+  const int Cp = ((a.C + 63) / 64) * 64;
+  const size_t acc_b = a.emit && a.C <= kMaxAccCols ? sizeof(uint32_t) * (size_t)((a.C + 3) & ~3) : 0;
+  const size_t smem = (size_t)ih * iw * 128 + sizeof(float) * 11 * (size_t)Cp + acc_b +
+                      sizeof(uint32_t) * (size_t)kDwMaxBlk * C32;
+  if (shape3 && ntiles < ((int64_t)1 << 31) && smem <= 200 * 1024) {
+    // 2-D tiles with the input staged in shared memory; one CTA runs every
+    // channel slice of its pixel tile when that still fills the GPU
     const int64_t cap = 3LL * device_sm_count();
-    const unsigned grid = (unsigned)(ntiles < cap ? ntiles : cap);
+    const int inner = (nsp >= 2LL * device_sm_count() && a.C <= 4096) ? 1 : 0;
+    const int64_t items = inner ? nsp : ntiles;
+    const unsigned grid = (unsigned)(items < cap ? items : cap);
     auto kern = a.stride == 1 ? dw3_kernel<1> : dw3_kernel<2>;
     static size_t attr1 = 0, attr2 = 0;
     size_t& attr = a.stride == 1 ? attr1 : attr2;
@@ -820,7 +872,7 @@ cudaError_t launch_dwconv(const DwArgs& a, cudaStream_t s) {
       if (e != cudaSuccess) return e;
       attr = smem;
     }
-    return launch_kernel(kern, dim3(grid), dim3(kTileThreads), smem, s, a);
+    return launch_kernel(kern, dim3(grid), dim3(kTileThreads), smem, s, a, inner);
   }
   return launch_kernel(dwconv_kernel, dim3(tile_grid(R, a.C)), dim3(kTileThreads),
                        acc_smem(a.emit, a.C), s, a);
