@@ -212,7 +212,7 @@ sparoa_status offer_splitk(sparoa_ctx* ctx, IgemmArgs* a) {
 // stats kernel writes the bitmaps whole).
 sparoa_status run_stats(sparoa_ctx* ctx, const void* x, int64_t R, int64_t C,
                         const sparoa_occupancy& o) {
-  SP_TRY(occ_clear(ctx, o, C <= kStatsWholeRowCols));
+  SP_TRY(occ_clear(ctx, o, stats_writes_rows_whole(R, (int)C)));
   SP_CUDA(launch_stats(static_cast<const __nv_bfloat16*>(x), R, (int)C, to_dev(o), ctx->stream));
   return SPAROA_OK;
 }

@@ -4,13 +4,18 @@
 // the columns k that hold a non-zero in that block take part (Sec. 2.1:
 // products with a zero activation are skipped without changing the output).
 // The block-column mask of x (one bit per column per 128-row block) gives the
-// occupied columns; the kernel compacts them into a list, gathers those
-// columns of x and the matching rows of W stored as [K, N] (each a contiguous
-// run of N values, so skipped columns cost no HBM traffic), and accumulates in
-// fp32 on the CUDA cores.  This is the path for small-M layers (a batch of
-// feature vectors), which are bound by the weight bytes, not by arithmetic.
+// occupied columns; the kernel compacts them into a list and reads only the
+// matching rows of W stored as [K, N] (each a contiguous run of N values, so
+// skipped columns cost no HBM traffic), accumulating in fp32 on the CUDA
+// cores.  This is the path for small-M layers (a batch of feature vectors),
+// which are bound by the weight bytes and by latency, not by arithmetic.
 //
-// CTA = 128 rows x 64 output columns, 256 threads, each owning 8 x 4 outputs.
+// CTA = 64 rows x 16 output columns (many CTAs even for a handful of rows),
+// 256 threads, each owning one row x 4 columns.  Per window of kKW columns of
+// K the CTA stages its x rows whole (coalesced cp.async; the padded pitch
+// spreads the per-row reads over the banks) and the W-row slices of the
+// window's occupied columns (fp32), then every thread runs over the occupied
+// columns only.
 #include "sparoa_kernels.h"
 
 namespace sparoa {
@@ -18,15 +23,29 @@ namespace sparoa {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kKC = 32;   // compacted columns per chunk
+constexpr int kTM = 64;           // rows per CTA
+constexpr int kTN = 16;           // output columns per CTA
+constexpr int kKW = 512;          // K window staged at once
+constexpr int kPitch = kKW + 8;   // bf16 elements per staged x row (16-byte multiple)
+
+constexpr int kMaxWin = 32;       // K windows (K <= kMaxWin * kKW)
+
+struct FcSmem {
+  static constexpr size_t kX = (size_t)kTM * kPitch * 2;   // x window, bf16, rows whole
+  static constexpr size_t kXC = (size_t)kKW * kTM * 2;     // occupied columns of it, [k][row], bf16
+  static constexpr size_t kW = (size_t)kKW * kTN * 4;      // occupied W rows, fp32
+  static constexpr size_t kBytes = kX + kXC + kW + (kMaxWin + 2) * 4;  // + window starts, count
+};
 
 __global__ void __launch_bounds__(kThreads) fcskip_kernel(const FcSkipArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
-  float* xs = reinterpret_cast<float*>(smem);               // [kKC][128]
-  float* ws = xs + kKC * 128;                               // [kKC][64]
-  uint64_t* s_nz = reinterpret_cast<uint64_t*>(ws + kKC * 64);  // [128]
-  int* s_cnt = reinterpret_cast<int*>(s_nz + 128);
-  int* cols = s_cnt + 4;                                    // [K]
+  __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(smem);                   // [kTM][kPitch]
+  __nv_bfloat16* xc = reinterpret_cast<__nv_bfloat16*>(smem + FcSmem::kX);      // [kk][kTM]
+  float* ws = reinterpret_cast<float*>(smem + FcSmem::kX + FcSmem::kXC);        // [kk][kTN]
+  int* s_misc = reinterpret_cast<int*>(smem + FcSmem::kX + FcSmem::kXC + FcSmem::kW);  // [0] count, [1..] window starts
+  short* s_col = reinterpret_cast<short*>(smem + FcSmem::kBytes);               // [K] occupied columns (< 32768)
+  __shared__ uint32_t s_cnt[kTN];
+  __shared__ uint32_t s_blk;
 
   pdl_wait();
   pdl_trigger();
@@ -34,16 +53,18 @@ __global__ void __launch_bounds__(kThreads) fcskip_kernel(const FcSkipArgs a) {
   if (path != 2) return;  // the dense kernel of this launch runs instead
   record_path(a.disp, path);
 
-  const int n0 = blockIdx.x * 64;
-  const int64_t m0 = (int64_t)blockIdx.y * 128;
-  const int tid = threadIdx.x;
-  const int warp = tid >> 5, lane = tid & 31;
+  const int n0 = blockIdx.x * kTN;
+  const int64_t m0 = (int64_t)blockIdx.y * kTM;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int row = tid >> 2, cq = tid & 3;  // this thread's row and 4-column group
+  const int64_t m = m0 + row;
 
-  // 1. occupied columns of this row block, in increasing order
+  // 1. occupied columns of the rows' 128-row block, in increasing order
   if (warp == 0) {
+    const int rb = (int)(m0 >> 7);
     int base = 0;
     for (int w0 = 0; w0 < a.in_C32; w0 += 32) {
-      uint32_t word = (w0 + lane < a.in_C32) ? a.in_blk[blockIdx.y * a.in_C32 + w0 + lane] : 0u;
+      uint32_t word = (w0 + lane < a.in_C32) ? a.in_blk[(int64_t)rb * a.in_C32 + w0 + lane] : 0u;
       const int cnt = __popc(word);
       int incl = cnt;
 #pragma unroll
@@ -54,94 +75,100 @@ __global__ void __launch_bounds__(kThreads) fcskip_kernel(const FcSkipArgs a) {
       int off = base + incl - cnt;
       while (word) {
         const int b = __ffs(word) - 1;
-        cols[off++] = (w0 + lane) * 32 + b;
+        const int k = (w0 + lane) * 32 + b;
+        if (k < a.K) s_col[off++] = (short)k;
         word &= word - 1;
       }
       base += __shfl_sync(0xffffffffu, incl, 31);
     }
-    if (lane == 0) *s_cnt = base;
+    if (lane == 0) s_misc[0] = base < a.K ? base : a.K;
   }
-  if (tid < 128) s_nz[tid] = 0ull;
+  if (tid < kTN) s_cnt[tid] = 0u;
+  if (tid == 0) s_blk = 0u;
   __syncthreads();
-  const int kc_total = *s_cnt;
-
-  const int rg = tid >> 4;   // rows rg*8 .. +8
-  const int cq = tid & 15;   // cols cq*4 .. +4
-  float acc[8][4];
-#pragma unroll
-  for (int i = 0; i < 8; ++i)
-#pragma unroll
-    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
-
-  for (int kc = 0; kc < kc_total; kc += kKC) {
-    // 2a. gather x[m0 + row, cols[kc + k]] -> xs[k][row]
-    {
-      const int row = tid >> 1, half = tid & 1;
-      const int64_t m = m0 + row;
-#pragma unroll 4
-      for (int j = 0; j < 16; ++j) {
-        const int k = kc + half * 16 + j;
-        float v = 0.f;
-        if (k < kc_total && m < a.M) v = __bfloat162float(a.x[m * a.K + cols[k]]);
-        xs[(half * 16 + j) * 128 + row] = v;
-      }
+  const int nocc = s_misc[0];
+  // where each K window starts in the (sorted) occupied list: binary search
+  const int nwin = (a.K + kKW - 1) / kKW;
+  if (tid <= nwin) {
+    const int bound = tid * kKW;
+    int lo = 0, hi = nocc;
+    while (lo < hi) {
+      const int mid = (lo + hi) >> 1;
+      if (s_col[mid] < bound) lo = mid + 1;
+      else hi = mid;
     }
-    // 2b. W_kn[cols[kc + kr], n0 .. n0+64) -> ws[kr][*]
-    {
-      const int kr = tid >> 3, cg = tid & 7;
-      const int k = kc + kr;
-      const int n = n0 + cg * 8;
-      float f[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      if (k < kc_total && n < a.N) {
-        const uint4 u = __ldg(reinterpret_cast<const uint4*>(a.w_kn + (int64_t)cols[k] * a.N + n));
-        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+    s_misc[1 + tid] = lo;
+  }
+  __syncthreads();
+
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  const uint32_t xs_u32 = smem_u32(xs);
+  for (int win = 0; win < nwin; ++win) {
+    const int k0 = win * kKW;
+    const int kw = a.K - k0 < kKW ? a.K - k0 : kKW;
+    const int oc = s_misc[1 + win];
+    const int nk = s_misc[2 + win] - oc;  // occupied columns of this window
+    if (nk > 0) {
+      // 2a. x rows of the window: 16-byte chunks, zero-filled past M
+      const int chunks = kw / 8;  // K % 8 == 0
+      for (int idx = tid; idx < kTM * chunks; idx += kThreads) {
+        const int r = idx / chunks, c = idx - (idx / chunks) * chunks;
+        const bool ok = m0 + r < a.M;
+        const __nv_bfloat16* src = ok ? a.x + (m0 + r) * a.K + k0 + c * 8 : a.x;
+        cp_async_16(xs_u32 + (uint32_t)((r * kPitch + c * 8) * 2), src, ok ? 16u : 0u);
+      }
+      cp_async_commit();
+      // 2b. W rows of the window's occupied columns, columns n0 .. n0 + 16
+      for (int idx = tid; idx < nk * (kTN / 8); idx += kThreads) {
+        const int kk = idx >> 1, h = idx & 1;
+        const int n = n0 + h * 8;
+        float f[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        if (n + 8 <= a.N) {
+          const uint4 u = __ldg(reinterpret_cast<const uint4*>(a.w_kn + (int64_t)s_col[oc + kk] * a.N + n));
+          const __nv_bfloat162* hp = reinterpret_cast<const __nv_bfloat162*>(&u);
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const float2 t = __bfloat1622float2(h[j]);
-          f[2 * j] = t.x;
-          f[2 * j + 1] = t.y;
+          for (int j = 0; j < 4; ++j) {
+            const float2 t = __bfloat1622float2(hp[j]);
+            f[2 * j] = t.x;
+            f[2 * j + 1] = t.y;
+          }
         }
+        float4* dst = reinterpret_cast<float4*>(ws + kk * kTN + h * 8);
+        dst[0] = make_float4(f[0], f[1], f[2], f[3]);
+        dst[1] = make_float4(f[4], f[5], f[6], f[7]);
       }
-#pragma unroll
-      for (int j = 0; j < 8; ++j) ws[kr * 64 + cg * 8 + j] = f[j];
-    }
-    __syncthreads();
-    // 2c. accumulate
+      cp_async_wait<0>();
+      __syncthreads();
+      // 2c. the occupied columns of x, compacted to [kk][row]
+      for (int idx = tid; idx < nk * kTM; idx += kThreads) {
+        const int kk = idx / kTM, r = idx - (idx / kTM) * kTM;
+        xc[idx] = xs[r * kPitch + (s_col[oc + kk] - k0)];
+      }
+      __syncthreads();
+      // 2d. accumulate over the occupied columns only
 #pragma unroll 8
-    for (int k = 0; k < kKC; ++k) {
-      const float4 a0 = *reinterpret_cast<const float4*>(&xs[k * 128 + rg * 8]);
-      const float4 a1 = *reinterpret_cast<const float4*>(&xs[k * 128 + rg * 8 + 4]);
-      const float4 b = *reinterpret_cast<const float4*>(&ws[k * 64 + cq * 4]);
-      const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-      const float bv[4] = {b.x, b.y, b.z, b.w};
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+      for (int kk = 0; kk < nk; ++kk) {
+        const float xv = __bfloat162float(xc[kk * kTM + row]);
+        const float4 wv = *reinterpret_cast<const float4*>(ws + kk * kTN + cq * 4);
+        acc[0] = fmaf(xv, wv.x, acc[0]);
+        acc[1] = fmaf(xv, wv.y, acc[1]);
+        acc[2] = fmaf(xv, wv.z, acc[2]);
+        acc[3] = fmaf(xv, wv.w, acc[3]);
+      }
+      __syncthreads();  // window buffers free for the next window
     }
-    __syncthreads();
   }
 
   // 3. epilogue
-  float sc[4], sh[4];
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    sc[j] = 1.f;
-    sh[j] = 0.f;
-    const int n = n0 + cq * 4 + j;
-    if (n < a.N) epi_affine(a.ep, a.N, n, sc[j], sh[j]);
-  }
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int row = rg * 8 + i;
-    const int64_t m = m0 + row;
-    if (m >= a.M) continue;
-    uint32_t bits = 0;
+  uint32_t bits = 0u;
+  if (m < a.M) {
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const int n = n0 + cq * 4 + j;
       if (n >= a.N) continue;
-      float v = fmaf(acc[i][j], sc[j], sh[j]);
+      float scv = 1.f, shv = 0.f;
+      epi_affine(a.ep, a.N, n, scv, shv);
+      float v = fmaf(acc[j], scv, shv);
       if (a.ep.residual) v += __bfloat162float(a.ep.residual[m * a.N + n]);
       v = epi_act(v, a.ep.act);
       if (a.y_f32) {
@@ -152,12 +179,37 @@ __global__ void __launch_bounds__(kThreads) fcskip_kernel(const FcSkipArgs a) {
         if (bf16_nz(__bfloat16_as_ushort(o))) bits |= 1u << j;
       }
     }
-    if (a.emit && bits) atomicOr(reinterpret_cast<unsigned long long*>(&s_nz[row]),
-                                 (unsigned long long)bits << (cq * 4));
   }
   if (a.emit) {
+    const OccDev o = a.out_occ;
+    // the row's 16 columns: 4 lanes (cq) per row
+    uint32_t rb16 = bits << (cq * 4);
+    rb16 |= __shfl_xor_sync(0xffffffffu, rb16, 1);
+    rb16 |= __shfl_xor_sync(0xffffffffu, rb16, 2);
+    if (cq == 0 && rb16 && m < a.M)
+      atomicOr(&o.row_bm[m * o.W64 + (n0 >> 12)], 1ull << ((n0 >> 6) & 63));
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if ((bits >> j) & 1u) atomicAdd(&s_cnt[cq * 4 + j], 1u);
+    // block mask: the 16 columns' bits over the CTA's rows (one 128-row block)
+    const uint32_t wbits = __reduce_or_sync(0xffffffffu, rb16);
+    if (lane == 0 && wbits) atomicOr(&s_blk, wbits);
     __syncthreads();
-    flush_tile(s_nz, m0, n0, a.out_occ, tid, kThreads);
+    if (tid < kTN) {
+      const uint32_t c = s_cnt[tid];
+      const int n = n0 + tid;
+      if (c && n < a.N) atomicAdd(&o.col_nnz[n], c);
+    }
+    if (tid == 0) {
+      uint32_t sum = 0u;
+      for (int j = 0; j < kTN; ++j) sum += s_cnt[j];
+      const int w = n0 >> 5;
+      if (s_blk && w < o.C32) atomicOr(&o.blk_mask[(m0 >> 7) * o.C32 + w], s_blk << (n0 & 31));
+      if (sum) {
+        atomicAdd(&o.tile_nnz[n0 >> 6], sum);
+        atomicAdd(o.nnz, (unsigned long long)sum);
+      }
+    }
   }
 }
 
@@ -165,7 +217,8 @@ __global__ void __launch_bounds__(kThreads) fcskip_kernel(const FcSkipArgs a) {
 
 cudaError_t launch_fcskip(const FcSkipArgs& a, cudaStream_t s) {
   if (a.M <= 0 || a.N <= 0) return cudaSuccess;
-  const size_t smem = (size_t)kKC * 128 * 4 + (size_t)kKC * 64 * 4 + 128 * 8 + 16 + (size_t)a.K * 4;
+  if (a.K % 8 != 0 || a.N % 8 != 0 || a.K > kMaxWin * kKW) return cudaErrorInvalidValue;
+  const size_t smem = FcSmem::kBytes + (size_t)a.K * sizeof(short);
   static size_t attr = 0;
   if (smem > 48 * 1024 && smem > attr) {
     cudaError_t e = cudaFuncSetAttribute(fcskip_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -173,7 +226,7 @@ cudaError_t launch_fcskip(const FcSkipArgs& a, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     attr = smem;
   }
-  dim3 grid((a.N + 63) / 64, (a.M + 127) / 128);
+  dim3 grid((a.N + kTN - 1) / kTN, (a.M + kTM - 1) / kTM);
   return launch_kernel(fcskip_kernel, grid, dim3(kThreads), smem, s, a);
 }
 

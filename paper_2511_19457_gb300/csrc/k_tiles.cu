@@ -177,7 +177,8 @@ __device__ __forceinline__ void stats_load(const __nv_bfloat16* __restrict__ x, 
 }
 
 __global__ void __launch_bounds__(kTileThreads) stats_kernel(const __nv_bfloat16* __restrict__ x,
-                                                             int64_t R, int C, OccDev o_param) {
+                                                             int64_t R, int C, OccDev o_param,
+                                                             int chunk) {
   const OccDev o = o_param;  // registers, not parameter-space loads
   extern __shared__ uint32_t s_acc[];  // [C] when acc
   __shared__ uint32_t s_cnt[8 * 64];
@@ -186,7 +187,7 @@ __global__ void __launch_bounds__(kTileThreads) stats_kernel(const __nv_bfloat16
   const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
   const bool vec = (C & 7) == 0;
   const int ctn = (C + 63) / 64;
-  const int nch = (ctn + kStatsChunk - 1) / kStatsChunk;
+  const int nch = (ctn + chunk - 1) / chunk;
   const bool own_row = nch == 1;  // one chunk holds every tile of a row
   const int64_t nrb = (R + 127) / 128;
   const int64_t items = nrb * nch;
@@ -199,8 +200,8 @@ __global__ void __launch_bounds__(kTileThreads) stats_kernel(const __nv_bfloat16
     const int64_t rb = item / nch;
     const int ch = (int)(item - rb * nch);
     const int64_t row0 = rb * 128;
-    const int ct0 = ch * kStatsChunk;
-    const int ct1 = ct0 + kStatsChunk < ctn ? ct0 + kStatsChunk : ctn;
+    const int ct0 = ch * chunk;
+    const int ct1 = ct0 + chunk < ctn ? ct0 + chunk : ctn;
     unsigned long long rw[4] = {0ull, 0ull, 0ull, 0ull};  // row bitmap bits of this chunk, per owned row
     uint4 u[4];
     uint32_t m[4];
@@ -815,15 +816,28 @@ unsigned tile_grid(int64_t R, int C) {
   return (unsigned)(tiles < cap ? tiles : cap);
 }
 
+// Column tiles per stats work item: whole chunks while the row blocks alone
+// give the GPU enough items, single tiles for short tensors.
+int stats_chunk(int64_t R, int C) {
+  const int64_t nrb = (R + 127) / 128;
+  return (C > 64 && nrb < device_sm_count()) ? 1 : kStatsChunk;
+}
+
 }  // namespace
+
+bool stats_writes_rows_whole(int64_t R, int C) {
+  const int ctn = (C + 63) / 64;
+  return ctn <= stats_chunk(R, C);
+}
 
 cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev& o, cudaStream_t s) {
   if (R <= 0 || C <= 0) return cudaSuccess;
-  const int64_t items = ((R + 127) / 128) * ((((C + 63) / 64) + kStatsChunk - 1) / kStatsChunk);
+  const int chunk = stats_chunk(R, C);
+  const int64_t items = ((R + 127) / 128) * ((((C + 63) / 64) + chunk - 1) / chunk);
   const int64_t cap = 4LL * device_sm_count();  // 4 CTAs per SM
   const unsigned grid = (unsigned)(items < cap ? items : cap);
   const size_t smem = C <= kMaxAccCols ? sizeof(uint32_t) * (size_t)C : 0;
-  return launch_kernel(stats_kernel, dim3(grid), dim3(kTileThreads), smem, s, x, R, C, o);
+  return launch_kernel(stats_kernel, dim3(grid), dim3(kTileThreads), smem, s, x, R, C, o, chunk);
 }
 
 cudaError_t launch_clear(const ClearArgs& a, cudaStream_t s) {

@@ -122,8 +122,8 @@ extern "C" sparoa_status sparoa_gemm_noalloc(void* stream, const void* x, int64_
     // unless K is wide
     ClearArgs z = {};
     z.p[0] = reinterpret_cast<uint32_t*>(b);
-    const char* end = K <= kStatsWholeRowCols ? reinterpret_cast<char*>(xo.row_bm)
-                                              : reinterpret_cast<char*>(xo.blk_mask);
+    const char* end = stats_writes_rows_whole(M, (int)K) ? reinterpret_cast<char*>(xo.row_bm)
+                                                         : reinterpret_cast<char*>(xo.blk_mask);
     z.words[0] = (int64_t)((end - b) / 4);
     if (launch_clear(z, s) != cudaSuccess) return SPAROA_ERR_CUDA;
   }

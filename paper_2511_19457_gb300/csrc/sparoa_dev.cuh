@@ -437,38 +437,5 @@ __device__ __forceinline__ float epi_act(float v, int act) {
   return v;
 }
 
-// ---------------------------------------------------------------------------
-// Occupancy flush of one 128-row x 64-column tile
-// ---------------------------------------------------------------------------
-// nzrow[r] bit c: element (row0 + r, col0 + c) is non-zero (zero outside the
-// tensor).  Called by `nthreads` threads (a multiple of 32, >= 64) with local
-// index `tid`; row0 must be a multiple of 128 and col0 a multiple of 64.
-__device__ __forceinline__ void flush_tile(const uint64_t* nzrow, int64_t row0, int col0,
-                                           const OccDev& o, int tid, int nthreads) {
-  const int t = col0 >> 6;
-  for (int r = tid; r < 128; r += nthreads) {
-    if (nzrow[r] != 0ull && row0 + r < o.R)
-      atomicOr(&o.row_bm[(row0 + r) * o.W64 + (t >> 6)], 1ull << (t & 63));
-  }
-  if (tid < 64) {
-    uint32_t cnt = 0;
-#pragma unroll 8
-    for (int r = 0; r < 128; ++r) cnt += (uint32_t)((nzrow[r] >> tid) & 1ull);
-    const int c = col0 + tid;
-    if (cnt && c < o.C) atomicAdd(&o.col_nnz[c], cnt);
-    const uint32_t word = __ballot_sync(0xffffffffu, cnt != 0);
-    uint32_t sum = cnt;
-#pragma unroll
-    for (int s = 16; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
-    if ((tid & 31) == 0) {
-      const int w = (col0 >> 5) + (tid >> 5);
-      if (word && w < o.C32) atomicOr(&o.blk_mask[(row0 >> 7) * o.C32 + w], word);
-      if (sum) {
-        atomicAdd(&o.tile_nnz[t], sum);
-        atomicAdd(o.nnz, (unsigned long long)sum);
-      }
-    }
-  }
-}
 
 }  // namespace sparoa

@@ -119,10 +119,11 @@ cudaError_t launch_fcskip(const FcSkipArgs& a, cudaStream_t s);
 // Memory-bound kernels (128-row x 64-channel tiles, occupancy fused)
 // ----------------------------------------------------------------------------
 // Eq. 1 statistics and bitmaps of x viewed as [R, C].  The block masks are
-// written whole, and so are the row bitmaps when C <= kStatsWholeRowCols;
-// the counters (nnz, col_nnz, tile_nnz), and the row bitmaps of wider
-// tensors, are accumulated and must be zero on entry.
+// written whole, and so are the row bitmaps when stats_writes_rows_whole(R, C);
+// the counters (nnz, col_nnz, tile_nnz), and otherwise the row bitmaps, are
+// accumulated and must be zero on entry.
 constexpr int kStatsWholeRowCols = 512;
+bool stats_writes_rows_whole(int64_t R, int C);
 cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev& o, cudaStream_t s);
 
 // Copy [P, C] to [P, Cp] with zero channels C..Cp-1.
