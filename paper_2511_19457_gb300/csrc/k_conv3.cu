@@ -159,13 +159,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp < 4) {
     // -------------------------------------------------------------- producers
     const int t_ = threadIdx.x;
-    if (t_ == 0) {
-      // weights once: box {64 channels, 1 tap, CO rows} per (tap, channel block)
-      mbar_arrive_expect_tx(bar_w, (uint32_t)G.w_bytes);
-      for (int tap = 0; tap < 9; ++tap)
-        for (int cb = 0; cb < C / 64; ++cb)
-          tma_load_3d(sW + (uint32_t)((tap * (C / 64) + cb) * CO * 128), &tmW, bar_w, cb * 64, tap, 0);
-    }
     int j = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++j) {
       if (!skip && warp != 0) break;  // dense path: warp 0 walks the tiles, lane 0 streams the slabs
@@ -184,6 +177,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int cb = 0; cb < C / 64; ++cb)
             tma_load_4d(dst + (uint32_t)(cb * G.chunk_stride), &tmX, bar_full + 8 * b, cb * 64, -1,
                         oh0 - 1, img);
+        }
+        if (j == 0) {
+          // weights once, after the first slab (the slab comes from HBM and gates
+          // the first MMAs; the weights are L2 hits for all but the first CTAs):
+          // box {64 channels, 1 tap, CO rows} per (tap, channel block)
+          mbar_arrive_expect_tx(bar_w, (uint32_t)G.w_bytes);
+          for (int tap = 0; tap < 9; ++tap)
+            for (int cb = 0; cb < C / 64; ++cb)
+              tma_load_3d(sW + (uint32_t)((tap * (C / 64) + cb) * CO * 128), &tmW, bar_w, cb * 64, tap, 0);
         }
       }
       if (skip) {
