@@ -12,7 +12,8 @@ pad 1, input ReLU(N(0,1)) (about half zeros), BN + ReLU epilogue:
 Metric: effective TFLOP/s = dense-equivalent FLOPs / time.
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl sparoa|reference]
-       [--workload conv|fc|resnet18|mobilenet_v2] [--batch B]
+       [--workload conv|fc|resnet18|mobilenet_v2|mlp_sweep|ops|calibrate] [--batch B]
+       [--thresholds default|calibrated] [--calib-out PATH]
 For N > 1 launch one process per GPU with torch.distributed.run; every rank
 runs its own replica (weak scaling), timing is the max over ranks.
 """
@@ -45,8 +46,12 @@ def parse_args():
     p.add_argument("--warmup", type=int, default=400)
     p.add_argument("--impl", default="sparoa", choices=["sparoa", "reference"])
     p.add_argument("--workload", default="conv",
-                   choices=["conv", "fc", "resnet18", "mobilenet_v2", "mlp_sweep", "ops"])
+                   choices=["conv", "fc", "resnet18", "mobilenet_v2", "mlp_sweep", "ops", "calibrate"])
     p.add_argument("--batch", type=int, default=32)
+    p.add_argument("--thresholds", default="default", choices=["default", "calibrated"],
+                   help="graph workloads: the default s_thr/c_thr, or the per-operator thresholds "
+                        "of the committed calibration table")
+    p.add_argument("--calib-out", default=None, help="calibrate: write the thresholds table here")
     p.add_argument("--no-cpu-baseline", action="store_true")
     return p.parse_args()
 
@@ -549,21 +554,24 @@ def run_mlp_sweep(args, rank, local_rank, world, peaks):
             "crossover_rho": cross, "table": table}
 
 
-def run_graph_workload(args, rank, local_rank, world, peaks, name):
-    """CNN images/s through sparoa_run_graph (not the default bench line)."""
+def time_graph_workload(ctx, name, batch, steps, warmup, thresholds="default"):
+    """ms per replay of one CUDA-graph-captured sparoa_run_graph over the
+    synthetic CNN, the L2 flushed before every replay; returns (ms, records)."""
     import torch
 
+    from paper_2511_19457_gb300 import calibrate as cal
     from paper_2511_19457_gb300 import sparoa as sp
     from paper_2511_19457_gb300 import synth
-    dev = torch.device("cuda", local_rank)
-    torch.cuda.set_device(dev)
-    ctx = sp.Context(local_rank)
-    ops, xb, shape = (synth.resnet18 if name == "resnet18" else synth.mobilenet_v2)(batch=args.batch)
+    dev = torch.device("cuda", ctx.device)
+    ops, xb, shape = (synth.resnet18 if name == "resnet18" else synth.mobilenet_v2)(batch=batch)
+    if thresholds == "calibrated":
+        ops = cal.apply(ops, shape, cal.load_table())
+    elif isinstance(thresholds, dict):
+        ops = cal.apply(ops, shape, thresholds)
     graph = sp.Graph(ops)
     x = sp.bits_to_device(xb).view(*shape)
     recs = sp.sparoa_run_graph(ctx, graph, x, records=True)
-    flops = sum(r.stats.flops for r in recs)
-    for _ in range(max(args.warmup, 3)):
+    for _ in range(max(warmup, 3)):
         sp.sparoa_run_graph(ctx, graph, x)
     torch.cuda.synchronize()
     g = torch.cuda.CUDAGraph()
@@ -574,7 +582,7 @@ def run_graph_workload(args, rank, local_rank, world, peaks, name):
     # outside the events that time the replay
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for _ in range(args.steps)]
+           for _ in range(steps)]
     torch.cuda.synchronize()
     for e0, e1 in evs:
         flush.zero_()
@@ -582,10 +590,26 @@ def run_graph_workload(args, rank, local_rank, world, peaks, name):
         g.replay()
         e1.record()
     torch.cuda.synchronize()
-    ms = sum(e0.elapsed_time(e1) for e0, e1 in evs) / args.steps
+    ms = sum(e0.elapsed_time(e1) for e0, e1 in evs) / steps
+    del g, flush
+    return ms, recs
+
+
+PATH_NAME = {0: "none", 1: "dense", 2: "zero-skip", 3: "depthwise"}
+
+
+def run_graph_workload(args, rank, local_rank, world, peaks, name):
+    """CNN images/s through sparoa_run_graph (not the default bench line)."""
+    import torch
+
+    from paper_2511_19457_gb300 import sparoa as sp
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    ctx = sp.Context(local_rank)
+    ms, recs = time_graph_workload(ctx, name, args.batch, args.steps, args.warmup, args.thresholds)
+    flops = sum(r.stats.flops for r in recs)
     ms = max_over_ranks(ms, world, dev)
-    path_name = {0: "none", 1: "dense", 2: "zero-skip", 3: "depthwise"}
-    ops_table = [{"op": i, "path": path_name.get(int(r.stats.path), str(int(r.stats.path))),
+    ops_table = [{"op": i, "path": PATH_NAME.get(int(r.stats.path), str(int(r.stats.path))),
                   "rho": round(float(r.stats.sparsity), 4), "gflop": round(r.stats.flops / 1e9, 4),
                   "flop_per_byte": round(float(r.stats.flops_per_byte), 1)}
                  for i, r in enumerate(recs)]
@@ -594,6 +618,7 @@ def run_graph_workload(args, rank, local_rank, world, peaks, name):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic", "effective_tflops": flops / (ms * 1e-3) / 1e12,
             "config": {"workload": f"{name} B={args.batch} through sparoa_run_graph (CUDA graph)",
+                       "thresholds": args.thresholds,
                        "global_batch": args.batch * world,
                        "l2": "flushed by a 256 MB write before every timed replay"},
             "ops": ops_table}
@@ -731,6 +756,44 @@ def run_ops(args, rank, local_rank, world, peaks):
             "ops": rows}
 
 
+def run_calibrate(args, rank, local_rank, world, peaks):
+    """Per-operator threshold calibration (Sec. 3.3's ground-truth grid, on
+    this GPU): forced dense vs forced zero-skip over rho x size x structure,
+    the crossover table, then ResNet-18 (B=8) and MobileNetV2 (B=32) images/s
+    under the default thresholds and under the fresh calibrated ones."""
+    import torch
+
+    from paper_2511_19457_gb300 import calibrate as cal
+    from paper_2511_19457_gb300 import sparoa as sp
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    ctx = sp.Context(local_rank)
+    t0 = time.time()
+    table = cal.calibrate(ctx, log=lambda e: print(json.dumps(
+        {"kind": e["kind"], "shape": e["shape"], "structure": e["structure"], "s_thr": e["s_thr"],
+         "dense_us": e["dense_us"], "skip_us": e["skip_us"]}), file=sys.stderr, flush=True))
+    cal_s = time.time() - t0
+    if args.calib_out:
+        with open(args.calib_out, "w") as f:
+            json.dump(table, f, indent=1)
+    graphs = {}
+    for name, batch in (("resnet18", 8), ("mobilenet_v2", 32)):
+        res = {}
+        for tag, thr in (("default", "default"), ("calibrated", table)):
+            ms, recs = time_graph_workload(ctx, name, batch, 50, 5, thr)
+            res[tag] = {"images_per_s": round(batch / (ms * 1e-3), 1), "ms": round(ms, 4),
+                        "paths": "".join({0: "-", 1: "D", 2: "S", 3: "w"}.get(int(r.stats.path), "?")
+                                         for r in recs)}
+        graphs[f"{name}_b{batch}"] = res
+    ctx.close()
+    return {"metric": METRIC, "value": None, "unit": "crossover rho per operator", "n_gpus": world,
+            "higher_is_better": False, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "threshold calibration: forced dense vs zero-skip per operator "
+                                   "kind and size over rho x {unstructured, block}",
+                       "seconds": round(cal_s, 1)},
+            "crossover": cal.summary(table), "graphs": graphs}
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -754,6 +817,8 @@ def main():
         line = run_mlp_sweep(args, rank, local_rank, world, peaks)
     elif args.workload == "ops":
         line = run_ops(args, rank, local_rank, world, peaks)
+    elif args.workload == "calibrate":
+        line = run_calibrate(args, rank, local_rank, world, peaks)
     else:
         raise SystemExit(f"workload {args.workload} is not wired into bench.py")
     if rank == 0:

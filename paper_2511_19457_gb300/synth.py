@@ -18,6 +18,9 @@ weights, which are not available; same shapes, 224x224 RGB, batch 1/8/32):
   mlp_hidden      the hidden activation of a 768 -> 3072 -> 768 ReLU MLP drawn
                   directly at a target zero fraction, unstructured or in
                   32-channel blocks per 128-token tile
+  structured_activation  a [M, K] or NHWC activation at a target zero
+                  fraction, unstructured or in blocks (threshold calibration;
+                  drawn on the device the caller names)
 """
 from __future__ import annotations
 
@@ -233,3 +236,34 @@ def mlp_hidden(M: int, rho: float, structure: str = "unstructured", seed: int = 
     else:
         raise ValueError(structure)
     return to_bf16_bits(h * keep.to(torch.float32))
+
+
+# --------------------------------------------------------------------------
+# threshold calibration inputs
+# --------------------------------------------------------------------------
+STRUCTURES = ("unstructured", "block")
+
+
+def structured_activation(shape, rho: float, structure: str, gen: torch.Generator,
+                          device="cpu") -> torch.Tensor:
+    """A bf16 activation of ``shape`` with |N(0,1)| + 1e-3 values and a target
+    zero fraction ``rho``, drawn with ``gen`` on ``device``:
+      unstructured  iid Bernoulli(rho) zeros (a ReLU output)
+      block         units zeroed together: 128 rows x 32 channels of a 2-D
+                    [M, K] input; 8 image rows x 64 channels of one image of
+                    an NHWC [B, H, W, C] input (spatially clustered zeros)"""
+    v = torch.randn(*shape, device=device, generator=gen).abs_() + 1e-3
+    if structure == "unstructured":
+        keep = torch.rand(*shape, device=device, generator=gen) >= rho
+    elif structure == "block" and len(shape) == 2:
+        M, K = shape
+        kb = torch.rand((M + 127) // 128, (K + 31) // 32, device=device, generator=gen) >= rho
+        keep = kb.repeat_interleave(128, dim=0)[:M].repeat_interleave(32, dim=1)[:, :K]
+    elif structure == "block" and len(shape) == 4:
+        B, H, W, C = shape
+        kb = torch.rand(B, (H + 7) // 8, 1, (C + 63) // 64, device=device, generator=gen) >= rho
+        keep = kb.repeat_interleave(8, dim=1)[:, :H].repeat_interleave(64, dim=3)[..., :C]
+        keep = keep.expand(B, H, W, C)
+    else:
+        raise ValueError(f"structure {structure!r} for shape {tuple(shape)}")
+    return (v * keep.to(v.dtype)).to(torch.bfloat16)

@@ -12,6 +12,7 @@ import pytest
 import torch
 
 from oracle import oracle as orc
+from paper_2511_19457_gb300 import calibrate as cal
 from paper_2511_19457_gb300 import synth
 from tests._parity import assert_close, assert_occ_equal
 
@@ -24,8 +25,10 @@ def sp():
     return sparoa
 
 
-def _run(sp, name, batch, thr=None):
+def _run(sp, name, batch, thr=None, table=None):
     ops, xb, shape = getattr(synth, name)(batch=batch, seed=0, thr=thr)
+    if table is not None:
+        ops = cal.apply(ops, shape, table)
     ctx = sp.Context(0)
     graph = sp.Graph(ops)
     x = sp.bits_to_device(xb).view(*shape)
@@ -97,3 +100,29 @@ def test_graph_chained_end_to_end(sp, name):
     got = synth.bits_to_f32(outs[-1][0]).astype(np.float64)
     # per-op parity is the bar; the chained drift of bf16 storage is bounded loosely
     assert_close(got, ref[-1].out_f64, max_rel=8e-2, fro_rel=3e-2, what=f"{name} chained logits")
+
+
+def _mixed_table():
+    """Per-kind thresholds spread over always / mid / never zero-skip."""
+    kinds = {"conv3x3s1": 0.45, "conv3x3s2": cal.NEVER, "conv1x1s2": 0.0, "conv1x1s1": 0.55,
+             "fc_small": 0.0, "gemm": cal.NEVER}
+    return {"entries": [{"kind": k, "structure": "unstructured", "flops": 1e9, "s_thr": v}
+                        for k, v in kinds.items()]}
+
+
+@pytest.mark.parametrize("source", ["mixed", "committed"])
+@pytest.mark.parametrize("name", ["resnet18", "mobilenet_v2"])
+def test_graph_teacher_forced_calibrated(sp, name, source):
+    """Per-operator calibrated thresholds: every op's dispatch under its own
+    thresholds matches the oracle's, outputs within tolerance."""
+    if source == "committed":
+        if not __import__("os").path.exists(cal.TABLE_PATH):
+            pytest.skip("no calibration table")
+        table = cal.load_table()
+    else:
+        table = _mixed_table()
+    ops, xb, shape, recs, outs, occs = _run(sp, name, batch=1, table=table)
+    _teacher_check(sp, ops, xb, shape, recs, outs, occs)
+    if source == "mixed":
+        paths = {int(r.stats.path) for r in recs}
+        assert sp.PATH_SKIP in paths and sp.PATH_DENSE in paths
