@@ -46,7 +46,8 @@ namespace sparoa {
 
 namespace {
 
-constexpr int kEpiWarps = 8;                   // two per TMEM lane quarter, 32 of each 64 columns
+constexpr int kEpiWarps = 8;
+constexpr int kMaxSplit = 4;  // K split: at most this many units per output tile                   // two per TMEM lane quarter, 32 of each 64 columns
 constexpr int kEpiThreads = 32 * kEpiWarps;
 constexpr int kMmaWarp = 4 + kEpiWarps;
 constexpr int kThreads = 32 * (kMmaWarp + 1);  // 4 producer warps, epilogue warps, MMA warp
@@ -157,6 +158,39 @@ __device__ __forceinline__ int64_t tile_row(const Geo& p, const TileGeo& g, int 
   return m;
 }
 
+// Everything a producer thread needs to know about work unit u (tile u / ks,
+// K range u % ks): pure arithmetic on the parameters, 32-bit throughout.
+struct UnitGeo {
+  int t, ks, kb0, kb1;
+  TileGeo g;
+  bool rvalid;
+  int img, oh, ow;
+  int cb, rr, ss;  // conv = 2: channel block and tap (row, column) of block kb0
+  int iy0, ix0;    // conv = 2: input origin of the tile
+};
+
+__device__ __forceinline__ UnitGeo unit_geo(const Geo& p, int u, int KS, int kblocks, int nt, int BN,
+                                            int BK, int r) {
+  UnitGeo q;
+  q.t = u / KS;
+  q.ks = u - q.t * KS;
+  q.kb0 = q.ks * kblocks / KS;
+  q.kb1 = (q.ks + 1) * kblocks / KS;
+  q.g = tile_geo(p, q.t, nt, BN);
+  tile_row(p, q.g, r, q.rvalid, q.img, q.oh, q.ow);
+  q.cb = q.rr = q.ss = 0;
+  if (p.conv == 2) {
+    const int cb_per_tap = p.Cp / BK;
+    const int tap = q.kb0 / cb_per_tap;
+    q.cb = q.kb0 - tap * cb_per_tap;
+    q.rr = tap / p.kw;
+    q.ss = tap - q.rr * p.kw;
+  }
+  q.iy0 = q.g.th0 * p.stride - p.pad;
+  q.ix0 = q.g.tw0 * p.stride - p.pad;
+  return q;
+}
+
 template <int BN, int BK>
 __global__ void __launch_bounds__(kThreads, 1)
     igemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -239,6 +273,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = threadIdx.x - 128; i < kBM; i += kEpiThreads) s_rowbm[i] = 0ull;
     for (int i = threadIdx.x - 128; i < BN / 32; i += kEpiThreads) s_blk[i] = 0u;
   }
+  // The producers' first work unit is laid out before the grid dependency
+  // wait: no memory is read, and under programmatic dependent launch this
+  // overlaps the tail of the kernel before.
+  UnitGeo ug{};
+  if (warp < 4 && (int)blockIdx.x < units) ug = unit_geo(p, blockIdx.x, KS, kblocks, nt, BN, BK, threadIdx.x);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -261,13 +300,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     int pending = 0;   // mode 1: filled stages whose A arrivals are still owed
     bool ok = true;
     for (int u = blockIdx.x; u < units; u += gridDim.x) {
-      const int t = u / KS, ks = u - (u / KS) * KS;
-      const int kb0 = (int)((int64_t)ks * kblocks / KS);
-      const int kb1 = (int)((int64_t)(ks + 1) * kblocks / KS);
-      const TileGeo g = tile_geo(p, t, nt, BN);
-      bool rvalid;
-      int img, oh, ow;
-      tile_row(p, g, r, rvalid, img, oh, ow);
+      if (u != (int)blockIdx.x) ug = unit_geo(p, u, KS, kblocks, nt, BN, BK, r);
+      const int kb0 = ug.kb0, kb1 = ug.kb1;
+      const TileGeo g = ug.g;
+      const bool rvalid = ug.rvalid;
+      const int img = ug.img, oh = ug.oh, ow = ug.ow;
       int last = kb1 - 1;
       if (skip) {
         // ---- occupied K blocks of this tile
@@ -351,14 +388,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           // slots are free by construction) waits for nothing.
           int slot = it % S;
           uint32_t ph = (uint32_t)((it / S) & 1);
-          int cb = 0, rr = 0, ss = 0;  // conv = 2: channel block and tap of block kb
-          if (p.conv == 2) {
-            const int tap = kb0 / cb_per_tap;
-            cb = kb0 - tap * cb_per_tap;
-            rr = tap / p.kw;
-            ss = tap - rr * p.kw;
-          }
-          const int iy0 = g.th0 * p.stride - p.pad, ix0 = g.tw0 * p.stride - p.pad;
+          int cb = ug.cb, rr = ug.rr, ss = ug.ss;  // conv = 2: channel block and tap of block kb
+          const int iy0 = ug.iy0, ix0 = ug.ix0;
           const uint32_t fb0 = bar_full, eb0 = bar_empty;
           for (int kb = kb0; kb <= last; ++kb) {
             const bool issue =
@@ -558,17 +589,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             __stcg(dst + i, make_float4(__uint_as_float(raw[4 * i]), __uint_as_float(raw[4 * i + 1]),
                                         __uint_as_float(raw[4 * i + 2]), __uint_as_float(raw[4 * i + 3])));
         }
-        __threadfence();
+        // One thread publishes the partial and takes the ticket: the barrier
+        // orders every epilogue thread's stores before that thread's fence
+        // (fences are cumulative), and the last arriver's fence after the
+        // ticket orders the other units' partials before the reads below,
+        // which the second barrier hands on to every thread.
         named_bar_sync(2, kEpiThreads);
-        if (et == 0) s_last[b] = atomicAdd(&P.ws_cnt[t], 1u) == (unsigned)(KS - 1) ? 1 : 0;
+        if (et == 0) {
+          __threadfence();
+          const int lst = atomicAdd(&P.ws_cnt[t], 1u) == (unsigned)(KS - 1) ? 1 : 0;
+          if (lst) {
+            __threadfence();
+            P.ws_cnt[t] = 0u;  // every unit of the tile has arrived: ready for reuse
+          }
+          s_last[b] = lst;
+        }
         named_bar_sync(2, kEpiThreads);
         if (!s_last[b]) {
           tc_fence_before();
           mbar_arrive(bar_acce + 8 * b);  // this unit's share is in the partial
           continue;
         }
-        __threadfence();
-        if (et == 0) P.ws_cnt[t] = 0u;  // every unit of the tile has arrived: ready for reuse
       }
       const OccDev o = P.out_occ;  // registers, not parameter-space loads
       const int blk = mvalid ? (int)(m >> 7) : -1;
@@ -592,18 +633,35 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld32_nowait(tbase + (uint32_t)(gcol * 64 + hf * 32), raw);
         tmem_wait_ld32(raw);
         if (KS > 1) {
-          // the other units' partials of this row's 32 columns
-          for (int k2 = 0; k2 < KS; ++k2) {
-            if (k2 == ks) continue;
-            const float4* src =
-                reinterpret_cast<const float4*>(ws_tile + ((int64_t)k2 * kBM + r) * BN + gcol * 64 + hf * 32);
+          // the other units' partials of this row's 32 columns, in two halves:
+          // every load of a half in flight before the first is used, added in
+          // unit order
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              const float4 v = __ldcg(src + i);
-              raw[4 * i] = __float_as_uint(__uint_as_float(raw[4 * i]) + v.x);
-              raw[4 * i + 1] = __float_as_uint(__uint_as_float(raw[4 * i + 1]) + v.y);
-              raw[4 * i + 2] = __float_as_uint(__uint_as_float(raw[4 * i + 2]) + v.z);
-              raw[4 * i + 3] = __float_as_uint(__uint_as_float(raw[4 * i + 3]) + v.w);
+          for (int h = 0; h < 2; ++h) {
+            float4 pv[kMaxSplit - 1][4];
+#pragma unroll
+            for (int k2i = 0; k2i < kMaxSplit - 1; ++k2i) {
+              const int k2 = k2i < ks ? k2i : k2i + 1;
+              if (k2 < KS) {
+                const float4* src = reinterpret_cast<const float4*>(
+                    ws_tile + ((int64_t)k2 * kBM + r) * BN + gcol * 64 + hf * 32 + h * 16);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) pv[k2i][i] = __ldcg(src + i);
+              }
+            }
+#pragma unroll
+            for (int k2i = 0; k2i < kMaxSplit - 1; ++k2i) {
+              const int k2 = k2i < ks ? k2i : k2i + 1;
+              if (k2 < KS) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                  uint32_t* q4 = raw + h * 16 + 4 * i;
+                  q4[0] = __float_as_uint(__uint_as_float(q4[0]) + pv[k2i][i].x);
+                  q4[1] = __float_as_uint(__uint_as_float(q4[1]) + pv[k2i][i].y);
+                  q4[2] = __float_as_uint(__uint_as_float(q4[2]) + pv[k2i][i].z);
+                  q4[3] = __float_as_uint(__uint_as_float(q4[3]) + pv[k2i][i].w);
+                }
+              }
             }
           }
         }
@@ -931,7 +989,7 @@ void choose_tiles(const IgemmArgs& a, int64_t mtiles, int* bn_out, int* ks_out) 
   int ks = 1;
   if (a.ws && a.ws_cnt && tiles < sms && tiles <= a.ws_cnt_len) {
     ks = (int)(sms / tiles);
-    if (ks > 4) ks = 4;
+    if (ks > kMaxSplit) ks = kMaxSplit;
     while (ks > 1 && (kblocks < 8 * ks || (size_t)tiles * ks * kBM * bn * 4 > a.ws_bytes)) --ks;
   }
   *bn_out = bn;
