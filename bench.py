@@ -12,7 +12,7 @@ pad 1, input ReLU(N(0,1)) (about half zeros), BN + ReLU epilogue:
 Metric: effective TFLOP/s = dense-equivalent FLOPs / time.
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl sparoa|reference]
-       [--workload conv|fc|resnet18|mobilenet_v2|mlp_sweep|ops|calibrate] [--batch B]
+       [--workload conv|fc|resnet18|mobilenet_v2|mlp_sweep|ops|calibrate|batching] [--batch B]
        [--thresholds default|calibrated] [--calib-out PATH]
 For N > 1 launch one process per GPU with torch.distributed.run; every rank
 runs its own replica (weak scaling), timing is the max over ranks.
@@ -46,7 +46,8 @@ def parse_args():
     p.add_argument("--warmup", type=int, default=400)
     p.add_argument("--impl", default="sparoa", choices=["sparoa", "reference"])
     p.add_argument("--workload", default="conv",
-                   choices=["conv", "fc", "resnet18", "mobilenet_v2", "mlp_sweep", "ops", "calibrate"])
+                   choices=["conv", "fc", "resnet18", "mobilenet_v2", "mlp_sweep", "ops", "calibrate",
+                            "batching"])
     p.add_argument("--batch", type=int, default=32)
     p.add_argument("--thresholds", default="default", choices=["default", "calibrated"],
                    help="graph workloads: the default s_thr/c_thr, or the per-operator thresholds "
@@ -794,6 +795,74 @@ def run_calibrate(args, rank, local_rank, world, peaks):
             "crossover": cal.summary(table), "graphs": graphs}
 
 
+def run_batching(args, rank, local_rank, world, peaks):
+    """Dynamic batching (Algorithm 2) on the synthetic CNNs: every evaluated
+    batch size is one CUDA-graph-captured sparoa_run_graph timed after an L2
+    flush; M(B) is the graph walk's workspace plus the input."""
+    import numpy as np
+    import torch
+
+    from paper_2511_19457_gb300 import batching as bt
+    from paper_2511_19457_gb300 import sparoa as sp
+    from paper_2511_19457_gb300 import synth
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    ctx = sp.Context(local_rank)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    out = {}
+    for name in ("resnet18", "mobilenet_v2"):
+        ops, _, _ = getattr(synth, name)(batch=1)
+        graph = sp.Graph(ops)
+        gen = torch.Generator(device=dev).manual_seed(0)
+        cache = {}
+
+        def latency(B):
+            if B in cache:
+                return cache[B]
+            x = torch.randn(B, 224, 224, 3, device=dev, generator=gen).to(torch.bfloat16)
+            for _ in range(3):
+                sp.sparoa_run_graph(ctx, graph, x)
+            torch.cuda.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                sp.sparoa_run_graph(ctx, graph, x)
+            g.replay()
+            ts = []
+            for _ in range(20):
+                flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                g.replay()
+                e1.record()
+                torch.cuda.synchronize()
+                ts.append(e0.elapsed_time(e1) * 1e-3)
+            del g, x
+            cache[B] = float(np.median(ts))
+            return cache[B]
+
+        def memory(B):
+            return sp.sparoa_graph_workspace(ctx, graph, (B, 224, 224, 3)) + B * 224 * 224 * 3 * 2
+
+        # the input's operator-level characteristics, FLOP-weighted over conv / FC
+        recs = sp.sparoa_run_graph(ctx, graph, torch.randn(8, 224, 224, 3, device=dev, generator=gen)
+                                   .to(torch.bfloat16), records=True)
+        fl = np.array([r.stats.flops for r in recs], dtype=np.float64)
+        rho = float((fl * np.array([r.stats.sparsity for r in recs])).sum() / fl.sum())
+        fpb = float((fl * np.array([r.stats.flops_per_byte for r in recs])).sum() / fl.sum())
+        tr = bt.dynamic_batch(latency, memory, 1, sparsity=rho, intensity=fpb, s_thr=0.5, c_thr=None,
+                              mem_max=32 * 2 ** 30, t_realtime=2e-3, b_max=256)
+        out[name] = {"input_sparsity": round(rho, 4), "input_flops_per_byte": round(fpb, 1),
+                     **tr.as_dict()}
+    ctx.close()
+    return {"metric": METRIC, "value": None, "unit": "batch size", "n_gpus": world,
+            "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "Algorithm 2 dynamic batching over sparoa_run_graph",
+                       "constraints": {"mem_max_gib": 32, "t_realtime_ms": 2.0, "s_thr": 0.5,
+                                       "c_thr": None, "B0": 1, "b_max": 256},
+                       "l2": "flushed by a 256 MB write before every timed replay"},
+            "graphs": out}
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -819,6 +888,8 @@ def main():
         line = run_ops(args, rank, local_rank, world, peaks)
     elif args.workload == "calibrate":
         line = run_calibrate(args, rank, local_rank, world, peaks)
+    elif args.workload == "batching":
+        line = run_batching(args, rank, local_rank, world, peaks)
     else:
         raise SystemExit(f"workload {args.workload} is not wired into bench.py")
     if rank == 0:

@@ -316,6 +316,18 @@ sparoa_status sparoa_run_graph(sparoa_ctx *ctx, const sparoa_op *ops, int32_t n_
                                const void *x, int64_t N, int64_t H, int64_t W, int64_t C, void *y,
                                uint64_t y_bytes, sparoa_record *records);
 
+/*
+ * Device workspace sparoa_run_graph needs for this operator list and input
+ * shape, in bytes: occupancy blocks of every value, recorded paths, every
+ * intermediate activation (bf16) and channel-padded copies.  Checks the list
+ * exactly as sparoa_run_graph does; no device work.  This is the memory model
+ * M(B) of the dynamic batching loop (Sec. 5.2, Algorithm 2).
+ *   bytes  host output
+ * Errors: INVALID_ARG, UNSUPPORTED (as sparoa_run_graph).
+ */
+sparoa_status sparoa_graph_workspace(sparoa_ctx *ctx, const sparoa_op *ops, int32_t n_ops,
+                                     int64_t N, int64_t H, int64_t W, int64_t C, uint64_t *bytes);
+
 /* ------------------------------------------------------------------------ */
 /* Variant for callers that cannot allocate device memory                     */
 /* ------------------------------------------------------------------------ */

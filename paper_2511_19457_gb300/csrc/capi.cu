@@ -834,27 +834,34 @@ sparoa_status sparoa_bn_act(sparoa_ctx* ctx, const void* x, int64_t R, int64_t C
 // ---------------------------------------------------------------------------
 // graph walk
 // ---------------------------------------------------------------------------
-sparoa_status sparoa_run_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_ops,
-                               const void* x, int64_t N, int64_t H, int64_t W, int64_t C, void* y,
-                               uint64_t y_bytes, sparoa_record* records) {
-  if (!ctx) return SPAROA_ERR_INVALID_ARG;
-  if (!ops || n_ops <= 0) return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: no operators");
-  if (N <= 0 || H <= 0 || W <= 0 || C <= 0 || !x)
-    return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: bad input");
-  if (C % 8 == 0 && !aligned16(x)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: misaligned input");
+namespace {
+
+// The graph walk's plan: every value's shape (checked against its operator),
+// and the layout of the context arena that holds the occupancy blocks, the
+// recorded paths, the activations and the channel-padded copies.
+struct Val {
+  int64_t n, h, w, c;
+  size_t act_off = 0, occ_off = 0;
+};
+struct Aux {
+  size_t padx = 0, padw = 0, fcocc = 0;
+  int64_t cp = 0;
+  bool fc_view = false;
+};
+struct GraphPlan {
+  std::vector<Val> vals;
+  std::vector<Aux> aux;
+  size_t nnz_off = 0, occ_end = 0, path_off = 0, total = 0;
+};
+
+sparoa_status plan_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_ops, int64_t N, int64_t H,
+                         int64_t W, int64_t C, GraphPlan& pl) {
   // ---- plan: shapes, checks and arena layout
-  struct Val {
-    int64_t n, h, w, c;
-    size_t act_off = 0, occ_off = 0;
-  };
-  std::vector<Val> vals((size_t)n_ops + 1);
+  std::vector<Val>& vals = pl.vals;
+  vals.assign((size_t)n_ops + 1, Val{});
   vals[0] = {N, H, W, C};
-  struct Aux {
-    size_t padx = 0, padw = 0, fcocc = 0;
-    int64_t cp = 0;
-    bool fc_view = false;
-  };
-  std::vector<Aux> aux((size_t)n_ops);
+  std::vector<Aux>& aux = pl.aux;
+  aux.assign((size_t)n_ops, Aux{});
   for (int i = 0; i < n_ops; ++i) {
     const sparoa_op& op = ops[i];
     if (op.input < 0 || op.input > i)
@@ -945,6 +952,42 @@ sparoa_status sparoa_run_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_
       off += align_up((size_t)(ops[i].c_out * ops[i].kh * ops[i].kw * aux[(size_t)i].cp) * 2);
     }
   }
+  pl.nnz_off = nnz_off;
+  pl.occ_end = occ_end;
+  pl.path_off = path_off;
+  pl.total = off;
+  return SPAROA_OK;
+}
+
+}  // namespace
+
+sparoa_status sparoa_graph_workspace(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_ops, int64_t N,
+                                     int64_t H, int64_t W, int64_t C, uint64_t* bytes) {
+  if (!ctx) return SPAROA_ERR_INVALID_ARG;
+  if (!bytes) return fail(ctx, SPAROA_ERR_INVALID_ARG, "graph_workspace: NULL bytes");
+  if (!ops || n_ops <= 0) return fail(ctx, SPAROA_ERR_INVALID_ARG, "graph_workspace: no operators");
+  if (N <= 0 || H <= 0 || W <= 0 || C <= 0)
+    return fail(ctx, SPAROA_ERR_INVALID_ARG, "graph_workspace: bad input");
+  GraphPlan pl;
+  SP_TRY(plan_graph(ctx, ops, n_ops, N, H, W, C, pl));
+  *bytes = (uint64_t)pl.total;
+  return SPAROA_OK;
+}
+
+sparoa_status sparoa_run_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_ops,
+                               const void* x, int64_t N, int64_t H, int64_t W, int64_t C, void* y,
+                               uint64_t y_bytes, sparoa_record* records) {
+  if (!ctx) return SPAROA_ERR_INVALID_ARG;
+  if (!ops || n_ops <= 0) return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: no operators");
+  if (N <= 0 || H <= 0 || W <= 0 || C <= 0 || !x)
+    return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: bad input");
+  if (C % 8 == 0 && !aligned16(x)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: misaligned input");
+  GraphPlan pl;
+  SP_TRY(plan_graph(ctx, ops, n_ops, N, H, W, C, pl));
+  std::vector<Val>& vals = pl.vals;
+  std::vector<Aux>& aux = pl.aux;
+  const size_t nnz_off = pl.nnz_off, occ_end = pl.occ_end, path_off = pl.path_off;
+  const size_t off = pl.total;
   const Val& last = vals.back();
   const uint64_t out_bytes = (uint64_t)(last.n * last.h * last.w * last.c) * 2;
   if (y && y_bytes < out_bytes)

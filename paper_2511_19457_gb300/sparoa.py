@@ -81,6 +81,7 @@ _sig("sparoa_create", [ctypes.POINTER(_P), ctypes.c_int, _P])
 _sig("sparoa_destroy", [_P])
 _sig("sparoa_set_stream", [_P, _P])
 _sig("sparoa_set_overlap", [_P, _I32])
+_sig("sparoa_graph_workspace", [_P, _P, _I32, _I64, _I64, _I64, _I64, ctypes.POINTER(ctypes.c_uint64)])
 _sig("sparoa_sync", [_P])
 _lib.sparoa_status_str.restype = ctypes.c_char_p
 _lib.sparoa_status_str.argtypes = [ctypes.c_int]
@@ -110,7 +111,7 @@ EXPORTED = ["sparoa_create", "sparoa_destroy", "sparoa_set_stream", "sparoa_set_
             "sparoa_status_str", "sparoa_last_error", "sparoa_occupancy_bytes",
             "sparoa_occupancy_init", "sparoa_op_stats", "sparoa_gemm", "sparoa_conv2d",
             "sparoa_maxpool2d", "sparoa_avgpool_global", "sparoa_bn_act", "sparoa_run_graph",
-            "sparoa_gemm_noalloc"]
+            "sparoa_graph_workspace", "sparoa_gemm_noalloc"]
 
 
 class SparoaError(RuntimeError):
@@ -351,6 +352,14 @@ class Graph:
                                thr.get("intensity_mode", 0), thr.get("force_path", 0))
         self.ops = arr
         self.n = len(ops)
+
+
+def sparoa_graph_workspace(ctx: Context, graph: Graph, x_shape) -> int:
+    """Bytes of device workspace sparoa_run_graph needs for this input shape."""
+    N, H, W, C = (int(v) for v in x_shape)
+    out = ctypes.c_uint64(0)
+    ctx._check(_lib.sparoa_graph_workspace(ctx.h, graph.ops, graph.n, N, H, W, C, ctypes.byref(out)))
+    return int(out.value)
 
 
 def sparoa_run_graph(ctx: Context, graph: Graph, x, y=None, records=False):
