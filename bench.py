@@ -12,7 +12,8 @@ pad 1, input ReLU(N(0,1)) (about half zeros), BN + ReLU epilogue:
 Metric: effective TFLOP/s = dense-equivalent FLOPs / time.
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl sparoa|reference]
-       [--workload conv|fc|resnet18|mobilenet_v2|mlp_sweep|ops|calibrate|batching] [--batch B]
+       [--workload conv|fc|resnet18|mobilenet_v2|mlp_sweep|ops|calibrate|batching|split]
+       [--batch B]
        [--thresholds default|calibrated] [--calib-out PATH]
 For N > 1 launch one process per GPU with torch.distributed.run; every rank
 runs its own replica (weak scaling), timing is the max over ranks.
@@ -47,7 +48,7 @@ def parse_args():
     p.add_argument("--impl", default="sparoa", choices=["sparoa", "reference"])
     p.add_argument("--workload", default="conv",
                    choices=["conv", "fc", "resnet18", "mobilenet_v2", "mlp_sweep", "ops", "calibrate",
-                            "batching"])
+                            "batching", "split"])
     p.add_argument("--batch", type=int, default=32)
     p.add_argument("--thresholds", default="default", choices=["default", "calibrated"],
                    help="graph workloads: the default s_thr/c_thr, or the per-operator thresholds "
@@ -863,6 +864,64 @@ def run_batching(args, rank, local_rank, world, peaks):
             "graphs": out}
 
 
+def run_split(args, rank, local_rank, world, peaks):
+    """Split execution on a batch of mixed sparsity: the MLP down projection
+    h [4096, 3072] x W2 [768, 3072]^T whose first `frac_sparse` of tokens carry
+    block-structured zeros at rho 0.9 and the rest none.  Dense, zero-skip and
+    split (rows [0, xi M) zero-skip, the rest dense, two streams) per call,
+    CUDA-graph replays over rotating sets larger than L2."""
+    import torch
+
+    from paper_2511_19457_gb300 import sparoa as sp
+    from paper_2511_19457_gb300 import synth
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    ctx = sp.Context(local_rank)
+    gen = torch.Generator(device=dev).manual_seed(0)
+    M, K, N = 4096, 3072, 768
+    W = (torch.randn(N, K, device=dev, generator=gen) / K ** 0.5).to(torch.bfloat16)
+    nb = 6
+    rows = []
+    for frac_sparse in (0.25, 0.5, 0.75):
+        ms = int(M * frac_sparse)
+        xs = []
+        for _ in range(nb):
+            h = synth.structured_activation((M, K), 0.9, "block", gen, dev)
+            h[ms:] = (torch.randn(M - ms, K, device=dev, generator=gen).abs() + 1e-3).to(torch.bfloat16)
+            xs.append(h)
+        ys = [torch.empty(M, N, dtype=torch.bfloat16, device=dev) for _ in range(nb)]
+        occ = [sp.OccupancyBuffer(M, K) for _ in range(nb)]
+        for j in range(nb):
+            sp.sparoa_op_stats(ctx, xs[j], (M, K), occ=occ[j], host=False)
+        calls = {"dense": lambda j: sp.sparoa_gemm(ctx, xs[j], W, ys[j], thr=sp.thresholds(force_path=1),
+                                                   x_occ=occ[j]),
+                 "zero-skip": lambda j: sp.sparoa_gemm(ctx, xs[j], W, ys[j],
+                                                       thr=sp.thresholds(force_path=2), x_occ=occ[j])}
+        for xi in (0.25, 0.5, 0.75):
+            calls[f"split xi={xi}"] = lambda j, xi=xi: sp.sparoa_gemm_split(ctx, xs[j], W, ys[j], xi,
+                                                                             x_occ=occ[j])
+        res = {}
+        for tag, call in calls.items():
+            for j in range(nb):
+                call(j)
+            torch.cuda.synchronize()
+            g = graph_of(call, nb)
+            g.replay()
+            res[tag] = round(time_graph(g, 20) * 1e3 / (20 * nb), 2)
+            del g
+        rows.append({"sparse_token_fraction": frac_sparse, "us_per_call": res,
+                     "best": min(res, key=res.get)})
+        del xs, ys, occ
+        torch.cuda.empty_cache()
+    ctx.close()
+    return {"metric": METRIC, "value": None, "unit": "us per call", "n_gpus": world,
+            "higher_is_better": False, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "split execution: MLP down projection [4096,3072]x[768,3072]^T, "
+                                   "a fraction of tokens block-sparse (rho 0.9), the rest dense",
+                       "l2": "rotating sets of 6 x (24 MB in + 6 MB out) > 129 MB"},
+            "rows": rows}
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -890,6 +949,8 @@ def main():
         line = run_calibrate(args, rank, local_rank, world, peaks)
     elif args.workload == "batching":
         line = run_batching(args, rank, local_rank, world, peaks)
+    elif args.workload == "split":
+        line = run_split(args, rank, local_rank, world, peaks)
     else:
         raise SystemExit(f"workload {args.workload} is not wired into bench.py")
     if rank == 0:

@@ -266,6 +266,24 @@ sparoa_status sparoa_gemm(sparoa_ctx *ctx, const void *x, int64_t M, int64_t K, 
                           sparoa_stats *host_out);
 
 /*
+ * Split execution of one FC operator (the single-GPU analogue of the paper's
+ * co-execution, Sec. 5.1 and its aggregation equation): rows [0, Ms) of x run
+ * through the zero-skip kernel and rows [Ms, M) through the dense tensor-core
+ * kernel, Ms = xi * M rounded to whole 128-row blocks.  The two parts are
+ * launched on two streams of the context (forked from and joined back into
+ * its stream, so stream capture records both) and write disjoint rows of y;
+ * y_occ, when given, is assembled from both parts.  The result equals that of
+ * sparoa_gemm up to the floating-point summation order of the chosen kernels.
+ *   xi      fraction of the rows for the zero-skip kernel, in [0, 1]
+ * Other arguments and requirements as sparoa_gemm (no host record).
+ * Errors: INVALID_ARG (also xi outside [0, 1]), UNSUPPORTED, CUDA, OOM.
+ */
+sparoa_status sparoa_gemm_split(sparoa_ctx *ctx, const void *x, int64_t M, int64_t K, const void *W,
+                                const void *W_kn, int64_t N, const sparoa_epilogue *ep, double xi,
+                                void *y, int32_t y_dtype, const sparoa_occupancy *x_occ,
+                                const sparoa_occupancy *y_occ);
+
+/*
  * 2-D convolution with threshold dispatch, NHWC:
  *   y[N, Ho, Wo, C_out] = epilogue( conv(x[N, H, W, C_in], w) ),
  *   Ho = (H + 2*pad - kh)/stride + 1,  Wo likewise.

@@ -41,6 +41,8 @@ struct sparoa_ctx {
   DevBuf splitk;      // split-K arrival counters (kept zero) + fp32 partial tiles
   std::vector<sparoa_occupancy> graph_occ;
   int overlap = 1;    // programmatic dependent launch between consecutive kernels
+  cudaStream_t aux = nullptr;                        // second stream of split execution
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;  // its fork / join with `stream`
   uint32_t* d_err() const { return reinterpret_cast<uint32_t*>(small.p); }
   int32_t* d_path() const { return reinterpret_cast<int32_t*>(reinterpret_cast<char*>(small.p) + 16); }
 };
@@ -199,12 +201,20 @@ constexpr int kSplitCounters = 65536;
 constexpr size_t kSplitCntBytes = sizeof(unsigned) * kSplitCounters;
 constexpr size_t kSplitWsBytes = (size_t)64 << 20;
 
-sparoa_status offer_splitk(sparoa_ctx* ctx, IgemmArgs* a) {
+// slot -1: the whole scratch; 0 / 1: disjoint halves, for two launches that
+// may run at the same time (split execution)
+sparoa_status offer_splitk(sparoa_ctx* ctx, IgemmArgs* a, int slot = -1) {
   if (!ctx->splitk.p) return SPAROA_OK;  // no split K
   a->ws_cnt = static_cast<unsigned*>(ctx->splitk.p);
   a->ws_cnt_len = kSplitCounters;
   a->ws = reinterpret_cast<float*>(static_cast<char*>(ctx->splitk.p) + kSplitCntBytes);
   a->ws_bytes = kSplitWsBytes;
+  if (slot >= 0) {
+    a->ws_cnt_len = kSplitCounters / 2;
+    a->ws_cnt += slot * (kSplitCounters / 2);
+    a->ws_bytes = kSplitWsBytes / 2;
+    a->ws += slot * (kSplitWsBytes / 2 / sizeof(float));
+  }
   return SPAROA_OK;
 }
 
@@ -347,7 +357,7 @@ struct GemmPlan {
   DispatchDev disp;
 };
 
-sparoa_status run_gemm(sparoa_ctx* ctx, const GemmPlan& g) {
+sparoa_status run_gemm(sparoa_ctx* ctx, const GemmPlan& g, cudaStream_t stream, int ws_slot = -1) {
   const bool small_skip = g.M <= 128 && g.W_kn != nullptr && g.K <= 8192 && (g.N % 8) == 0;
   const int force = g.disp.force;
   OccDev yo{};
@@ -370,8 +380,8 @@ sparoa_status run_gemm(sparoa_ctx* ctx, const GemmPlan& g) {
     a.out_occ = yo;
     a.emit = g.yo ? 1 : 0;
     a.err = ctx->d_err();
-    SP_TRY(offer_splitk(ctx, &a));
-    SP_CUDA(launch_igemm(a, ctx->stream));
+    SP_TRY(offer_splitk(ctx, &a, ws_slot));
+    SP_CUDA(launch_igemm(a, stream));
   }
   if (small_skip && force != 1) {
     FcSkipArgs f;
@@ -388,7 +398,7 @@ sparoa_status run_gemm(sparoa_ctx* ctx, const GemmPlan& g) {
     f.disp = g.disp;
     f.out_occ = yo;
     f.emit = g.yo ? 1 : 0;
-    SP_CUDA(launch_fcskip(f, ctx->stream));
+    SP_CUDA(launch_fcskip(f, stream));
   }
   return SPAROA_OK;
 }
@@ -504,7 +514,21 @@ sparoa_status sparoa_create(sparoa_ctx** out, int device, void* stream) {
     return SPAROA_ERR_OOM;
   }
   ctx->splitk.bytes = kSplitCntBytes + kSplitWsBytes;
+  if (cudaStreamCreateWithFlags(&ctx->aux, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&ctx->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&ctx->ev_join, cudaEventDisableTiming) != cudaSuccess) {
+    cudaGetLastError();
+    if (ctx->ev_fork) cudaEventDestroy(ctx->ev_fork);
+    if (ctx->aux) cudaStreamDestroy(ctx->aux);
+    cudaFree(ctx->splitk.p);
+    cudaFree(ctx->small.p);
+    delete ctx;
+    return SPAROA_ERR_CUDA;
+  }
   if (cudaMemset(ctx->splitk.p, 0, kSplitCntBytes) != cudaSuccess || cudaStreamSynchronize(0) != cudaSuccess) {
+    cudaEventDestroy(ctx->ev_join);
+    cudaEventDestroy(ctx->ev_fork);
+    cudaStreamDestroy(ctx->aux);
     cudaFree(ctx->splitk.p);
     cudaFree(ctx->small.p);
     delete ctx;
@@ -518,8 +542,12 @@ sparoa_status sparoa_destroy(sparoa_ctx* ctx) {
   if (!ctx) return SPAROA_OK;
   DeviceGuard g(ctx->device, ctx->overlap);
   cudaStreamSynchronize(ctx->stream);
+  if (ctx->aux) cudaStreamSynchronize(ctx->aux);
   for (DevBuf* b : {&ctx->small, &ctx->occ, &ctx->pad_x, &ctx->pad_w, &ctx->arena, &ctx->splitk})
     if (b->p) cudaFree(b->p);
+  if (ctx->ev_fork) cudaEventDestroy(ctx->ev_fork);
+  if (ctx->ev_join) cudaEventDestroy(ctx->ev_join);
+  if (ctx->aux) cudaStreamDestroy(ctx->aux);
   delete ctx;
   return SPAROA_OK;
 }
@@ -643,7 +671,7 @@ sparoa_status sparoa_gemm(sparoa_ctx* ctx, const void* x, int64_t M, int64_t K, 
   p.disp.fpb_ok = intensity_ok(t, w);
   p.disp.force = t.force_path;
   p.disp.path_out = ctx->d_path();
-  if (M > 0) SP_TRY(run_gemm(ctx, p));
+  if (M > 0) SP_TRY(run_gemm(ctx, p, ctx->stream));
   if (!host_out) return SPAROA_OK;
   uint64_t nnz = 0;
   int32_t path = 0;
@@ -652,6 +680,98 @@ sparoa_status sparoa_gemm(sparoa_ctx* ctx, const void* x, int64_t M, int64_t K, 
   SP_TRY(read_device_error(ctx));
   if (M == 0) path = host_rule(t, 0, 0, w);
   fill_stats(host_out, (uint64_t)(M * K), nnz, w, (int)M, (int)K, 1, 1, path);
+  return SPAROA_OK;
+}
+
+namespace {
+
+// The occupancy of rows [r0, R) of a tensor whose occupancy is `o`: the row
+// bitmaps and block-column masks of those rows (r0 a multiple of 128, so the
+// blocks align), the Eq. 1 counters shared.
+sparoa_occupancy occ_rows(const sparoa_occupancy& o, int64_t r0) {
+  sparoa_occupancy v = o;
+  const int64_t T = (o.C + 63) / 64, W64 = (T + 63) / 64, C32 = (o.C + 31) / 32;
+  v.row_bm = o.row_bm + r0 * W64;
+  v.blk_mask = o.blk_mask + (r0 / 128) * C32;
+  v.R = o.R - r0;
+  return v;
+}
+
+}  // namespace
+
+sparoa_status sparoa_gemm_split(sparoa_ctx* ctx, const void* x, int64_t M, int64_t K, const void* W,
+                                const void* W_kn, int64_t N, const sparoa_epilogue* ep, double xi,
+                                void* y, int32_t y_dtype, const sparoa_occupancy* x_occ,
+                                const sparoa_occupancy* y_occ) {
+  if (!ctx) return SPAROA_ERR_INVALID_ARG;
+  if (M < 0 || K <= 0 || N <= 0) return fail(ctx, SPAROA_ERR_INVALID_ARG, "gemm_split: bad shape");
+  if (M > (int64_t)1 << 30 || K > (1 << 30) || N > (1 << 30))
+    return fail(ctx, SPAROA_ERR_UNSUPPORTED, "gemm_split: dimension too large");
+  if (K % 8 || N % 8) return fail(ctx, SPAROA_ERR_INVALID_ARG, "gemm_split: K and N must be multiples of 8");
+  if (M > 0 && (!x || !W || !y)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "gemm_split: NULL tensor");
+  if (!aligned16(x) || !aligned16(W) || !aligned16(y) || (W_kn && !aligned16(W_kn)))
+    return fail(ctx, SPAROA_ERR_INVALID_ARG, "gemm_split: tensors must be 16-byte aligned");
+  if (y_dtype != SPAROA_BF16 && y_dtype != SPAROA_F32)
+    return fail(ctx, SPAROA_ERR_INVALID_ARG, "gemm_split: bad y_dtype");
+  if (y_occ && y_dtype != SPAROA_BF16)
+    return fail(ctx, SPAROA_ERR_UNSUPPORTED, "gemm_split: occupancy of an fp32 output");
+  if (!(xi >= 0.0 && xi <= 1.0)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "gemm_split: xi outside [0, 1]");
+  SP_TRY(check_ep(ctx, ep));
+  SP_TRY(check_occ(ctx, x_occ, M, K, "gemm_split x_occ"));
+  SP_TRY(check_occ(ctx, y_occ, M, N, "gemm_split y_occ"));
+  if (M == 0) return SPAROA_OK;
+  DeviceGuard g(ctx->device, ctx->overlap);
+  // rows [0, Ms) zero-skip, [Ms, M) dense; Ms whole 128-row blocks
+  int64_t Ms = (int64_t)llround(xi * (double)M / 128.0) * 128;
+  if (Ms > M) Ms = M;
+  GemmPlan p;
+  p.x = x;
+  p.M = M;
+  p.K = K;
+  p.N = N;
+  p.W = W;
+  p.W_kn = W_kn;
+  p.ep = to_dev(ep);
+  p.y = y;
+  p.y_f32 = y_dtype == SPAROA_F32;
+  p.yo = nullptr;
+  if (x_occ) p.xo = *x_occ;
+  else SP_TRY(measure(ctx, x, M, K, &p.xo));
+  if (y_occ) SP_TRY(occ_clear(ctx, *y_occ));
+  p.disp.in_nnz = reinterpret_cast<const unsigned long long*>(p.xo.nnz);
+  p.disp.numel = (unsigned long long)(M * K);
+  p.disp.s_thr = 0.5;
+  p.disp.fpb_ok = 1;
+  p.disp.path_out = nullptr;
+  const size_t ysz = p.y_f32 ? 4 : 2;
+  sparoa_occupancy yo_a, yo_b;
+  GemmPlan a = p, b = p;
+  a.M = Ms;
+  a.disp.force = 2;  // zero-skip
+  if (y_occ) {
+    yo_a = *y_occ;
+    yo_a.R = Ms;
+    a.yo = &yo_a;
+  }
+  b.x = static_cast<const char*>(x) + Ms * K * 2;
+  b.y = static_cast<char*>(y) + Ms * N * ysz;
+  b.M = M - Ms;
+  b.xo = occ_rows(p.xo, Ms);
+  b.disp.force = 1;  // dense
+  if (y_occ) {
+    yo_b = occ_rows(*y_occ, Ms);
+    b.yo = &yo_b;
+  }
+  if (Ms == 0) return run_gemm(ctx, b, ctx->stream);
+  if (Ms == M) return run_gemm(ctx, a, ctx->stream);
+  // the two parts on two streams (each takes half of the split-K scratch),
+  // forked from and joined back into the context stream
+  SP_CUDA(cudaEventRecord(ctx->ev_fork, ctx->stream));
+  SP_CUDA(cudaStreamWaitEvent(ctx->aux, ctx->ev_fork, 0));
+  SP_TRY(run_gemm(ctx, a, ctx->aux, 1));
+  SP_TRY(run_gemm(ctx, b, ctx->stream, 0));
+  SP_CUDA(cudaEventRecord(ctx->ev_join, ctx->aux));
+  SP_CUDA(cudaStreamWaitEvent(ctx->stream, ctx->ev_join, 0));
   return SPAROA_OK;
 }
 
@@ -1117,7 +1237,7 @@ sparoa_status sparoa_run_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_
         p.disp.fpb_ok = intensity_ok(t, wk);
         p.disp.force = t.force_path;
         p.disp.path_out = d_paths + i;
-        SP_TRY(run_gemm(ctx, p));
+        SP_TRY(run_gemm(ctx, p, ctx->stream));
         break;
       }
       case SPAROA_OP_MAXPOOL:

@@ -82,6 +82,7 @@ _sig("sparoa_destroy", [_P])
 _sig("sparoa_set_stream", [_P, _P])
 _sig("sparoa_set_overlap", [_P, _I32])
 _sig("sparoa_graph_workspace", [_P, _P, _I32, _I64, _I64, _I64, _I64, ctypes.POINTER(ctypes.c_uint64)])
+_sig("sparoa_gemm_split", [_P, _P, _I64, _I64, _P, _P, _I64, _P, ctypes.c_double, _P, _I32, _P, _P])
 _sig("sparoa_sync", [_P])
 _lib.sparoa_status_str.restype = ctypes.c_char_p
 _lib.sparoa_status_str.argtypes = [ctypes.c_int]
@@ -111,7 +112,7 @@ EXPORTED = ["sparoa_create", "sparoa_destroy", "sparoa_set_stream", "sparoa_set_
             "sparoa_status_str", "sparoa_last_error", "sparoa_occupancy_bytes",
             "sparoa_occupancy_init", "sparoa_op_stats", "sparoa_gemm", "sparoa_conv2d",
             "sparoa_maxpool2d", "sparoa_avgpool_global", "sparoa_bn_act", "sparoa_run_graph",
-            "sparoa_graph_workspace", "sparoa_gemm_noalloc"]
+            "sparoa_graph_workspace", "sparoa_gemm_split", "sparoa_gemm_noalloc"]
 
 
 class SparoaError(RuntimeError):
@@ -237,6 +238,19 @@ def sparoa_gemm(ctx: Context, x, W, y, W_kn=None, bias=None, bn=None, eps=1e-5, 
                                 ctypes.byref(thr) if thr is not None else None, _ptr(y), ydt,
                                 _occ(x_occ), _occ(y_occ), ctypes.byref(st) if host else None))
     return st
+
+
+def sparoa_gemm_split(ctx: Context, x, W, y, xi, W_kn=None, bias=None, bn=None, eps=1e-5,
+                      act=ACT_NONE, residual=None, x_occ=None, y_occ=None):
+    """y = epilogue(x W^T) with rows [0, xi*M) (whole 128-row blocks) on the
+    zero-skip kernel and the rest on the dense kernel, on two streams."""
+    M, K = x.shape
+    N = W.shape[0]
+    ctx._bind()
+    ep = _epi(bias, bn, eps, act, residual)
+    ydt = F32 if y.dtype == torch.float32 else BF16
+    ctx._check(_lib.sparoa_gemm_split(ctx.h, _ptr(x), M, K, _ptr(W), _ptr(W_kn), N, ctypes.byref(ep),
+                                      float(xi), _ptr(y), ydt, _occ(x_occ), _occ(y_occ)))
 
 
 def sparoa_conv2d(ctx: Context, x, w, y, stride=1, pad=0, groups=1, bias=None, bn=None, eps=1e-5,
