@@ -11,11 +11,14 @@
 // which are bound by the weight bytes and by latency, not by arithmetic.
 //
 // CTA = 64 rows x 16 output columns (many CTAs even for a handful of rows),
-// 256 threads, each owning one row x 4 columns.  Per window of kKW columns of
-// K the CTA stages its x rows whole (coalesced cp.async; the padded pitch
-// spreads the per-row reads over the banks) and the W-row slices of the
-// window's occupied columns (fp32), then every thread runs over the occupied
-// columns only.
+// 256 threads.  Per window of kKW columns of K the CTA stages its x rows whole
+// (coalesced cp.async; the first window is in flight while the occupied
+// columns are listed) and the W-row slices of the window's occupied columns
+// (bf16), then the threads split the occupied columns four ways: thread
+// (slice, row group, column group) accumulates a 4-row x 4-column outer
+// product over every fourth occupied column, reading x straight from the
+// staged rows (no compaction pass).  The four slices' sums meet in shared
+// memory, where every thread takes one row x 4 columns for the epilogue.
 #include "sparoa_kernels.h"
 
 namespace sparoa {
@@ -26,23 +29,36 @@ constexpr int kThreads = 256;
 constexpr int kTM = 64;           // rows per CTA
 constexpr int kTN = 16;           // output columns per CTA
 constexpr int kKW = 512;          // K window staged at once
-constexpr int kPitch = kKW + 8;   // bf16 elements per staged x row (16-byte multiple)
-
+constexpr int kPitch = kKW + 8;   // bf16 elements per staged x row (16-byte multiple; rows 1..7
+                                  // apart fall in different banks)
+constexpr int kSlices = 4;        // ways the occupied columns are split
 constexpr int kMaxWin = 32;       // K windows (K <= kMaxWin * kKW)
 
 struct FcSmem {
   static constexpr size_t kX = (size_t)kTM * kPitch * 2;   // x window, bf16, rows whole
-  static constexpr size_t kXC = (size_t)kKW * kTM * 2;     // occupied columns of it, [k][row], bf16
-  static constexpr size_t kW = (size_t)kKW * kTN * 4;      // occupied W rows, fp32
-  static constexpr size_t kBytes = kX + kXC + kW + (kMaxWin + 2) * 4;  // + window starts, count
+  static constexpr size_t kW = (size_t)kKW * kTN * 2;      // occupied W rows, bf16; then the slice sums
+  static_assert(kW >= (size_t)kSlices * kTM * kTN * 4, "slice sums fit the W buffer");
+  static constexpr size_t kBytes = kX + kW + (kMaxWin + 2) * 4;  // + window starts, count
 };
+
+__device__ __forceinline__ void stage_x(uint32_t xs_u32, const FcSkipArgs& a, int64_t m0, int k0, int kw,
+                                        int tid) {
+  const int chunks = kw / 8;  // K % 8 == 0
+  for (int idx = tid; idx < kTM * chunks; idx += kThreads) {
+    const int r = idx / chunks, c = idx - (idx / chunks) * chunks;
+    const bool ok = m0 + r < a.M;
+    const __nv_bfloat16* src = ok ? a.x + (m0 + r) * a.K + k0 + c * 8 : a.x;
+    cp_async_16(xs_u32 + (uint32_t)((r * kPitch + c * 8) * 2), src, ok ? 16u : 0u);
+  }
+  cp_async_commit();
+}
 
 __global__ void __launch_bounds__(kThreads) fcskip_kernel(const FcSkipArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
   __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(smem);                   // [kTM][kPitch]
-  __nv_bfloat16* xc = reinterpret_cast<__nv_bfloat16*>(smem + FcSmem::kX);      // [kk][kTM]
-  float* ws = reinterpret_cast<float*>(smem + FcSmem::kX + FcSmem::kXC);        // [kk][kTN]
-  int* s_misc = reinterpret_cast<int*>(smem + FcSmem::kX + FcSmem::kXC + FcSmem::kW);  // [0] count, [1..] window starts
+  __nv_bfloat16* wsb = reinterpret_cast<__nv_bfloat16*>(smem + FcSmem::kX);     // [kk][kTN]
+  float* red = reinterpret_cast<float*>(smem + FcSmem::kX);                     // [slice][kTM][kTN]
+  int* s_misc = reinterpret_cast<int*>(smem + FcSmem::kX + FcSmem::kW);  // [0] count, [1..] window starts
   short* s_col = reinterpret_cast<short*>(smem + FcSmem::kBytes);               // [K] occupied columns (< 32768)
   __shared__ uint32_t s_cnt[kTN];
   __shared__ uint32_t s_blk;
@@ -56,8 +72,15 @@ __global__ void __launch_bounds__(kThreads) fcskip_kernel(const FcSkipArgs a) {
   const int n0 = blockIdx.x * kTN;
   const int64_t m0 = (int64_t)blockIdx.y * kTM;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int row = tid >> 2, cq = tid & 3;  // this thread's row and 4-column group
+  const int row = tid >> 2, cq = tid & 3;  // epilogue: this thread's row and 4-column group
   const int64_t m = m0 + row;
+  // accumulation: slice sl takes occupied columns sl, sl + 4, ...; rows rg + 16 i, columns 4 cg ..
+  const int sl = tid >> 6, u = tid & 63, rg = u >> 2, cg = u & 3;
+  const uint32_t xs_u32 = smem_u32(xs);
+  const int nwin = (a.K + kKW - 1) / kKW;
+
+  // 0. the first x window is loaded while the occupied columns are listed
+  stage_x(xs_u32, a, m0, 0, a.K < kKW ? a.K : kKW, tid);
 
   // 1. occupied columns of the rows' 128-row block, in increasing order
   if (warp == 0) {
@@ -88,7 +111,6 @@ __global__ void __launch_bounds__(kThreads) fcskip_kernel(const FcSkipArgs a) {
   __syncthreads();
   const int nocc = s_misc[0];
   // where each K window starts in the (sorted) occupied list: binary search
-  const int nwin = (a.K + kKW - 1) / kKW;
   if (tid <= nwin) {
     const int bound = tid * kKW;
     int lo = 0, hi = nocc;
@@ -101,62 +123,64 @@ __global__ void __launch_bounds__(kThreads) fcskip_kernel(const FcSkipArgs a) {
   }
   __syncthreads();
 
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
-  const uint32_t xs_u32 = smem_u32(xs);
+  float acc[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
   for (int win = 0; win < nwin; ++win) {
     const int k0 = win * kKW;
     const int kw = a.K - k0 < kKW ? a.K - k0 : kKW;
     const int oc = s_misc[1 + win];
     const int nk = s_misc[2 + win] - oc;  // occupied columns of this window
+    if (win > 0 && nk > 0) stage_x(xs_u32, a, m0, k0, kw, tid);
     if (nk > 0) {
-      // 2a. x rows of the window: 16-byte chunks, zero-filled past M
-      const int chunks = kw / 8;  // K % 8 == 0
-      for (int idx = tid; idx < kTM * chunks; idx += kThreads) {
-        const int r = idx / chunks, c = idx - (idx / chunks) * chunks;
-        const bool ok = m0 + r < a.M;
-        const __nv_bfloat16* src = ok ? a.x + (m0 + r) * a.K + k0 + c * 8 : a.x;
-        cp_async_16(xs_u32 + (uint32_t)((r * kPitch + c * 8) * 2), src, ok ? 16u : 0u);
-      }
-      cp_async_commit();
-      // 2b. W rows of the window's occupied columns, columns n0 .. n0 + 16
+      // 2a. W rows of the window's occupied columns, columns n0 .. n0 + 16 (bf16)
       for (int idx = tid; idx < nk * (kTN / 8); idx += kThreads) {
         const int kk = idx >> 1, h = idx & 1;
         const int n = n0 + h * 8;
-        float f[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        if (n + 8 <= a.N) {
-          const uint4 u = __ldg(reinterpret_cast<const uint4*>(a.w_kn + (int64_t)s_col[oc + kk] * a.N + n));
-          const __nv_bfloat162* hp = reinterpret_cast<const __nv_bfloat162*>(&u);
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const float2 t = __bfloat1622float2(hp[j]);
-            f[2 * j] = t.x;
-            f[2 * j + 1] = t.y;
-          }
-        }
-        float4* dst = reinterpret_cast<float4*>(ws + kk * kTN + h * 8);
-        dst[0] = make_float4(f[0], f[1], f[2], f[3]);
-        dst[1] = make_float4(f[4], f[5], f[6], f[7]);
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (n + 8 <= a.N) v = __ldg(reinterpret_cast<const uint4*>(a.w_kn + (int64_t)s_col[oc + kk] * a.N + n));
+        *reinterpret_cast<uint4*>(wsb + kk * kTN + h * 8) = v;
       }
-      cp_async_wait<0>();
-      __syncthreads();
-      // 2c. the occupied columns of x, compacted to [kk][row]
-      for (int idx = tid; idx < nk * kTM; idx += kThreads) {
-        const int kk = idx / kTM, r = idx - (idx / kTM) * kTM;
-        xc[idx] = xs[r * kPitch + (s_col[oc + kk] - k0)];
-      }
-      __syncthreads();
-      // 2d. accumulate over the occupied columns only
-#pragma unroll 8
-      for (int kk = 0; kk < nk; ++kk) {
-        const float xv = __bfloat162float(xc[kk * kTM + row]);
-        const float4 wv = *reinterpret_cast<const float4*>(ws + kk * kTN + cq * 4);
-        acc[0] = fmaf(xv, wv.x, acc[0]);
-        acc[1] = fmaf(xv, wv.y, acc[1]);
-        acc[2] = fmaf(xv, wv.z, acc[2]);
-        acc[3] = fmaf(xv, wv.w, acc[3]);
-      }
-      __syncthreads();  // window buffers free for the next window
     }
+    cp_async_wait<0>();
+    __syncthreads();
+    if (nk > 0) {
+      // 2b. this slice's occupied columns: 4 rows x 4 columns per column
+      const __nv_bfloat16* xr = xs + rg * kPitch - k0;
+#pragma unroll 4
+      for (int kk = sl; kk < nk; kk += kSlices) {
+        const int col = s_col[oc + kk];
+        const uint2 wv = *reinterpret_cast<const uint2*>(wsb + kk * kTN + cg * 4);
+        const float2 w01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&wv.x));
+        const float2 w23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&wv.y));
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float xv = __bfloat162float(xr[i * 16 * kPitch + col]);
+          acc[i][0] = fmaf(xv, w01.x, acc[i][0]);
+          acc[i][1] = fmaf(xv, w01.y, acc[i][1]);
+          acc[i][2] = fmaf(xv, w23.x, acc[i][2]);
+          acc[i][3] = fmaf(xv, w23.y, acc[i][3]);
+        }
+      }
+    }
+    __syncthreads();  // window buffers free for the next window
+  }
+  // 2c. the slices' sums meet in shared memory (the W buffer is free now)
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    *reinterpret_cast<float4*>(red + ((sl * kTM) + rg + 16 * i) * kTN + cg * 4) =
+        make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+  __syncthreads();
+  float sum4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int s2 = 0; s2 < kSlices; ++s2) {
+    const float4 v = *reinterpret_cast<const float4*>(red + ((s2 * kTM) + row) * kTN + cq * 4);
+    sum4[0] += v.x;
+    sum4[1] += v.y;
+    sum4[2] += v.z;
+    sum4[3] += v.w;
   }
 
   // 3. epilogue
@@ -168,7 +192,7 @@ __global__ void __launch_bounds__(kThreads) fcskip_kernel(const FcSkipArgs a) {
       if (n >= a.N) continue;
       float scv = 1.f, shv = 0.f;
       epi_affine(a.ep, a.N, n, scv, shv);
-      float v = fmaf(acc[j], scv, shv);
+      float v = fmaf(sum4[j], scv, shv);
       if (a.ep.residual) v += __bfloat162float(a.ep.residual[m * a.N + n]);
       v = epi_act(v, a.ep.act);
       if (a.y_f32) {
