@@ -403,6 +403,9 @@ __global__ void __launch_bounds__(kTileThreads) dwconv_kernel(const DwArgs a_par
 // every input column it needs once per kernel row.  Tiles run channel-slice
 // major so a CTA's consecutive tiles keep their weights and affine.
 constexpr int kDwTH = 8, kDwTW = 16;
+// input tiles a stride-S CTA keeps in shared memory: two (the next step's tile
+// loads while this one is computed) when they fit next to two CTAs per SM
+constexpr int dw3_buffers(int S) { return S == 1 ? 2 : 1; }
 
 constexpr int kDwMaxBlk = 16;  // 128-row blocks one output tile can touch (Wo up to ~280)
 
@@ -411,10 +414,11 @@ __global__ void __launch_bounds__(kTileThreads) dw3_kernel(const DwArgs a_param,
   const DwArgs a = a_param;  // registers, not parameter-space loads
   constexpr int IH = (kDwTH - 1) * S + 3, IW = (kDwTW - 1) * S + 3;
   constexpr int NCOL = 3 * S + 3;  // input columns a 4-pixel strip reads: (4 - 1) S + 3
+  constexpr int NB = dw3_buffers(S);  // input tiles in flight: 2 = the next one loads during this one
   extern __shared__ __align__(16) uint8_t dsm[];
   const int Cp = ((a.C + 63) / 64) * 64;  // channels rounded up to whole slices
-  __nv_bfloat16* s_in = reinterpret_cast<__nv_bfloat16*>(dsm);  // [IH][IW][64]
-  float* s_wf = reinterpret_cast<float*>(dsm + IH * IW * 128);   // [9][Cp] weights
+  __nv_bfloat16* s_in0 = reinterpret_cast<__nv_bfloat16*>(dsm);  // [NB][IH][IW][64]
+  float* s_wf = reinterpret_cast<float*>(dsm + NB * IH * IW * 128);  // [9][Cp] weights
   float* s_sc = s_wf + 9 * Cp;                                   // [Cp] affine scale
   float* s_sh = s_sc + Cp;                                       // [Cp] affine shift
   uint32_t* s_acc = reinterpret_cast<uint32_t*>(s_sh + Cp);      // [C] when acc
@@ -453,36 +457,77 @@ __global__ void __launch_bounds__(kTileThreads) dw3_kernel(const DwArgs a_param,
   const int tiles_h = (a.Ho + kDwTH - 1) / kDwTH, tiles_w = (a.Wo + kDwTW - 1) / kDwTW;
   const int nsp = a.N * tiles_h * tiles_w;
   const int64_t items = own ? (int64_t)nsp : (int64_t)nsp * ctn;
-  const uint32_t s_in_u32 = smem_u32(s_in);
-  for (int64_t item = blockIdx.x; item < items; item += gridDim.x) {
+  // A step is one (item, channel slice): owned items run all their slices,
+  // otherwise an item is one slice.  Steps of this CTA in order: items
+  // blockIdx.x, + gridDim.x, ...; slices ct_begin .. ct_end - 1 of each.
+  struct Step {
+    int64_t item;
+    int n, ty, tx, ct, ct_end;
+  };
+  auto make_step = [&](int64_t item, int ct) {
+    Step q;
+    q.item = item;
     const int ct_begin = own ? 0 : (int)(item / nsp);
-    const int ct_end = own ? ctn : ct_begin + 1;
+    q.ct_end = own ? ctn : ct_begin + 1;
+    q.ct = ct < 0 ? ct_begin : ct;
     int rest = (int)(own ? item : item - (int64_t)ct_begin * nsp);
-    const int n = rest / (tiles_h * tiles_w);
-    rest -= n * tiles_h * tiles_w;
-    const int ty = rest / tiles_w, tx = rest - (rest / tiles_w) * tiles_w;
+    q.n = rest / (tiles_h * tiles_w);
+    rest -= q.n * tiles_h * tiles_w;
+    q.ty = rest / tiles_w;
+    q.tx = rest - q.ty * tiles_w;
+    return q;
+  };
+  auto next_step = [&](const Step& q) {
+    if (q.ct + 1 < q.ct_end) {
+      Step r = q;
+      r.ct = q.ct + 1;
+      return r;
+    }
+    return make_step(q.item + gridDim.x, -1);
+  };
+  // stage a step's input tile: 16-byte chunks (8 channels) of IH x IW pixels
+  auto stage = [&](const Step& q, int buf) {
+    const uint32_t dst = smem_u32(s_in0) + (uint32_t)(buf * IH * IW * 128);
+    const int col0 = q.ct * 64;
+    const int gy0 = q.ty * kDwTH * S - 1, gx0 = q.tx * kDwTW * S - 1;
+    const __nv_bfloat16* ximg = a.x + (int64_t)q.n * a.H * a.W * a.C;
+    for (int idx = threadIdx.x; idx < IH * IW * 8; idx += kTileThreads) {
+      const int p = idx >> 3, ch = idx & 7;
+      const int iy = p / IW, ix = p - (p / IW) * IW;
+      const int gy = gy0 + iy, gx = gx0 + ix;
+      const int cc = col0 + ch * 8;
+      const bool ok = gy >= 0 && gy < a.H && gx >= 0 && gx < a.W && cc < a.C;
+      const __nv_bfloat16* src = ok ? ximg + ((uint32_t)(gy * a.W + gx) * (uint32_t)a.C + cc) : a.x;
+      cp_async_16(dst + (uint32_t)(p * 128 + ch * 16), src, ok ? 16u : 0u);
+    }
+    cp_async_commit();
+  };
+  Step cur = make_step(blockIdx.x, -1);
+  if (NB == 2 && cur.item < items) stage(cur, 0);
+  for (int sj = 0; cur.item < items; ++sj) {
+    const Step nxt = next_step(cur);
+    const int buf = NB == 2 ? (sj & 1) : 0;
+    __syncthreads();  // the step before is done with its buffer (and, owned, with the tile flush)
+    if (NB == 2) {
+      if (nxt.item < items) {
+        stage(nxt, buf ^ 1);
+        cp_async_wait<1>();
+      } else {
+        cp_async_wait<0>();
+      }
+    } else {
+      stage(cur, 0);
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    const __nv_bfloat16* s_in = s_in0 + buf * IH * IW * 64;
+    const int n = cur.n, ty = cur.ty, tx = cur.tx, ct = cur.ct;
     // first 128-row block the tile touches (block-mask words gathered relative to it)
     const int b0 = (int)((((uint32_t)n * a.Ho + ty * kDwTH) * a.Wo + tx * kDwTW) >> 7);
-    for (int ct = ct_begin; ct < ct_end; ++ct) {
+    {
       const int col0 = ct * 64;
       const int c0 = col0 + cg * 8;
       const bool cvalid = c0 < a.C;
-      __syncthreads();  // the previous slice's readers of s_in are done
-      // stage the input tile: 16-byte chunks (8 channels) of IH x IW pixels
-      const int gy0 = ty * kDwTH * S - 1, gx0 = tx * kDwTW * S - 1;
-      const __nv_bfloat16* ximg = a.x + (int64_t)n * a.H * a.W * a.C;
-      for (int idx = threadIdx.x; idx < IH * IW * 8; idx += kTileThreads) {
-        const int p = idx >> 3, ch = idx & 7;
-        const int iy = p / IW, ix = p - (p / IW) * IW;
-        const int gy = gy0 + iy, gx = gx0 + ix;
-        const int cc = col0 + ch * 8;
-        const bool ok = gy >= 0 && gy < a.H && gx >= 0 && gx < a.W && cc < a.C;
-        const __nv_bfloat16* src = ok ? ximg + ((uint32_t)(gy * a.W + gx) * (uint32_t)a.C + cc) : a.x;
-        cp_async_16(s_in_u32 + (uint32_t)(p * 128 + ch * 16), src, ok ? 16u : 0u);
-      }
-      cp_async_commit();
-      cp_async_wait<0>();
-      __syncthreads();
       // compute: warp = output row of the tile, strip st = pixels 4 st .. 4 st + 3
       const int oy = warp, ox0 = st * 4;
       float accv[4][8];
@@ -595,7 +640,7 @@ __global__ void __launch_bounds__(kTileThreads) dw3_kernel(const DwArgs a_param,
         }
       }
     }
-    if (own && a.emit) {
+    if (own && a.emit && cur.ct + 1 == cur.ct_end) {
       // the tile's row words (owned: plain stores) and its block-mask words
       __syncthreads();
       if (threadIdx.x < kDwTH * kDwTW) {
@@ -614,6 +659,7 @@ __global__ void __launch_bounds__(kTileThreads) dw3_kernel(const DwArgs a_param,
         }
       }
     }
+    cur = nxt;
   }
   if (a.emit) cta_done(o, s_acc, acc);
 }
@@ -869,19 +915,22 @@ cudaError_t launch_dwconv(const DwArgs& a, cudaStream_t s) {
   const int C32 = (a.C + 31) / 32;
   const int Cp = ((a.C + 63) / 64) * 64;
   const size_t acc_b = a.emit && a.C <= kMaxAccCols ? sizeof(uint32_t) * (size_t)((a.C + 3) & ~3) : 0;
-  const size_t smem = (size_t)ih * iw * 128 + sizeof(float) * 11 * (size_t)Cp + acc_b +
+  const size_t smem = (size_t)dw3_buffers(a.stride) * ih * iw * 128 + sizeof(float) * 11 * (size_t)Cp + acc_b +
                       sizeof(uint32_t) * (size_t)kDwMaxBlk * C32;
   if (shape3 && ntiles < ((int64_t)1 << 31) && smem <= 200 * 1024) {
     // 2-D tiles with the input staged in shared memory; one CTA runs every
     // channel slice of its pixel tile when that still fills the GPU
-    const int64_t cap = 3LL * device_sm_count();
+    // pipelined (two input tiles) CTAs stay resident two per SM and loop over
+    // their steps; the single-buffered ones get a third CTA per SM to hide loads
+    const int64_t cap = (dw3_buffers(a.stride) == 2 ? 2LL : 3LL) * device_sm_count();
     const int inner = (nsp >= 2LL * device_sm_count() && a.C <= 4096) ? 1 : 0;
     const int64_t items = inner ? nsp : ntiles;
     const unsigned grid = (unsigned)(items < cap ? items : cap);
     auto kern = a.stride == 1 ? dw3_kernel<1> : dw3_kernel<2>;
     static size_t attr1 = 0, attr2 = 0;
     size_t& attr = a.stride == 1 ? attr1 : attr2;
-    if (smem > 48 * 1024 && smem > attr) {
+    // opt in above the 48 KB default, which also counts the static shared memory
+    if (smem > 40 * 1024 && smem > attr) {
       cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
       if (e != cudaSuccess) return e;
       attr = smem;
