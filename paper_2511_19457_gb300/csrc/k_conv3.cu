@@ -97,6 +97,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t bar_empty = sCtl + 24;
   const uint32_t bar_accf = sCtl + 40;
   const uint32_t bar_acce = sCtl + 56;
+  const uint32_t bar_mask = sCtl + 80;  // [2] zero-skip: the 128 mask threads of a slab's tile are done
   volatile int* s_abort = reinterpret_cast<volatile int*>(ctl + 72);
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(ctl + 76);
   uint32_t* s_tapm = reinterpret_cast<uint32_t*>(ctl + 128);  // [3] 9-bit occupied-tap masks
@@ -121,34 +122,42 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     mbar_init(bar_w, 1u);
     for (int b = 0; b < 2; ++b) {
+      mbar_init(bar_full + 8 * b, 1u);
+      mbar_init(bar_mask + 8 * b, 128u);
       mbar_init(bar_empty + 8 * b, 1u);
       mbar_init(bar_accf + 8 * b, 1u);
       mbar_init(bar_acce + 8 * b, (uint32_t)kEpiThreads);
     }
     *s_abort = 0;
+    fence_mbar_init();
     prefetch_tmap(&tmX);
     prefetch_tmap(&tmW);
   }
   if (warp == kMmaWarp) tmem_alloc(smem_u32(s_tmem), (uint32_t)(2 * CO));
+  // the first tile's slab origin (arithmetic on the parameters only)
+  const int t_first = blockIdx.x;
+  const int img_first = t_first / G.tiles_per_img;
+  const int oh0_first = (t_first - img_first * G.tiles_per_img) * kBM / Wp;
   pdl_wait();
   pdl_trigger();
+  if (threadIdx.x == 0 && t_first < tiles) {
+    // The first slab and the weights go out before anything else: the slab
+    // comes from HBM and gates the first MMAs.  Either path needs them.
+    mbar_arrive_expect_tx(bar_full, (uint32_t)(C / 64 * 128 * Wp * G.R));
+    for (int cb = 0; cb < C / 64; ++cb)
+      tma_load_4d(sSlab + (uint32_t)(cb * G.chunk_stride), &tmX, bar_full, cb * 64, -1, oh0_first - 1,
+                  img_first);
+    mbar_arrive_expect_tx(bar_w, (uint32_t)G.w_bytes);
+    for (int tap = 0; tap < 9; ++tap)
+      for (int cb = 0; cb < C / 64; ++cb)
+        tma_load_3d(sW + (uint32_t)((tap * (C / 64) + cb) * CO * 128), &tmW, bar_w, cb * 64, tap, 0);
+  }
   const int path = decide_path(P.disp);
   record_path(P.disp, path);
   const bool skip = path == 2;
-  if (threadIdx.x == 0) {
-    // zero-skip slabs complete on 128 mask arrivals + the TMA's arrival
-    for (int b = 0; b < 2; ++b) mbar_init(bar_full + 8 * b, skip ? 129u : 1u);
-    fence_mbar_init();
-  }
   if (warp >= 4 && warp < kMmaWarp) {
     const int et = threadIdx.x - 128;
-    for (int c = et; c < CO; c += kEpiThreads) {
-      float sc = 1.f, sh = 0.f;
-      if (c < G.Co) epi_affine(P.ep, G.Co, c, sc, sh);
-      s_scale[c] = sc;
-      s_shift[c] = sh;
-      s_acc[c] = 0u;
-    }
+    for (int c = et; c < CO; c += kEpiThreads) s_acc[c] = 0u;
     for (int i = et; i < kBM; i += kEpiThreads) s_rowbm[i] = 0ull;
   }
   tc_fence_before();
@@ -169,7 +178,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int oh0 = q0 / Wp;
       // the slab first, so that its load overlaps the mask computation below
       bool ok = true;
-      if (t_ == 0) {
+      if (t_ == 0 && j > 0) {  // the first slab went out with the weights
         ok = mbar_wait(bar_empty + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutEmpty);
         if (ok) {
           const uint32_t dst = sSlab + (uint32_t)(b * G.slab_bytes);
@@ -177,15 +186,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int cb = 0; cb < C / 64; ++cb)
             tma_load_4d(dst + (uint32_t)(cb * G.chunk_stride), &tmX, bar_full + 8 * b, cb * 64, -1,
                         oh0 - 1, img);
-        }
-        if (j == 0) {
-          // weights once, after the first slab (the slab comes from HBM and gates
-          // the first MMAs; the weights are L2 hits for all but the first CTAs):
-          // box {64 channels, 1 tap, CO rows} per (tap, channel block)
-          mbar_arrive_expect_tx(bar_w, (uint32_t)G.w_bytes);
-          for (int tap = 0; tap < 9; ++tap)
-            for (int cb = 0; cb < C / 64; ++cb)
-              tma_load_3d(sW + (uint32_t)((tap * (C / 64) + cb) * CO * 128), &tmW, bar_w, cb * 64, tap, 0);
         }
       }
       if (skip) {
@@ -228,7 +228,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // all masks written (and s_pos free for the next tile); uniform abort decision
       if (named_bar_or(1, 128, !ok)) break;
-      mbar_arrive(bar_full + 8 * b);  // 128 mask arrivals + the TMA's expect_tx arrival
+      mbar_arrive(bar_mask + 8 * b);  // this tile's masks are written
     }
   } else if (warp == kMmaWarp) {
     // -------------------------------------------------------------- MMA issue
@@ -244,7 +244,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int b = j & 1;
       if (lane == 0) {
         ok = mbar_wait(bar_acce + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutAcc) &&
-             mbar_wait(bar_full + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutFull);
+             mbar_wait(bar_full + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutFull) &&
+             (!skip || mbar_wait(bar_mask + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutFull));
       }
       if (lane == 0 && ok) {
         const int q0 = (t - (t / G.tiles_per_img) * G.tiles_per_img) * kBM;
@@ -309,6 +310,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     const OccDev o = P.out_occ;
     const bool acc_smem = emit != 0;
     const bool affine = P.ep.bias != nullptr || P.ep.bn != nullptr;  // else the column affine is 1, 0
+    // the column affine, read here rather than before the CTA barrier so that
+    // its global loads do not hold up the first MMAs
+    for (int c = et; c < CO; c += kEpiThreads) {
+      float sc = 1.f, sh = 0.f;
+      if (c < G.Co) epi_affine(P.ep, G.Co, c, sc, sh);
+      s_scale[c] = sc;
+      s_shift[c] = sh;
+    }
+    named_bar_sync(2, kEpiThreads);
     int j = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++j) {
       const int b = j & 1;
