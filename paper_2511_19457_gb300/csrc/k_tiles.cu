@@ -176,9 +176,9 @@ __device__ __forceinline__ void stats_load(const __nv_bfloat16* __restrict__ x, 
   }
 }
 
-__global__ void __launch_bounds__(kTileThreads) stats_kernel(const __nv_bfloat16* __restrict__ x,
-                                                             int64_t R, int C, OccDev o_param,
-                                                             int chunk) {
+__global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloat16* __restrict__ x,
+                                                                int64_t R, int C, OccDev o_param,
+                                                                int chunk) {
   const OccDev o = o_param;  // registers, not parameter-space loads
   extern __shared__ uint32_t s_acc[];  // [C] when acc
   __shared__ uint32_t s_cnt[8 * 64];
@@ -196,6 +196,14 @@ __global__ void __launch_bounds__(kTileThreads) stats_kernel(const __nv_bfloat16
   __syncthreads();
   pdl_wait();
   pdl_trigger();
+  // The loads of the next tile -- of this item, else the first of the CTA's
+  // next item -- are in flight while the current one is reduced.
+  uint4 u[4];
+  uint32_t m[4];
+  if ((int64_t)blockIdx.x < items) {
+    const int64_t rb = blockIdx.x / nch;
+    stats_load(x, R, C, vec, rb * 128, (int)(blockIdx.x - rb * nch) * chunk * 64, cg, rs, u, m);
+  }
   for (int64_t item = blockIdx.x; item < items; item += gridDim.x) {
     const int64_t rb = item / nch;
     const int ch = (int)(item - rb * nch);
@@ -203,9 +211,6 @@ __global__ void __launch_bounds__(kTileThreads) stats_kernel(const __nv_bfloat16
     const int ct0 = ch * chunk;
     const int ct1 = ct0 + chunk < ctn ? ct0 + chunk : ctn;
     unsigned long long rw[4] = {0ull, 0ull, 0ull, 0ull};  // row bitmap bits of this chunk, per owned row
-    uint4 u[4];
-    uint32_t m[4];
-    stats_load(x, R, C, vec, row0, ct0 * 64, cg, rs, u, m);
     for (int ct = ct0; ct < ct1; ++ct) {
       const int col0 = ct * 64;
       if (vec) {
@@ -213,7 +218,12 @@ __global__ void __launch_bounds__(kTileThreads) stats_kernel(const __nv_bfloat16
         for (int i = 0; i < 4; ++i) m[i] = nz_mask8(u[i]);
       }
       uint32_t mc[4] = {m[0], m[1], m[2], m[3]};
-      if (ct + 1 < ct1) stats_load(x, R, C, vec, row0, col0 + 64, cg, rs, u, m);  // next tile in flight
+      if (ct + 1 < ct1) {
+        stats_load(x, R, C, vec, row0, col0 + 64, cg, rs, u, m);  // next tile in flight
+      } else if (item + gridDim.x < items) {
+        const int64_t ni = item + gridDim.x, nrb2 = ni / nch;
+        stats_load(x, R, C, vec, nrb2 * 128, (int)(ni - nrb2 * nch) * chunk * 64, cg, rs, u, m);
+      }
       // row bits: lanes 8k..8k+7 share a row
       uint32_t cnt[8];
 #pragma unroll
@@ -880,7 +890,7 @@ cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev&
   if (R <= 0 || C <= 0) return cudaSuccess;
   const int chunk = stats_chunk(R, C);
   const int64_t items = ((R + 127) / 128) * ((((C + 63) / 64) + chunk - 1) / chunk);
-  const int64_t cap = 4LL * device_sm_count();  // 4 CTAs per SM
+  const int64_t cap = 3LL * device_sm_count();  // the resident CTAs (3 per SM) loop over the items
   const unsigned grid = (unsigned)(items < cap ? items : cap);
   const size_t smem = C <= kMaxAccCols ? sizeof(uint32_t) * (size_t)C : 0;
   return launch_kernel(stats_kernel, dim3(grid), dim3(kTileThreads), smem, s, x, R, C, o, chunk);
