@@ -12,7 +12,7 @@ pad 1, input ReLU(N(0,1)) (about half zeros), BN + ReLU epilogue:
 Metric: effective TFLOP/s = dense-equivalent FLOPs / time.
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl sparoa|reference]
-       [--workload conv|fc|resnet18|mobilenet_v2|mlp_sweep|ops|calibrate|batching|split]
+       [--workload conv|fc|resnet18|mobilenet_v2|vit_b16|mlp_sweep|ops|calibrate|batching|split]
        [--batch B]
        [--thresholds default|calibrated] [--calib-out PATH]
 For N > 1 launch one process per GPU with torch.distributed.run; every rank
@@ -47,8 +47,8 @@ def parse_args():
     p.add_argument("--warmup", type=int, default=400)
     p.add_argument("--impl", default="sparoa", choices=["sparoa", "reference"])
     p.add_argument("--workload", default="conv",
-                   choices=["conv", "fc", "resnet18", "mobilenet_v2", "mlp_sweep", "ops", "calibrate",
-                            "batching", "split"])
+                   choices=["conv", "fc", "resnet18", "mobilenet_v2", "vit_b16", "mlp_sweep", "ops",
+                            "calibrate", "batching", "split"])
     p.add_argument("--batch", type=int, default=32)
     p.add_argument("--thresholds", default="default", choices=["default", "calibrated"],
                    help="graph workloads: the default s_thr/c_thr, or the per-operator thresholds "
@@ -565,7 +565,8 @@ def time_graph_workload(ctx, name, batch, steps, warmup, thresholds="default"):
     from paper_2511_19457_gb300 import sparoa as sp
     from paper_2511_19457_gb300 import synth
     dev = torch.device("cuda", ctx.device)
-    ops, xb, shape = (synth.resnet18 if name == "resnet18" else synth.mobilenet_v2)(batch=batch)
+    ops, xb, shape = {"resnet18": synth.resnet18, "mobilenet_v2": synth.mobilenet_v2,
+                      "vit_b16": synth.vit}[name](batch=batch)
     if thresholds == "calibrated":
         ops = cal.apply(ops, shape, cal.load_table())
     elif isinstance(thresholds, dict):
@@ -937,7 +938,7 @@ def main():
         line = run_conv(args, rank, local_rank, world, peaks)
         if rank == 0 and not args.no_cpu_baseline:
             line["cpu_baseline"] = cpu_baseline_conv()
-    elif args.workload in ("resnet18", "mobilenet_v2"):
+    elif args.workload in ("resnet18", "mobilenet_v2", "vit_b16"):
         line = run_graph_workload(args, rank, local_rank, world, peaks, args.workload)
     elif args.workload == "fc":
         line = run_fc(args, rank, local_rank, world, peaks)

@@ -61,14 +61,32 @@ typedef enum {
     SPAROA_PATH_DEPTHWISE = 3   /* depthwise kernel (groups == channels)      */
 } sparoa_path;
 
-typedef enum { SPAROA_ACT_NONE = 0, SPAROA_ACT_RELU = 1, SPAROA_ACT_RELU6 = 2 } sparoa_act;
+/* GELU (transformer MLPs) is computed in the tanh form of Hendrycks and
+ * Gimpel, within about 1e-3 of the exact v * Phi(v). */
+typedef enum {
+    SPAROA_ACT_NONE = 0, SPAROA_ACT_RELU = 1, SPAROA_ACT_RELU6 = 2, SPAROA_ACT_GELU = 3
+} sparoa_act;
 
 typedef enum {
     SPAROA_OP_CONV2D = 1,       /* groups 1 (dispatched) or depthwise          */
     SPAROA_OP_FC = 2,           /* fully connected, input flattened to [M, K]  */
     SPAROA_OP_MAXPOOL = 3,      /* k x k max pool (kh, stride, pad)            */
     SPAROA_OP_AVGPOOL = 4,      /* global average pool, [N,H,W,C] -> [N,C]     */
-    SPAROA_OP_BN_ACT = 5        /* element-wise epilogue only                  */
+    SPAROA_OP_BN_ACT = 5,       /* element-wise epilogue only                  */
+    /* Vision-transformer operators (Sec. 6, Table 2: ViT-B16).  Tokens are the
+     * W positions of an [N, 1, T, C] value; a token-wise linear layer is a 1x1
+     * CONV2D on it. */
+    SPAROA_OP_LAYERNORM = 6,    /* per row over C; bn = fp32 [2][C] gamma, beta
+                                   (nullable), bn_eps = epsilon; C % 8 == 0   */
+    SPAROA_OP_ATTENTION = 7,    /* input rows q | k | v (3 D = 3 heads hd
+                                   values), groups = heads; output [.., D];
+                                   T <= 512, hd <= 64, hd % 8 == 0            */
+    SPAROA_OP_TOKENS = 8,       /* [N, h, w, D] -> [N, 1, 1 + h w, D]: row 0
+                                   weight (bf16 [D], the class token), rows
+                                   1.. the positions; + bias (fp32 position
+                                   table [1 + h w][D]); D % 8 == 0           */
+    SPAROA_OP_SELECT = 9        /* [N, H, W, D] -> [N, 1, 1, D]: position
+                                   `pad` of H x W (the class token: 0)       */
 } sparoa_op_kind;
 
 /*
@@ -317,6 +335,24 @@ sparoa_status sparoa_avgpool_global(sparoa_ctx *ctx, const void *x, int64_t N, i
  * C % 8 == 0.  Errors: INVALID_ARG, CUDA. */
 sparoa_status sparoa_bn_act(sparoa_ctx *ctx, const void *x, int64_t R, int64_t C,
                             const sparoa_epilogue *ep, void *y, const sparoa_occupancy *y_occ);
+
+/* Layer normalisation of x [R, C] (bf16) over C (Sec. 3.2's LN): per row
+ * (x - mean) / sqrt(biased variance + eps), then gamma * . + beta.
+ *   gamma_beta  device fp32 [2][C] or NULL (1, 0)
+ *   y_occ       occupancy of y to write (nullable)
+ * C % 8 == 0.  Errors: INVALID_ARG, CUDA. */
+sparoa_status sparoa_layernorm(sparoa_ctx *ctx, const void *x, int64_t R, int64_t C,
+                               const float *gamma_beta, float eps, void *y,
+                               const sparoa_occupancy *y_occ);
+
+/* Multi-head self-attention (Sec. 3.2's MHSA) of N sequences of T tokens:
+ * qkv [N, T, 3 D] bf16 holds per token q | k | v, each heads x head_dim values
+ * (D = heads head_dim); per head, y = softmax(Q K^T / sqrt(head_dim)) V with the
+ * heads concatenated, y [N, T, D] bf16.  T <= 512, head_dim <= 64 and a
+ * multiple of 8.  Errors: INVALID_ARG, UNSUPPORTED (sizes), CUDA. */
+sparoa_status sparoa_attention(sparoa_ctx *ctx, const void *qkv, int64_t N, int64_t T,
+                               int32_t heads, int32_t head_dim, void *y,
+                               const sparoa_occupancy *y_occ);
 
 /*
  * Run a topologically ordered operator list (Sec. 4.1 layer execution order;

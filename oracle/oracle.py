@@ -31,7 +31,7 @@ _lock = threading.Lock()
 _lib = None
 
 PATH_NONE, PATH_DENSE, PATH_SKIP, PATH_DEPTHWISE = 0, 1, 2, 3
-ACT_NONE, ACT_RELU, ACT_RELU6 = 0, 1, 2
+ACT_NONE, ACT_RELU, ACT_RELU6, ACT_GELU = 0, 1, 2, 3
 
 
 def build(force: bool = False) -> str:
@@ -257,6 +257,58 @@ def bn_act(x_bits, R, C, bias=None, bn=None, eps=1e-5, residual_bits=None, act=A
 
 
 # --------------------------------------------------------------------------
+# Vision-transformer operators (the attention-based models of Sec. 6, Table 2:
+# ViT-B16).  Plain fp64 definitions on the bf16 input values.
+# --------------------------------------------------------------------------
+def gelu(v):
+    """GELU, exact form: v * Phi(v), Phi the standard normal CDF."""
+    v = np.asarray(v, dtype=np.float64)
+    erf = np.vectorize(__import__("math").erf, otypes=[np.float64])
+    return 0.5 * v * (1.0 + erf(v / np.sqrt(2.0)))
+
+
+def layernorm(x_bits, R, C, gamma_beta=None, eps=1e-6):
+    """Layer normalisation (the LN of Sec. 3.2's encoder): per row, the C values
+    minus their mean, over sqrt(biased variance + eps); then gamma * . + beta
+    (gamma_beta fp32 [2, C]; None = 1, 0)."""
+    x = bf16_to_f64(x_bits).reshape(R, C)
+    mu = x.mean(axis=1, keepdims=True)
+    var = ((x - mu) ** 2).mean(axis=1, keepdims=True)
+    y = (x - mu) / np.sqrt(var + eps)
+    if gamma_beta is not None:
+        gb = np.asarray(gamma_beta, dtype=np.float64).reshape(2, C)
+        y = y * gb[0] + gb[1]
+    return y
+
+
+def attention(qkv_bits, N, T, heads, hd):
+    """Multi-head self-attention (the MHSA of Sec. 3.2's encoder) on the token
+    rows of one projection: row t of image n holds q | k | v, each of heads x hd
+    values; per head, out = softmax(Q K^T / sqrt(hd)) V; heads concatenated."""
+    x = bf16_to_f64(qkv_bits).reshape(N, T, 3, heads, hd)
+    q, k, v = x[:, :, 0], x[:, :, 1], x[:, :, 2]
+    s = np.einsum("nthd,nshd->nhts", q, k) / np.sqrt(hd)
+    s = s - s.max(axis=-1, keepdims=True)
+    e = np.exp(s)
+    p = e / e.sum(axis=-1, keepdims=True)
+    return np.einsum("nhts,nshd->nthd", p, v).reshape(N, T, heads * hd)
+
+
+def tokens(x_bits, N, P, D, cls_bits, pos):
+    """Token sequence of a patch embedding: row 0 the class token, rows 1..P the
+    P patch vectors, each plus its position embedding (pos fp32 [1 + P, D])."""
+    x = bf16_to_f64(x_bits).reshape(N, P, D)
+    cls = bf16_to_f64(cls_bits).reshape(1, 1, D)
+    seq = np.concatenate([np.broadcast_to(cls, (N, 1, D)), x], axis=1)
+    return seq + np.asarray(pos, dtype=np.float64).reshape(1, P + 1, D)
+
+
+def select_token(x_bits, N, T, D, index):
+    """Token `index` of every image: [N, T, D] -> [N, D]."""
+    return bf16_to_f64(x_bits).reshape(N, T, D)[:, index, :]
+
+
+# --------------------------------------------------------------------------
 # Graph walk
 # --------------------------------------------------------------------------
 @dataclass
@@ -276,7 +328,8 @@ def run_op(op: dict, x_bits: np.ndarray, x_shape: tuple, residual_bits=None,
     """Run one operator of a graph description on a bf16 input.
 
     ``op`` is a plain dict (see the workload builders): kind in
-    {"conv", "fc", "maxpool", "avgpool", "bn_act"}, plus the layer geometry,
+    {"conv", "fc", "maxpool", "avgpool", "bn_act", "layernorm", "attention",
+    "tokens", "select"}, plus the layer geometry,
     bf16 weights (uint16), fp32 bias / bn, activation and thresholds.
     """
     kind = op["kind"]
@@ -334,6 +387,38 @@ def run_op(op: dict, x_bits: np.ndarray, x_shape: tuple, residual_bits=None,
         y = bn_act(x_bits, R, C, op.get("bias"), op.get("bn"), op.get("eps", 1e-5), residual_bits,
                    op.get("act", ACT_NONE)).reshape(x_shape)
         shape = tuple(x_shape)
+    elif kind == "layernorm":
+        R = int(np.prod(x_shape[:-1]))
+        C = x_shape[-1]
+        st = stats(x_bits, R, C)
+        wk = None
+        path = PATH_NONE
+        y = layernorm(x_bits, R, C, op.get("gamma_beta"), op.get("eps", 1e-6))
+        shape = tuple(x_shape)
+    elif kind == "attention":
+        N, H, W, C3 = x_shape
+        T = H * W
+        heads = op["heads"]
+        hd = C3 // 3 // heads
+        st = stats(x_bits, N * T, C3)
+        wk = None
+        path = PATH_NONE
+        y = attention(x_bits, N, T, heads, hd)
+        shape = (N, H, W, C3 // 3)
+    elif kind == "tokens":
+        N, H, W, D = x_shape
+        st = stats(x_bits, N * H * W, D)
+        wk = None
+        path = PATH_NONE
+        y = tokens(x_bits, N, H * W, D, op["cls"], op["pos"])
+        shape = (N, 1, H * W + 1, D)
+    elif kind == "select":
+        N, H, W, D = x_shape
+        st = stats(x_bits, N * H * W, D)
+        wk = None
+        path = PATH_NONE
+        y = select_token(x_bits, N, H * W, D, op.get("index", 0))
+        shape = (N, 1, 1, D)
     else:
         raise ValueError(f"unknown operator kind {kind!r}")
     bits = f64_to_bf16(y).reshape(shape)

@@ -232,7 +232,8 @@ int orc_decide(uint64_t numel, uint64_t nnz, double fpb, uint64_t macs_eq2,
 /* ------------------------------------------------------------------------ */
 /* Epilogue: + bias, batch norm, + residual, activation (all in fp64)        */
 /* ------------------------------------------------------------------------ */
-/* act: 0 = identity, 1 = ReLU, 2 = ReLU6.
+/* act: 0 = identity, 1 = ReLU, 2 = ReLU6, 3 = GELU (exact: v * Phi(v), Phi the
+ * standard normal CDF, Phi(v) = (1 + erf(v / sqrt 2)) / 2).
  * bn (nullable) holds 4 rows of C values: gamma, beta, running mean, running var;
  * BN(v) = (v - mean) * gamma / sqrt(var + eps) + beta. */
 static double epilogue(double acc, int64_t c, int64_t C, const float *bias,
@@ -252,6 +253,8 @@ static double epilogue(double acc, int64_t c, int64_t C, const float *bias,
         v = v > 0.0 ? v : 0.0;
     else if (act == 2)
         v = v > 0.0 ? (v < 6.0 ? v : 6.0) : 0.0;
+    else if (act == 3)
+        v = 0.5 * v * (1.0 + erf(v / sqrt(2.0)));
     return v;
 }
 

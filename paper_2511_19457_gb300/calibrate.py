@@ -117,6 +117,12 @@ def graph_input_shapes(ops: list, x_shape) -> list:
             shapes.append((B, Ho, Wo, op["cout"] if kind == "conv" else C))
         elif kind == "avgpool":
             shapes.append((B, 1, 1, C))
+        elif kind == "attention":
+            shapes.append((B, H, W, C // 3))
+        elif kind == "tokens":
+            shapes.append((B, 1, H * W + 1, C))
+        elif kind == "select":
+            shapes.append((B, 1, 1, C))
         elif kind == "fc":
             shapes.append((B, 1, 1, op["cout"]))
         else:

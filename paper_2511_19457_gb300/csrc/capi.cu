@@ -262,6 +262,16 @@ Work fc_work(int64_t M, int64_t K, int64_t N) {
   return w;
 }
 
+// Q K^T and P V of every head: 2 T^2 D MACs per sequence; input bytes of q, k, v.
+Work attention_work(int64_t N, int64_t T, int64_t D) {
+  Work w;
+  w.macs = (uint64_t)(2 * N * T * T * D);
+  w.flops = 2 * w.macs;
+  w.in_bytes = (uint64_t)(N * T * 3 * D * 2);
+  w.fpb = w.in_bytes ? (double)w.flops / (double)w.in_bytes : 0.0;
+  return w;
+}
+
 sparoa_thresholds thr_or_default(const sparoa_thresholds* t) {
   if (t) return *t;
   sparoa_thresholds d;
@@ -306,7 +316,7 @@ EpiDev to_dev(const sparoa_epilogue* ep) {
 }
 
 sparoa_status check_ep(sparoa_ctx* ctx, const sparoa_epilogue* ep) {
-  if (ep && (ep->act < 0 || ep->act > 2)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "bad activation");
+  if (ep && (ep->act < 0 || ep->act > 3)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "bad activation");
   if (ep && ep->residual && !aligned16(ep->residual))
     return fail(ctx, SPAROA_ERR_INVALID_ARG, "residual must be 16-byte aligned");
   return SPAROA_OK;
@@ -933,6 +943,40 @@ sparoa_status sparoa_avgpool_global(sparoa_ctx* ctx, const void* x, int64_t N, i
   return SPAROA_OK;
 }
 
+sparoa_status sparoa_layernorm(sparoa_ctx* ctx, const void* x, int64_t R, int64_t C,
+                               const float* gamma_beta, float eps, void* y,
+                               const sparoa_occupancy* y_occ) {
+  if (!ctx) return SPAROA_ERR_INVALID_ARG;
+  if (R < 0 || C <= 0 || C % 8) return fail(ctx, SPAROA_ERR_INVALID_ARG, "layernorm: bad shape");
+  if (R > 0 && (!x || !y)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "layernorm: NULL tensor");
+  if (!aligned16(x) || !aligned16(y)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "layernorm: misaligned");
+  if (!(eps >= 0.f)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "layernorm: eps");
+  SP_TRY(check_occ(ctx, y_occ, R, C, "layernorm y_occ"));
+  DeviceGuard g(ctx->device, ctx->overlap);
+  SP_CUDA(launch_layernorm(static_cast<const __nv_bfloat16*>(x), R, (int)C, gamma_beta, eps,
+                           static_cast<__nv_bfloat16*>(y), ctx->stream));
+  if (y_occ) SP_TRY(run_stats(ctx, y, R, C, *y_occ));
+  return SPAROA_OK;
+}
+
+sparoa_status sparoa_attention(sparoa_ctx* ctx, const void* qkv, int64_t N, int64_t T, int32_t heads,
+                               int32_t head_dim, void* y, const sparoa_occupancy* y_occ) {
+  if (!ctx) return SPAROA_ERR_INVALID_ARG;
+  if (N < 0 || T <= 0 || heads <= 0 || head_dim <= 0)
+    return fail(ctx, SPAROA_ERR_INVALID_ARG, "attention: bad shape");
+  if (T > 512 || head_dim > 64 || head_dim % 8)
+    return fail(ctx, SPAROA_ERR_UNSUPPORTED, "attention: T <= 512, head_dim <= 64 and % 8 only");
+  if (N > 0 && (!qkv || !y)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "attention: NULL tensor");
+  if (!aligned16(qkv) || !aligned16(y)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "attention: misaligned");
+  const int64_t D = (int64_t)heads * head_dim;
+  SP_TRY(check_occ(ctx, y_occ, N * T, D, "attention y_occ"));
+  DeviceGuard g(ctx->device, ctx->overlap);
+  SP_CUDA(launch_attention(static_cast<const __nv_bfloat16*>(qkv), (int)N, (int)T, heads, head_dim,
+                           static_cast<__nv_bfloat16*>(y), ctx->stream));
+  if (y_occ) SP_TRY(run_stats(ctx, y, N * T, D, *y_occ));
+  return SPAROA_OK;
+}
+
 sparoa_status sparoa_bn_act(sparoa_ctx* ctx, const void* x, int64_t R, int64_t C,
                             const sparoa_epilogue* ep, void* y, const sparoa_occupancy* y_occ) {
   if (!ctx) return SPAROA_ERR_INVALID_ARG;
@@ -1031,9 +1075,36 @@ sparoa_status plan_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_ops, i
         if (in.c % 8) return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: op %d bn_act", i);
         out = {in.n, in.h, in.w, in.c};
         break;
+      case SPAROA_OP_LAYERNORM:
+        if (in.c % 8) return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: op %d layernorm C %% 8", i);
+        out = {in.n, in.h, in.w, in.c};
+        break;
+      case SPAROA_OP_ATTENTION: {
+        const int64_t T = in.h * in.w;
+        if (op.groups <= 0 || in.c % (3 * op.groups))
+          return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: op %d attention heads", i);
+        const int64_t hd = in.c / 3 / op.groups;
+        if (T > 512 || hd > 64 || hd % 8)
+          return fail(ctx, SPAROA_ERR_UNSUPPORTED, "run_graph: op %d attention T %lld hd %lld", i,
+                      (long long)T, (long long)hd);
+        out = {in.n, in.h, in.w, in.c / 3};
+        break;
+      }
+      case SPAROA_OP_TOKENS:
+        if (in.c % 8 || !op.weight || !op.bias)
+          return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: op %d tokens", i);
+        out = {in.n, 1, 1 + in.h * in.w, in.c};
+        break;
+      case SPAROA_OP_SELECT:
+        if (in.c % 8 || op.pad < 0 || op.pad >= in.h * in.w)
+          return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: op %d select", i);
+        out = {in.n, 1, 1, in.c};
+        break;
       default:
         return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: op %d kind %d", i, op.kind);
     }
+    if (op.act < 0 || op.act > 3)
+      return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: op %d activation %d", i, op.act);
     if (op.residual >= 0) {
       const Val& r = vals[(size_t)op.residual];
       if (r.n != out.n || r.h != out.h || r.w != out.w || r.c != out.c)
@@ -1255,6 +1326,32 @@ sparoa_status sparoa_run_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_
                               (int)in.c, ep, static_cast<__nv_bfloat16*>(act(i + 1)), to_dev(*yo), 1,
                               ctx->stream));
         break;
+      case SPAROA_OP_LAYERNORM:
+        SP_CUDA(launch_layernorm(static_cast<const __nv_bfloat16*>(act(op.input)), in.n * in.h * in.w,
+                                 (int)in.c, op.bn, op.bn_eps, static_cast<__nv_bfloat16*>(act(i + 1)),
+                                 ctx->stream));
+        break;
+      case SPAROA_OP_ATTENTION:
+        SP_CUDA(launch_attention(static_cast<const __nv_bfloat16*>(act(op.input)), (int)in.n,
+                                 (int)(in.h * in.w), op.groups, (int)(in.c / 3 / op.groups),
+                                 static_cast<__nv_bfloat16*>(act(i + 1)), ctx->stream));
+        break;
+      case SPAROA_OP_TOKENS:
+        SP_CUDA(launch_tokens(static_cast<const __nv_bfloat16*>(act(op.input)), (int)in.n,
+                              (int)(in.h * in.w), (int)in.c, static_cast<const __nv_bfloat16*>(op.weight),
+                              op.bias, static_cast<__nv_bfloat16*>(act(i + 1)), ctx->stream));
+        break;
+      case SPAROA_OP_SELECT:
+        SP_CUDA(launch_select(static_cast<const __nv_bfloat16*>(act(op.input)), (int)in.n,
+                              (int)(in.h * in.w), (int)in.c, op.pad, static_cast<__nv_bfloat16*>(act(i + 1)),
+                              ctx->stream));
+        break;
+    }
+    if (op.kind >= SPAROA_OP_LAYERNORM) {
+      // these kernels write no occupancy: the stats kernel measures the output
+      // (the walk cleared every occupancy block when it started)
+      SP_CUDA(launch_stats(static_cast<const __nv_bfloat16*>(act(i + 1)), out.n * out.h * out.w,
+                           (int)out.c, to_dev(*yo), ctx->stream));
     }
   }
   if (y) SP_CUDA(cudaMemcpyAsync(y, act(n_ops), out_bytes, cudaMemcpyDeviceToDevice, ctx->stream));
@@ -1275,6 +1372,8 @@ sparoa_status sparoa_run_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_
       wk = conv_work(in.n, in.h, in.w, in.c, op.c_out, op.kh, op.kw, out.h, out.w, op.groups);
     else if (op.kind == SPAROA_OP_FC)
       wk = fc_work(in.n, in.h * in.w * in.c, op.c_out);
+    else if (op.kind == SPAROA_OP_ATTENTION)
+      wk = attention_work(in.n, in.h * in.w, in.c / 3);
     sparoa_record& r = records[i];
     fill_stats(&r.stats, (uint64_t)(in.n * in.h * in.w * in.c), nnz[(size_t)op.input], wk, (int)in.n,
                (int)in.c, (int)in.h, (int)in.w, paths[(size_t)i]);

@@ -381,6 +381,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           } else if (act == 2) {
 #pragma unroll
             for (int jj = 0; jj < 16; ++jj) v[jj] = v[jj] > 0.f ? (v[jj] < 6.f ? v[jj] : 6.f) : 0.f;
+          } else if (act == 3) {
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj) v[jj] = gelu_f(v[jj]);
           }
           uint32_t pk[8];
 #pragma unroll

@@ -716,6 +716,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           } else if (act == 2) {
 #pragma unroll
             for (int jj = 0; jj < 16; ++jj) o32[jj] = fminf(fmaxf(o32[jj], 0.f), 6.f);
+          } else if (act == 3) {
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj) o32[jj] = gelu_f(o32[jj]);
           }
           if (y_f32) {
             if (mvalid) {

@@ -16,16 +16,6 @@ namespace {
 
 constexpr int kTileThreads = 256;
 
-__device__ __forceinline__ void unpack8(const uint4& u, float (&f)[8]) {
-  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    const float2 t = __bfloat1622float2(h[j]);
-    f[2 * j] = t.x;
-    f[2 * j + 1] = t.y;
-  }
-}
-
 __device__ __forceinline__ uint32_t nz_mask8(const uint4& u) {
   const uint32_t w[4] = {u.x, u.y, u.z, u.w};
   uint32_t m = 0;
@@ -37,18 +27,6 @@ __device__ __forceinline__ uint32_t nz_mask8(const uint4& u) {
   return m;
 }
 
-// Pack 8 floats to bf16 (round to nearest even); returns the vector.
-__device__ __forceinline__ uint4 pack8(const float (&f)[8]) {
-  uint4 u;
-  uint32_t* w = reinterpret_cast<uint32_t*>(&u);
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(f[2 * j]));
-    const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(f[2 * j + 1]));
-    w[j] = lo | (hi << 16);
-  }
-  return u;
-}
 
 // Occupancy of the 128-row x 64-column tiles a CTA produces.  Each thread
 // holds an 8-bit non-zero mask per row it owns (lanes 8k..8k+7 of a warp share

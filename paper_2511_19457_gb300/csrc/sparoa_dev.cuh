@@ -431,9 +431,44 @@ __device__ __forceinline__ void epi_affine(const EpiDev& e, int C, int c, float&
   }
 }
 
+// 8 bf16 values (one 16-byte chunk) to floats.
+__device__ __forceinline__ void unpack8(const uint4& u, float (&f)[8]) {
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float2 t = __bfloat1622float2(h[j]);
+    f[2 * j] = t.x;
+    f[2 * j + 1] = t.y;
+  }
+}
+
+// Pack 8 floats to bf16 (round to nearest even); returns the vector.
+__device__ __forceinline__ uint4 pack8(const float (&f)[8]) {
+  uint4 u;
+  uint32_t* w = reinterpret_cast<uint32_t*>(&u);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(f[2 * j]));
+    const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(f[2 * j + 1]));
+    w[j] = lo | (hi << 16);
+  }
+  return u;
+}
+
+// GELU in the tanh form of Hendrycks and Gimpel, 0.5 v (1 + tanh(sqrt(2/pi)
+// (v + 0.044715 v^3))), with the hardware tanh approximation: within about
+// 1e-3 of the exact form v * Phi(v), below the bf16 spacing of the result.
+__device__ __forceinline__ float gelu_f(float v) {
+  const float u = 0.7978845608028654f * fmaf(0.044715f * v, v * v, v);
+  float t;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(u));
+  return 0.5f * v * (1.f + t);
+}
+
 __device__ __forceinline__ float epi_act(float v, int act) {
   if (act == 1) return v > 0.f ? v : 0.f;
   if (act == 2) return v > 0.f ? (v < 6.f ? v : 6.f) : 0.f;
+  if (act == 3) return gelu_f(v);
   return v;
 }
 

@@ -116,6 +116,24 @@ struct FcSkipArgs {
 cudaError_t launch_fcskip(const FcSkipArgs& a, cudaStream_t s);
 
 // ----------------------------------------------------------------------------
+// Vision-transformer operators (k_vit.cu)
+// ----------------------------------------------------------------------------
+// y[r, :] = LN(x[r, :]) over C (C % 8 == 0); gb fp32 [2][C] gamma, beta or NULL.
+cudaError_t launch_layernorm(const __nv_bfloat16* x, int64_t R, int C, const float* gb, float eps,
+                             __nv_bfloat16* y, cudaStream_t s);
+// qkv [N, T, 3 D] (q | k | v per token, D = heads * hd) -> y [N, T, D];
+// T <= 512, hd <= 64, hd % 8 == 0.
+cudaError_t launch_attention(const __nv_bfloat16* qkv, int N, int T, int heads, int hd, __nv_bfloat16* y,
+                             cudaStream_t s);
+size_t attention_smem(int T, int hd);
+// x [N, P, D] -> y [N, 1 + P, D]: class token row, then the patches; + pos [1 + P][D].
+cudaError_t launch_tokens(const __nv_bfloat16* x, int N, int P, int D, const __nv_bfloat16* cls,
+                          const float* pos, __nv_bfloat16* y, cudaStream_t s);
+// x [N, T, D] -> y [N, D]: token `index`.
+cudaError_t launch_select(const __nv_bfloat16* x, int N, int T, int D, int index, __nv_bfloat16* y,
+                          cudaStream_t s);
+
+// ----------------------------------------------------------------------------
 // Memory-bound kernels (128-row x 64-channel tiles, occupancy fused)
 // ----------------------------------------------------------------------------
 // Eq. 1 statistics and bitmaps of x viewed as [R, C].  The block masks are

@@ -23,8 +23,9 @@ _lib = ctypes.CDLL(LIB_PATH)
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_OOM, ERR_CUDA, ERR_TIMEOUT = range(6)
 BF16, F32 = 0, 1
 PATH_NONE, PATH_DENSE, PATH_SKIP, PATH_DEPTHWISE = 0, 1, 2, 3
-ACT_NONE, ACT_RELU, ACT_RELU6 = 0, 1, 2
+ACT_NONE, ACT_RELU, ACT_RELU6, ACT_GELU = 0, 1, 2, 3
 OP_CONV2D, OP_FC, OP_MAXPOOL, OP_AVGPOOL, OP_BN_ACT = 1, 2, 3, 4, 5
+OP_LAYERNORM, OP_ATTENTION, OP_TOKENS, OP_SELECT = 6, 7, 8, 9
 
 _P = ctypes.c_void_p
 _I64 = ctypes.c_int64
@@ -103,6 +104,8 @@ _sig("sparoa_maxpool2d", [_P, _P, _I64, _I64, _I64, _I64, _I32, _I32, _I32, _P,
                           ctypes.POINTER(Occupancy)])
 _sig("sparoa_avgpool_global", [_P, _P, _I64, _I64, _I64, _I64, _P, ctypes.POINTER(Occupancy)])
 _sig("sparoa_bn_act", [_P, _P, _I64, _I64, ctypes.POINTER(Epilogue), _P, ctypes.POINTER(Occupancy)])
+_sig("sparoa_layernorm", [_P, _P, _I64, _I64, _P, ctypes.c_float, _P, ctypes.POINTER(Occupancy)])
+_sig("sparoa_attention", [_P, _P, _I64, _I64, _I32, _I32, _P, ctypes.POINTER(Occupancy)])
 _sig("sparoa_run_graph", [_P, ctypes.POINTER(Op), _I32, _P, _I64, _I64, _I64, _I64, _P,
                           ctypes.c_uint64, ctypes.POINTER(Record)])
 _sig("sparoa_gemm_noalloc", [_P, _P, _I64, _I64, _P, _P, _I64, ctypes.POINTER(Epilogue),
@@ -112,7 +115,8 @@ EXPORTED = ["sparoa_create", "sparoa_destroy", "sparoa_set_stream", "sparoa_set_
             "sparoa_status_str", "sparoa_last_error", "sparoa_occupancy_bytes",
             "sparoa_occupancy_init", "sparoa_op_stats", "sparoa_gemm", "sparoa_conv2d",
             "sparoa_maxpool2d", "sparoa_avgpool_global", "sparoa_bn_act", "sparoa_run_graph",
-            "sparoa_graph_workspace", "sparoa_gemm_split", "sparoa_gemm_noalloc"]
+            "sparoa_graph_workspace", "sparoa_gemm_split", "sparoa_layernorm", "sparoa_attention",
+            "sparoa_gemm_noalloc"]
 
 
 class SparoaError(RuntimeError):
@@ -290,6 +294,24 @@ def sparoa_bn_act(ctx: Context, x, y, bias=None, bn=None, eps=1e-5, act=ACT_NONE
     ctx._check(_lib.sparoa_bn_act(ctx.h, _ptr(x), R, C, ctypes.byref(ep), _ptr(y), _occ(y_occ)))
 
 
+def sparoa_layernorm(ctx: Context, x, y, gamma_beta=None, eps=1e-6, y_occ=None):
+    """y = LN(x) over the last dimension; gamma_beta fp32 [2, C] or None."""
+    R = int(np.prod(x.shape[:-1]))
+    C = x.shape[-1]
+    ctx._bind()
+    ctx._check(_lib.sparoa_layernorm(ctx.h, _ptr(x), R, C, _ptr(gamma_beta), float(eps), _ptr(y),
+                                     _occ(y_occ)))
+
+
+def sparoa_attention(ctx: Context, qkv, y, heads, y_occ=None):
+    """Multi-head self-attention: qkv [N, T, 3 D] (q | k | v per token), y [N, T, D]."""
+    N, T, C3 = qkv.shape
+    D = C3 // 3
+    ctx._bind()
+    ctx._check(_lib.sparoa_attention(ctx.h, _ptr(qkv), N, T, int(heads), D // int(heads), _ptr(y),
+                                     _occ(y_occ)))
+
+
 def sparoa_gemm_noalloc(x, W, y, W_kn=None, bias=None, bn=None, eps=1e-5, act=ACT_NONE,
                         residual=None, thr: Thresholds | None = None, host=False):
     """sparoa_gemm for callers that cannot allocate: no context, the input's
@@ -312,7 +334,8 @@ def sparoa_gemm_noalloc(x, W, y, W_kn=None, bias=None, bn=None, eps=1e-5, act=AC
 # ---------------------------------------------------------------------------
 # graphs
 # ---------------------------------------------------------------------------
-_KIND = {"conv": OP_CONV2D, "fc": OP_FC, "maxpool": OP_MAXPOOL, "avgpool": OP_AVGPOOL,
+_KIND = {"layernorm": OP_LAYERNORM, "attention": OP_ATTENTION, "tokens": OP_TOKENS, "select": OP_SELECT,
+         "conv": OP_CONV2D, "fc": OP_FC, "maxpool": OP_MAXPOOL, "avgpool": OP_AVGPOOL,
          "bn_act": OP_BN_ACT}
 
 
@@ -355,6 +378,22 @@ class Graph:
             elif d["kind"] == "maxpool":
                 o.kh = o.kw = d["k"]
                 o.stride, o.pad = d["stride"], d["pad"]
+            elif d["kind"] == "layernorm":
+                if d.get("gamma_beta") is not None:
+                    t = torch.from_numpy(np.ascontiguousarray(d["gamma_beta"], dtype=np.float32)).to(device)
+                    self.keep.append(t)
+                    o.bn = t.data_ptr()
+                o.bn_eps = d.get("eps", 1e-6)
+            elif d["kind"] == "attention":
+                o.groups = d["heads"]
+            elif d["kind"] == "tokens":
+                c = bits_to_device(d["cls"], device)
+                pos = torch.from_numpy(np.ascontiguousarray(d["pos"], dtype=np.float32)).to(device)
+                self.keep += [c, pos]
+                o.weight = c.data_ptr()
+                o.bias = pos.data_ptr()
+            elif d["kind"] == "select":
+                o.pad = d.get("index", 0)
             for name in ("bias", "bn"):
                 if d.get(name) is not None:
                     t = torch.from_numpy(np.ascontiguousarray(d[name], dtype=np.float32)).to(device)

@@ -18,6 +18,8 @@ weights, which are not available; same shapes, 224x224 RGB, batch 1/8/32):
   mlp_hidden      the hidden activation of a 768 -> 3072 -> 768 ReLU MLP drawn
                   directly at a target zero fraction, unstructured or in
                   32-channel blocks per 128-token tile
+  vit             ViT-B/16 shaped transformer (patch conv, class token, pre-norm
+                  encoder layers with GELU MLPs, head), random weights
   structured_activation  a [M, K] or NHWC activation at a target zero
                   fraction, unstructured or in blocks (threshold calibration;
                   drawn on the device the caller names)
@@ -29,7 +31,7 @@ import math
 import numpy as np
 import torch
 
-ACT_NONE, ACT_RELU, ACT_RELU6 = 0, 1, 2
+ACT_NONE, ACT_RELU, ACT_RELU6, ACT_GELU = 0, 1, 2, 3
 
 
 def _gen(seed: int) -> torch.Generator:
@@ -267,3 +269,64 @@ def structured_activation(shape, rho: float, structure: str, gen: torch.Generato
     else:
         raise ValueError(f"structure {structure!r} for shape {tuple(shape)}")
     return (v * keep.to(v.dtype)).to(torch.bfloat16)
+
+
+# --------------------------------------------------------------------------
+# vision transformer
+# --------------------------------------------------------------------------
+def _lin_op(g, inp, cin, cout, act, residual=-1, thr=None):
+    """Token-wise linear layer as a 1x1 conv with bias (no batch norm)."""
+    w = torch.randn(cout, cin, generator=g) / math.sqrt(cin)
+    return {
+        "kind": "conv", "input": inp, "residual": residual, "cin": cin, "cout": cout, "k": 1,
+        "stride": 1, "pad": 0, "groups": 1, "act": act,
+        "w": to_bf16_bits(w.reshape(cout, 1, 1, cin)),
+        "bias": (0.02 * torch.randn(cout, generator=g)).numpy().astype(np.float32), "bn": None,
+        "eps": 1e-5, "thr": dict(thr or {}),
+    }
+
+
+def _ln_op(g, inp, c):
+    gb = np.stack([1.0 + 0.1 * torch.randn(c, generator=g).numpy(),
+                   0.02 * torch.randn(c, generator=g).numpy()]).astype(np.float32)
+    return {"kind": "layernorm", "input": inp, "residual": -1, "gamma_beta": gb, "eps": 1e-6}
+
+
+def vit(batch: int = 1, seed: int = 0, img: int = 224, patch: int = 16, dim: int = 768, depth: int = 12,
+        heads: int = 12, mlp: int = 3072, classes: int = 1000, act: int = 3, thr=None):
+    """ViT-B/16 shaped (Table 2: 86M parameters, 17.6 G): 16x16/16 patch
+    embedding (conv) on [batch, 224, 224, 3], class token + position
+    embedding, `depth` pre-norm encoder layers (LN, QKV, MHSA, projection +
+    residual, LN, MLP dim -> mlp (GELU, act = 3) -> dim + residual), final LN,
+    the class token, FC -> classes.  Random N(0, 1/fan_in) weights; tokens
+    live as [batch, 1, T, dim]."""
+    g = _gen(seed)
+    x = torch.randn(batch, img, img, 3, generator=g)
+    ops = []
+
+    def add(op):
+        ops.append(op)
+        return len(ops)
+
+    P = (img // patch) ** 2
+    w = torch.randn(dim, 3 * patch * patch, generator=g) / math.sqrt(3 * patch * patch)
+    v = add({"kind": "conv", "input": 0, "residual": -1, "cin": 3, "cout": dim, "k": patch,
+             "stride": patch, "pad": 0, "groups": 1, "act": ACT_NONE,
+             "w": to_bf16_bits(w.reshape(dim, patch, patch, 3)),
+             "bias": (0.02 * torch.randn(dim, generator=g)).numpy().astype(np.float32), "bn": None,
+             "eps": 1e-5, "thr": dict(thr or {})})
+    v = add({"kind": "tokens", "input": v, "residual": -1,
+             "cls": to_bf16_bits(0.02 * torch.randn(dim, generator=g)),
+             "pos": (0.02 * torch.randn(P + 1, dim, generator=g)).numpy().astype(np.float32)})
+    for _ in range(depth):
+        a = add(_ln_op(g, v, dim))
+        q = add(_lin_op(g, a, dim, 3 * dim, ACT_NONE, thr=thr))
+        o = add({"kind": "attention", "input": q, "residual": -1, "heads": heads})
+        v = add(_lin_op(g, o, dim, dim, ACT_NONE, residual=v, thr=thr))
+        b = add(_ln_op(g, v, dim))
+        h = add(_lin_op(g, b, dim, mlp, act, thr=thr))
+        v = add(_lin_op(g, h, mlp, dim, ACT_NONE, residual=v, thr=thr))
+    v = add(_ln_op(g, v, dim))
+    v = add({"kind": "select", "input": v, "residual": -1, "index": 0})
+    add(_fc_op(g, v, dim, classes, thr=thr))
+    return ops, to_bf16_bits(x), (batch, img, img, 3)
