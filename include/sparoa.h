@@ -80,7 +80,7 @@ typedef enum {
                                    (nullable), bn_eps = epsilon; C % 8 == 0   */
     SPAROA_OP_ATTENTION = 7,    /* input rows q | k | v (3 D = 3 heads hd
                                    values), groups = heads; output [.., D];
-                                   T <= 512, hd <= 64, hd % 8 == 0            */
+                                   T <= 512, hd 16, 32 or 64                 */
     SPAROA_OP_TOKENS = 8,       /* [N, h, w, D] -> [N, 1, 1 + h w, D]: row 0
                                    weight (bf16 [D], the class token), rows
                                    1.. the positions; + bias (fp32 position
@@ -348,8 +348,9 @@ sparoa_status sparoa_layernorm(sparoa_ctx *ctx, const void *x, int64_t R, int64_
 /* Multi-head self-attention (Sec. 3.2's MHSA) of N sequences of T tokens:
  * qkv [N, T, 3 D] bf16 holds per token q | k | v, each heads x head_dim values
  * (D = heads head_dim); per head, y = softmax(Q K^T / sqrt(head_dim)) V with the
- * heads concatenated, y [N, T, D] bf16.  T <= 512, head_dim <= 64 and a
- * multiple of 8.  Errors: INVALID_ARG, UNSUPPORTED (sizes), CUDA. */
+ * heads concatenated, y [N, T, D] bf16; tensor cores, fp32 softmax and
+ * accumulation, the probabilities rounded to bf16 for the P V products.
+ * T <= 512, head_dim 16, 32 or 64.  Errors: INVALID_ARG, UNSUPPORTED (sizes), CUDA. */
 sparoa_status sparoa_attention(sparoa_ctx *ctx, const void *qkv, int64_t N, int64_t T,
                                int32_t heads, int32_t head_dim, void *y,
                                const sparoa_occupancy *y_occ);

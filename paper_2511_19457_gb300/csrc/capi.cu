@@ -964,8 +964,8 @@ sparoa_status sparoa_attention(sparoa_ctx* ctx, const void* qkv, int64_t N, int6
   if (!ctx) return SPAROA_ERR_INVALID_ARG;
   if (N < 0 || T <= 0 || heads <= 0 || head_dim <= 0)
     return fail(ctx, SPAROA_ERR_INVALID_ARG, "attention: bad shape");
-  if (T > 512 || head_dim > 64 || head_dim % 8)
-    return fail(ctx, SPAROA_ERR_UNSUPPORTED, "attention: T <= 512, head_dim <= 64 and % 8 only");
+  if (T > 512 || (head_dim != 16 && head_dim != 32 && head_dim != 64))
+    return fail(ctx, SPAROA_ERR_UNSUPPORTED, "attention: T <= 512 and head_dim 16, 32 or 64 only");
   if (N > 0 && (!qkv || !y)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "attention: NULL tensor");
   if (!aligned16(qkv) || !aligned16(y)) return fail(ctx, SPAROA_ERR_INVALID_ARG, "attention: misaligned");
   const int64_t D = (int64_t)heads * head_dim;
@@ -1084,7 +1084,7 @@ sparoa_status plan_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_ops, i
         if (op.groups <= 0 || in.c % (3 * op.groups))
           return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: op %d attention heads", i);
         const int64_t hd = in.c / 3 / op.groups;
-        if (T > 512 || hd > 64 || hd % 8)
+        if (T > 512 || (hd != 16 && hd != 32 && hd != 64))
           return fail(ctx, SPAROA_ERR_UNSUPPORTED, "run_graph: op %d attention T %lld hd %lld", i,
                       (long long)T, (long long)hd);
         out = {in.n, in.h, in.w, in.c / 3};

@@ -61,114 +61,173 @@ __global__ void __launch_bounds__(kVitThreads) layernorm_kernel(const __nv_bfloa
 }
 
 // ---------------------------------------------------------------------------
-// Multi-head self-attention.  Input rows (one per token) hold q | k | v, each
-// heads x hd values; CTA = (image, head, block of 64 queries).  The head's K
-// and V (T rows of hd bf16, rows padded by 16 bytes so that lanes reading
-// different rows hit different banks) are staged in shared memory; each warp
-// takes 8 queries in turn: lane j scores keys j, j + 32, ... against the query
-// (held in registers), the warp forms the softmax, and lane l accumulates
-// output dimensions 2l, 2l + 1 over all keys.
-constexpr int kAttnQ = 64;       // queries per CTA
-constexpr int kAttnMaxT = 512;   // tokens (16 scores per lane)
-constexpr int kAttnMaxHd = 64;   // head dimension held per lane (2 per lane)
+// Multi-head self-attention on the tensor cores (mma.sync m16n8k16, bf16 in,
+// fp32 accumulate), flash-attention style.  Input rows (one per token) hold
+// q | k | v, each heads x HD values; CTA = (image, head, block of 64 queries),
+// 4 warps of 16 queries.  The head's K (row-major) and V (transposed: one row
+// per dimension) are staged once per CTA in shared memory, zero-filled past T,
+// rows padded by 16 bytes so that the fragment loads of 8 rows x 4 columns hit
+// 32 different banks.  A warp walks the keys in blocks of 64: S = Q K^T (the
+// Q fragments stay in registers), an online softmax per query row (running
+// maximum and sum, rescaling the output), and O += P V with P taken straight
+// from the S accumulators (their layout is the A-operand layout of the next
+// MMA).  O / sum is stored as bf16.
+constexpr int kAttnQ = 64;       // queries per CTA (4 warps x 16)
+constexpr int kAttnThreads = 128;
+constexpr int kAttnMaxT = 512;
+constexpr int kAttnKB = 64;      // keys per block
 
-__global__ void __launch_bounds__(kVitThreads) attention_kernel(const __nv_bfloat16* __restrict__ qkv, int T,
-                                                                int heads, int hd,
-                                                                __nv_bfloat16* __restrict__ y) {
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                               uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+template <int HD>
+__global__ void __launch_bounds__(kAttnThreads) attention_kernel(const __nv_bfloat16* __restrict__ qkv, int T,
+                                                                 int heads, __nv_bfloat16* __restrict__ y) {
   extern __shared__ __align__(16) uint8_t smem[];
-  const int pitch = hd * 2 + 16;  // bytes per staged row
-  uint8_t* sK = smem;
-  uint8_t* sV = smem + (size_t)T * pitch;
+  const int Tp = (T + kAttnKB - 1) / kAttnKB * kAttnKB;
+  constexpr int KP = HD + 8;  // K row pitch (elements)
+  const int VP = Tp + 8;      // transposed-V row pitch (elements)
+  __nv_bfloat16* sK = reinterpret_cast<__nv_bfloat16*>(smem);        // [Tp][KP]
+  __nv_bfloat16* sVt = sK + (size_t)Tp * KP;                          // [HD][VP]
   const int n = blockIdx.x / heads, h = blockIdx.x - (blockIdx.x / heads) * heads;
-  const int D = heads * hd, row3 = 3 * D;
+  const int D = heads * HD, row3 = 3 * D;
   const __nv_bfloat16* base = qkv + (int64_t)n * T * row3;
   pdl_wait();
   pdl_trigger();
-  // stage K and V of this head: 16-byte chunks
-  const int cpr = hd / 8;  // chunks per row
-  for (int idx = threadIdx.x; idx < T * cpr; idx += kVitThreads) {
-    const int t = idx / cpr, c = idx - (idx / cpr) * cpr;
-    const __nv_bfloat16* src = base + (int64_t)t * row3 + h * hd + c * 8;
-    *reinterpret_cast<uint4*>(sK + t * pitch + c * 16) = *reinterpret_cast<const uint4*>(src + D);
-    *reinterpret_cast<uint4*>(sV + t * pitch + c * 16) = *reinterpret_cast<const uint4*>(src + 2 * D);
+  // stage K and V^T (8 values per step), zero past T
+  for (int idx = threadIdx.x; idx < Tp * (HD / 8); idx += kAttnThreads) {
+    const int t = idx / (HD / 8), c = idx - (idx / (HD / 8)) * (HD / 8);
+    uint4 kv = make_uint4(0u, 0u, 0u, 0u), vv = make_uint4(0u, 0u, 0u, 0u);
+    if (t < T) {
+      const __nv_bfloat16* src = base + (int64_t)t * row3 + h * HD + c * 8;
+      kv = *reinterpret_cast<const uint4*>(src + D);
+      vv = *reinterpret_cast<const uint4*>(src + 2 * D);
+    }
+    *reinterpret_cast<uint4*>(sK + t * KP + c * 8) = kv;
+    const __nv_bfloat16* ve = reinterpret_cast<const __nv_bfloat16*>(&vv);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) sVt[(c * 8 + k) * VP + t] = ve[k];
   }
   __syncthreads();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const float scale = rsqrtf((float)hd);
-  for (int qi = 0; qi < kAttnQ / 8; ++qi) {
-    const int t = blockIdx.y * kAttnQ + warp * (kAttnQ / 8) + qi;
-    if (t >= T) break;  // uniform across the warp
-    float q[kAttnMaxHd];
-    const __nv_bfloat16* qr = base + (int64_t)t * row3 + h * hd;
+  const int g = lane >> 2, tq = lane & 3;
+  const int q0 = blockIdx.y * kAttnQ + warp * 16;  // this warp's first query
+  if (q0 >= T) return;                             // no barrier follows
+  // Q fragments (A operand, rows g and g + 8, HD / 16 k-steps), zero past T
+  uint32_t qa[HD / 16][4];
+  {
+    const int r0 = q0 + g, r1 = q0 + g + 8;
+    const __nv_bfloat16* p0 = base + (int64_t)(r0 < T ? r0 : 0) * row3 + h * HD;
+    const __nv_bfloat16* p1 = base + (int64_t)(r1 < T ? r1 : 0) * row3 + h * HD;
 #pragma unroll
-    for (int c = 0; c < kAttnMaxHd / 8; ++c) {
-      if (c < cpr) {
-        float f[8];
-        unpack8(*reinterpret_cast<const uint4*>(qr + c * 8), f);
+    for (int kk = 0; kk < HD / 16; ++kk) {
+      const int c = kk * 16 + 2 * tq;
+      qa[kk][0] = r0 < T ? *reinterpret_cast<const uint32_t*>(p0 + c) : 0u;
+      qa[kk][1] = r1 < T ? *reinterpret_cast<const uint32_t*>(p1 + c) : 0u;
+      qa[kk][2] = r0 < T ? *reinterpret_cast<const uint32_t*>(p0 + c + 8) : 0u;
+      qa[kk][3] = r1 < T ? *reinterpret_cast<const uint32_t*>(p1 + c + 8) : 0u;
+    }
+  }
+  const float sl2 = rsqrtf((float)HD) * 1.4426950408889634f;  // 1/sqrt(HD) * log2(e)
+  float o[HD / 8][4];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) q[c * 8 + k] = f[k] * scale;
-      } else {
+  for (int j = 0; j < HD / 8; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+  float m0 = -3.0e38f, m1 = -3.0e38f, l0 = 0.f, l1 = 0.f;  // rows g, g + 8
+  for (int kb = 0; kb < Tp; kb += kAttnKB) {
+    // S = Q K^T for 64 keys: 8 n-tiles of 8 keys
+    float s[kAttnKB / 8][4];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) q[c * 8 + k] = 0.f;
+    for (int nt = 0; nt < kAttnKB / 8; ++nt) {
+      s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+      const __nv_bfloat16* kr = sK + (kb + nt * 8 + g) * KP + 2 * tq;
+#pragma unroll
+      for (int kk = 0; kk < HD / 16; ++kk) {
+        const uint32_t b0 = *reinterpret_cast<const uint32_t*>(kr + kk * 16);
+        const uint32_t b1 = *reinterpret_cast<const uint32_t*>(kr + kk * 16 + 8);
+        mma_bf16_16816(s[nt], qa[kk], b0, b1);
       }
     }
-    // scores of keys lane, lane + 32, ...
-    float sc[kAttnMaxT / 32];
-    float mx = -3.402823466e38f;
+    // keys past T do not take part
+    if (kb + kAttnKB > T) {
 #pragma unroll
-    for (int i = 0; i < kAttnMaxT / 32; ++i) {
-      const int j = lane + 32 * i;
-      float sv = -3.402823466e38f;
-      if (j < T) {
-        sv = 0.f;
-        const uint8_t* kr = sK + j * pitch;
-#pragma unroll
-        for (int c = 0; c < kAttnMaxHd / 8; ++c) {
-          if (c < cpr) {
-            float f[8];
-            unpack8(*reinterpret_cast<const uint4*>(kr + c * 16), f);
-#pragma unroll
-            for (int k = 0; k < 8; ++k) sv = fmaf(q[c * 8 + k], f[k], sv);
-          }
-        }
-      }
-      sc[i] = sv;
-      mx = fmaxf(mx, sv);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    float sum = 0.f;
-#pragma unroll
-    for (int i = 0; i < kAttnMaxT / 32; ++i) {
-      const int j = lane + 32 * i;
-      const float e = j < T ? expf(sc[i] - mx) : 0.f;
-      sc[i] = e;
-      sum += e;
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    const float inv = 1.f / sum;
-    // output dims 2 lane, 2 lane + 1: sum over keys of p_j v_j
-    float o0 = 0.f, o1 = 0.f;
-    const bool dl = 2 * lane < hd;
-#pragma unroll
-    for (int i = 0; i < kAttnMaxT / 32; ++i) {
-      if (32 * i >= T) break;
-      const float pi = sc[i];
-      const int jn = T - 32 * i < 32 ? T - 32 * i : 32;
-      for (int l2 = 0; l2 < jn; ++l2) {
-        const float p = __shfl_sync(0xffffffffu, pi, l2);
-        if (dl) {
-          const float2 v = __bfloat1622float2(
-              *reinterpret_cast<const __nv_bfloat162*>(sV + (32 * i + l2) * pitch + lane * 4));
-          o0 = fmaf(p, v.x, o0);
-          o1 = fmaf(p, v.y, o1);
-        }
+      for (int nt = 0; nt < kAttnKB / 8; ++nt) {
+        const int key = kb + nt * 8 + 2 * tq;
+        if (key >= T) s[nt][0] = s[nt][2] = -3.0e38f;
+        if (key + 1 >= T) s[nt][1] = s[nt][3] = -3.0e38f;
       }
     }
-    if (dl)
-      *reinterpret_cast<__nv_bfloat162*>(y + ((int64_t)n * T + t) * D + h * hd + 2 * lane) =
-          __floats2bfloat162_rn(o0 * inv, o1 * inv);
+    // online softmax: block maxima of rows g and g + 8 over the 4 lanes of a quad
+    float bm0 = -3.0e38f, bm1 = -3.0e38f;
+#pragma unroll
+    for (int nt = 0; nt < kAttnKB / 8; ++nt) {
+      bm0 = fmaxf(bm0, fmaxf(s[nt][0], s[nt][1]));
+      bm1 = fmaxf(bm1, fmaxf(s[nt][2], s[nt][3]));
+    }
+    bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 1));
+    bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 2));
+    bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 1));
+    bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 2));
+    const float nm0 = fmaxf(m0, bm0), nm1 = fmaxf(m1, bm1);
+    const float c0 = exp2f((m0 - nm0) * sl2), c1 = exp2f((m1 - nm1) * sl2);
+    m0 = nm0;
+    m1 = nm1;
+    float rs0 = 0.f, rs1 = 0.f;
+    uint32_t pa[kAttnKB / 16][4];  // P as A fragments of the P V MMAs
+#pragma unroll
+    for (int nt = 0; nt < kAttnKB / 8; ++nt) {
+      const float p0 = exp2f((s[nt][0] - nm0) * sl2), p1 = exp2f((s[nt][1] - nm0) * sl2);
+      const float p2 = exp2f((s[nt][2] - nm1) * sl2), p3 = exp2f((s[nt][3] - nm1) * sl2);
+      rs0 += p0 + p1;
+      rs1 += p2 + p3;
+      pa[nt >> 1][(nt & 1) * 2 + 0] = pack_bf16x2(p0, p1);
+      pa[nt >> 1][(nt & 1) * 2 + 1] = pack_bf16x2(p2, p3);
+    }
+    l0 = l0 * c0 + rs0;
+    l1 = l1 * c1 + rs1;
+#pragma unroll
+    for (int j = 0; j < HD / 8; ++j) {
+      o[j][0] *= c0;
+      o[j][1] *= c0;
+      o[j][2] *= c1;
+      o[j][3] *= c1;
+    }
+    // O += P V: n-tiles of 8 dimensions, k-steps of 16 keys
+#pragma unroll
+    for (int j = 0; j < HD / 8; ++j) {
+      const __nv_bfloat16* vr = sVt + (j * 8 + g) * VP + kb + 2 * tq;
+#pragma unroll
+      for (int kk = 0; kk < kAttnKB / 16; ++kk) {
+        const uint32_t b0 = *reinterpret_cast<const uint32_t*>(vr + kk * 16);
+        const uint32_t b1 = *reinterpret_cast<const uint32_t*>(vr + kk * 16 + 8);
+        mma_bf16_16816(o[j], pa[kk], b0, b1);
+      }
+    }
+  }
+  // row sums over the quad, then O / sum
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+  const float i0 = 1.f / l0, i1 = 1.f / l1;
+  const int r0 = q0 + g, r1 = q0 + g + 8;
+#pragma unroll
+  for (int j = 0; j < HD / 8; ++j) {
+    const int c = h * HD + j * 8 + 2 * tq;
+    if (r0 < T)
+      *reinterpret_cast<uint32_t*>(y + ((int64_t)n * T + r0) * D + c) = pack_bf16x2(o[j][0] * i0, o[j][1] * i0);
+    if (r1 < T)
+      *reinterpret_cast<uint32_t*>(y + ((int64_t)n * T + r1) * D + c) = pack_bf16x2(o[j][2] * i1, o[j][3] * i1);
   }
 }
 
@@ -224,7 +283,41 @@ unsigned grid_for(int64_t work, int per_cta) {
 
 }  // namespace
 
-size_t attention_smem(int T, int hd) { return (size_t)2 * T * (hd * 2 + 16); }
+size_t attention_smem(int T, int hd) {
+  const size_t Tp = (size_t)(T + kAttnKB - 1) / kAttnKB * kAttnKB;
+  return 2 * (Tp * (hd + 8) + (size_t)hd * (Tp + 8));
+}
+
+namespace {
+
+template <int HD>
+cudaError_t launch_attention_hd(const __nv_bfloat16* qkv, int N, int T, int heads, __nv_bfloat16* y,
+                                cudaStream_t s) {
+  const size_t smem = attention_smem(T, HD);
+  static size_t attr = 0;
+  if (smem > 40 * 1024 && smem > attr) {
+    cudaError_t e = cudaFuncSetAttribute(attention_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    attr = smem;
+  }
+  dim3 grid((unsigned)(N * heads), (unsigned)((T + kAttnQ - 1) / kAttnQ));
+  return launch_kernel(attention_kernel<HD>, grid, dim3(kAttnThreads), smem, s, qkv, T, heads, y);
+}
+
+}  // namespace
+
+cudaError_t launch_attention(const __nv_bfloat16* qkv, int N, int T, int heads, int hd, __nv_bfloat16* y,
+                             cudaStream_t s) {
+  if (N <= 0 || T <= 0) return cudaSuccess;
+  if (T > kAttnMaxT || heads <= 0) return cudaErrorInvalidValue;
+  switch (hd) {
+    case 16: return launch_attention_hd<16>(qkv, N, T, heads, y, s);
+    case 32: return launch_attention_hd<32>(qkv, N, T, heads, y, s);
+    case 64: return launch_attention_hd<64>(qkv, N, T, heads, y, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
 
 cudaError_t launch_layernorm(const __nv_bfloat16* x, int64_t R, int C, const float* gb, float eps,
                              __nv_bfloat16* y, cudaStream_t s) {
@@ -232,21 +325,6 @@ cudaError_t launch_layernorm(const __nv_bfloat16* x, int64_t R, int C, const flo
   if (C % 8) return cudaErrorInvalidValue;
   return launch_kernel(layernorm_kernel, dim3(grid_for(R, kVitThreads / 32)), dim3(kVitThreads), 0, s, x, R,
                        C, gb, eps, y);
-}
-
-cudaError_t launch_attention(const __nv_bfloat16* qkv, int N, int T, int heads, int hd, __nv_bfloat16* y,
-                             cudaStream_t s) {
-  if (N <= 0 || T <= 0) return cudaSuccess;
-  if (T > kAttnMaxT || hd > kAttnMaxHd || hd % 8 || heads <= 0) return cudaErrorInvalidValue;
-  const size_t smem = attention_smem(T, hd);
-  static size_t attr = 0;
-  if (smem > 40 * 1024 && smem > attr) {
-    cudaError_t e = cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr = smem;
-  }
-  dim3 grid((unsigned)(N * heads), (unsigned)((T + kAttnQ - 1) / kAttnQ));
-  return launch_kernel(attention_kernel, grid, dim3(kVitThreads), smem, s, qkv, T, heads, hd, y);
 }
 
 cudaError_t launch_tokens(const __nv_bfloat16* x, int N, int P, int D, const __nv_bfloat16* cls,

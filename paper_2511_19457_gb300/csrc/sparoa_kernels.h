@@ -122,7 +122,7 @@ cudaError_t launch_fcskip(const FcSkipArgs& a, cudaStream_t s);
 cudaError_t launch_layernorm(const __nv_bfloat16* x, int64_t R, int C, const float* gb, float eps,
                              __nv_bfloat16* y, cudaStream_t s);
 // qkv [N, T, 3 D] (q | k | v per token, D = heads * hd) -> y [N, T, D];
-// T <= 512, hd <= 64, hd % 8 == 0.
+// T <= 512, hd 16, 32 or 64.
 cudaError_t launch_attention(const __nv_bfloat16* qkv, int N, int T, int heads, int hd, __nv_bfloat16* y,
                              cudaStream_t s);
 size_t attention_smem(int T, int hd);
