@@ -63,7 +63,17 @@ struct Cfg {
   static constexpr int kAStage = kBM * BK * 2;
   static constexpr int kBStage = BN * BK * 2;
   static constexpr int kStageBytes = kAStage + kBStage;
-  static constexpr int kBudget = 200 * 1024 - 2 * kStgBytes - 6 * 1024 - kMaxAccCols * 4;
+  // Stage ring: about 200 KB of shared memory in all; a deeper ring made the
+  // latency-bound small GEMMs and convs slower on GB300 (256 x 3072 x 768:
+  // 13.6 -> 16.4 us).  192-wide tiles take all of the 227 KB for a fourth
+  // 40 KB stage (4096 x 3072 x 768: 26.1 -> 22.3 us).  kFixed is everything
+  // but the ring (barriers and flags of at most 12 stages) plus the 1024 bytes
+  // of alignment slack.
+  static constexpr int kFixed = 2 * kStgBytes + (2 * 12 + 4) * 8 + (12 + 8) * 4 + 16 + kMaxKWords * 4 +
+                                kMaxTaps * 8 + 4 * BN * 4 + 4 * BN * 4 + kMaxAccCols * 4 + kBM * 8 +
+                                (BN / 32) * 4 + 16 + 1024;
+  static constexpr int kBudget =
+      BN == 192 ? 227 * 1024 - kFixed : 200 * 1024 - 2 * kStgBytes - 6 * 1024 - kMaxAccCols * 4;
   static constexpr int kStagesRaw = kBudget / kStageBytes;
   static constexpr int kStages = kStagesRaw > 12 ? 12 : kStagesRaw;
   static constexpr int kLag = kStages - 2;  // cp.async stages in flight (mode 1)
@@ -83,6 +93,11 @@ struct Cfg {
   static constexpr int kBlkOff = kRowOff + kBM * 8;           // [BN / 32] block-mask words
   static constexpr int kBytes = kBlkOff + (BN / 32) * 4 + 16;
   static constexpr int kSmem = kBytes + 1024;  // slack for 1024-byte alignment
+  // TMEM: accumulator b starts at column b * kAccCols (BN rounded up to a
+  // power of two, so each starts on a power-of-two column); the allocation
+  // covers both
+  static constexpr uint32_t kAccCols = BN <= 64 ? 64u : (BN <= 128 ? 128u : 256u);
+  static constexpr uint32_t kTmemCols = 2 * kAccCols;
   static_assert(kStages >= 2, "stages");
   static_assert(kSmem <= 227 * 1024, "shared memory");
 };
@@ -266,7 +281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tmap(&tmB);
     if (!y_f32) prefetch_tmap(&tmY);
   }
-  if (warp == kMmaWarp) tmem_alloc(smem_u32(s_tmem), (uint32_t)(2 * BN));
+  if (warp == kMmaWarp) tmem_alloc(smem_u32(s_tmem), C::kTmemCols);
   if (acc_smem && warp >= 4 && warp < kMmaWarp)
     for (int c = threadIdx.x - 128; c < p.N; c += kEpiThreads) s_acc[c] = 0u;
   if (warp >= 4 && warp < kMmaWarp) {
@@ -483,7 +498,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                        kErrTimeoutAcc))
           break;
         tc_fence_after();
-        const uint32_t d = tmem + (uint32_t)(b * BN);
+        const uint32_t d = tmem + (uint32_t)b * C::kAccCols;
         bool first = true;
         int slot = it % S;
         uint32_t ph = (uint32_t)((it / S) & 1);
@@ -571,7 +586,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // epilogue warp (a warp that left alone would strand the others at a barrier)
       if (named_bar_or(2, kEpiThreads, !ok)) break;
       tc_fence_after();
-      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * BN);
+      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)b * C::kAccCols;
       // split K: every unit stores its fp32 partial tile, then takes a ticket;
       // the unit that arrives last adds the others' partials and finishes the
       // tile (nobody waits for anybody)
@@ -854,7 +869,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (warp == kMmaWarp) {
     tc_fence_after();
-    tmem_dealloc(tmem, (uint32_t)(2 * BN));
+    tmem_dealloc(tmem, C::kTmemCols);
   }
 }
 
@@ -969,25 +984,42 @@ void choose_spatial_tile(IgemmArgs& a) {
   }
 }
 
-// N tile and K split, from a sweep of (BN, ksplit) on GB300 over GEMMs
-// (M 256..4096, K 768..3072) and 3x3 convs (ResNet stages at batch 1..32):
-// 128-wide tiles win or tie nearly everywhere, 256-wide ones when there are
-// still two tiles per SM, 64-wide ones when 128-wide tiles would fill under
-// half of the SMs; splitting K pays only while the
-// tiles leave SMs idle, at most 4 ways and with at least 8 K blocks per unit
-// (the tile's last unit reads the other partials alone).
+// N tile and K split.  The main loop is bound by shared-memory traffic: a
+// K block of a 128 x BN tile is written by TMA and read back by the MMAs,
+// (128 + BN) rows each way, so a tile costs about (128 + BN) per K block and
+// the tiles take ceil(tiles / SMs) rounds over the SMs.  Of 128, 192 and 256
+// wide tiles the cheapest total wins, ties going to the narrower (a shorter
+// epilogue); 64 wide ones when 128 wide tiles would fill under half of the
+// SMs.  On GB300, GEMMs with M 1024..8192, K 768..3072 and N 768..3072 follow
+// this ordering.  K blocks are 64 wide (128-byte swizzle) wherever the
+// channel layout allows: 32 wide ones were slower at every tile width.
+// Splitting K pays only while the tiles leave SMs idle, at most 4 ways and
+// with at least 8 K blocks per unit (the tile's last unit reads the other
+// partials alone); splitting further to even out the rounds was slower (the
+// partial stores and reads cost more than the main-loop time they save).
+static int k_block(const IgemmArgs& a) { return (a.conv == 2 ? (a.Cp % 64 == 0) : (a.Ktot > 32)) ? 64 : 32; }
+
 void choose_tiles(const IgemmArgs& a, int64_t mtiles, int* bn_out, int* ks_out) {
   const int sms = num_sms();
   int bn = a.N > 64 ? 128 : 64;
   int64_t tiles = mtiles * ((a.N + bn - 1) / bn);
-  if (a.N > 128 && mtiles * ((a.N + 255) / 256) >= 2 * sms) {
-    bn = 256;  // plenty of tiles even at 256 wide: the wider epilogue amortises better
-    tiles = mtiles * ((a.N + bn - 1) / bn);
-  } else if (bn == 128 && tiles < sms / 2) {
-    bn = 64;
-    tiles = mtiles * ((a.N + bn - 1) / bn);
+  if (bn == 128) {
+    int64_t best = ((tiles + sms - 1) / sms) * (128 + 128);
+    for (int cand = 192; cand <= 256 && cand <= a.N; cand += 64) {
+      const int64_t t = mtiles * ((a.N + cand - 1) / cand);
+      const int64_t cost = ((t + sms - 1) / sms) * (128 + cand);
+      if (cost < best) {
+        best = cost;
+        bn = cand;
+        tiles = t;
+      }
+    }
+    if (bn == 128 && tiles < sms / 2) {
+      bn = 64;
+      tiles = mtiles * ((a.N + bn - 1) / bn);
+    }
   }
-  const int bk = (bn < 256 && (a.conv == 2 ? (a.Cp % 64 == 0) : (a.Ktot > 32))) ? 64 : 32;
+  const int bk = k_block(a);
   const int kblocks = (a.Ktot + bk - 1) / bk;
   int ks = 1;
   if (a.ws && a.ws_cnt && tiles < sms && tiles <= a.ws_cnt_len) {
@@ -1008,9 +1040,7 @@ cudaError_t launch_igemm(const IgemmArgs& a_in, cudaStream_t s) {
   int bn = 64, ks = 1;
   choose_tiles(a, mtiles, &bn, &ks);
   a.ksplit = ks;
-  // K block: 64 (128-byte swizzle) when the channel layout allows it and the
-  // stage ring still holds at least four stages; 32 otherwise
-  const int bk = (bn < 256 && (a.conv == 2 ? (a.Cp % 64 == 0) : (a.Ktot > 32))) ? 64 : 32;
+  const int bk = k_block(a);
   CUtensorMap tA, tB, tY;
   memset(&tA, 0, sizeof(tA));
   memset(&tY, 0, sizeof(tY));
@@ -1040,12 +1070,14 @@ cudaError_t launch_igemm(const IgemmArgs& a_in, cudaStream_t s) {
     switch (bn) {
       case 64: return launch_cfg<64, 64>(a, tA, tB, tY, tiles, s);
       case 128: return launch_cfg<128, 64>(a, tA, tB, tY, tiles, s);
+      case 192: return launch_cfg<192, 64>(a, tA, tB, tY, tiles, s);
       default: return launch_cfg<256, 64>(a, tA, tB, tY, tiles, s);
     }
   }
   switch (bn) {
     case 64: return launch_cfg<64, 32>(a, tA, tB, tY, tiles, s);
     case 128: return launch_cfg<128, 32>(a, tA, tB, tY, tiles, s);
+    case 192: return launch_cfg<192, 32>(a, tA, tB, tY, tiles, s);
     default: return launch_cfg<256, 32>(a, tA, tB, tY, tiles, s);
   }
 }

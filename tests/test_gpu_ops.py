@@ -124,7 +124,9 @@ def test_fc_layer_fp32(sp, ctx, force, with_kn):
 
 
 @pytest.mark.parametrize("M,K,N", [(200, 136, 72), (1, 512, 1000), (128, 64, 64), (300, 1280, 200),
-                                   (260, 4096, 136), (256, 3072, 768)])  # last two: few tiles, split K
+                                   (260, 4096, 136), (256, 3072, 768),  # few tiles, split K
+                                   (4096, 256, 712),   # 192-wide tiles, ragged last column tile
+                                   (6304, 128, 768)])  # 256-wide tiles, ragged last row tile
 @pytest.mark.parametrize("force", [1, 2])
 def test_gemm_epilogue_and_occupancy(sp, ctx, M, K, N, force):
     g = torch.Generator().manual_seed(M + K + N)
