@@ -28,7 +28,9 @@ def _rand_bits(shape, seed, scale=1.0, shift=0.0):
     return synth.to_bf16_bits(shift + scale * torch.randn(*shape, generator=g))
 
 
-@pytest.mark.parametrize("R,C,affine", [(300, 768, True), (197, 64, False), (1, 8, True), (4099, 192, True)])
+@pytest.mark.parametrize("R,C,affine", [(300, 768, True), (197, 64, False), (1, 8, True), (4099, 192, True),
+                                         (7, 1024, True),    # longest row held in registers
+                                         (5, 1032, True)])   # re-read path
 def test_layernorm(sp, ctx, R, C, affine):
     xb = _rand_bits((R, C), R + C, 2.0, 1.0)
     gb = None
@@ -49,7 +51,7 @@ def test_layernorm(sp, ctx, R, C, affine):
 
 
 @pytest.mark.parametrize("N,T,heads,hd", [(2, 197, 12, 64), (1, 17, 3, 64), (3, 50, 4, 32), (1, 1, 1, 16),
-                                          (1, 512, 2, 64)])
+                                          (1, 512, 2, 64), (2, 64, 2, 16), (1, 200, 2, 32)])
 def test_attention(sp, ctx, N, T, heads, hd):
     D = heads * hd
     qkvb = _rand_bits((N, T, 3 * D), N * T + D)
