@@ -172,9 +172,9 @@ sparoa_status check_occ(sparoa_ctx* ctx, const sparoa_occupancy* o, int64_t R, i
 }
 
 // Clear an occupancy block with the clear kernel (a kernel, not a memset, so
-// that consecutive launches keep overlapping).  counters_only: the Eq. 1
-// counters alone (the stats kernel writes the bitmaps whole).
-sparoa_status occ_clear(sparoa_ctx* ctx, const sparoa_occupancy& o, bool counters_only = false) {
+// that consecutive launches keep overlapping).  rows_whole: everything but the
+// row bitmaps (the stats kernel writes those whole).
+sparoa_status occ_clear(sparoa_ctx* ctx, const sparoa_occupancy& o, bool rows_whole = false) {
   const int64_t T = (o.C + 63) / 64, W64 = (T + 63) / 64, RB = (o.R + 127) / 128,
                 C32 = (o.C + 31) / 32;
   ClearArgs a = {};
@@ -184,12 +184,12 @@ sparoa_status occ_clear(sparoa_ctx* ctx, const sparoa_occupancy& o, bool counter
   a.words[1] = o.C;
   a.p[2] = o.tile_nnz;
   a.words[2] = T;
-  if (!counters_only) {
+  if (!rows_whole) {
     a.p[3] = reinterpret_cast<uint32_t*>(o.row_bm);
     a.words[3] = 2 * o.R * W64;
-    a.p[4] = o.blk_mask;
-    a.words[4] = RB * C32;
   }
+  a.p[4] = o.blk_mask;
+  a.words[4] = RB * C32;
   SP_CUDA(launch_clear(a, ctx->stream));
   return SPAROA_OK;
 }
@@ -218,8 +218,8 @@ sparoa_status offer_splitk(sparoa_ctx* ctx, IgemmArgs* a, int slot = -1) {
   return SPAROA_OK;
 }
 
-// Eq. 1 count and bitmaps of x [R, C] into `o` (counters cleared first; the
-// stats kernel writes the bitmaps whole).
+// Eq. 1 count and bitmaps of x [R, C] into `o` (counters and masks cleared
+// first; the row bitmaps too unless the stats kernel writes them whole).
 sparoa_status run_stats(sparoa_ctx* ctx, const void* x, int64_t R, int64_t C,
                         const sparoa_occupancy& o) {
   SP_TRY(occ_clear(ctx, o, stats_writes_rows_whole(R, (int)C)));

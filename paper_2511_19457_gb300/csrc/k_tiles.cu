@@ -3,7 +3,8 @@
 // 16-byte vector) in rows t/8 + 32*i, i = 0..3.  Each kernel fuses the
 // occupancy emission of its output (Eq. 1 count and bitmaps, Sec. 3.1) so the
 // next operator's dispatch reads them without another pass over HBM.
-//   stats_kernel    Eq. 1 count and bitmaps of an existing tensor
+//   stats_kernel    Eq. 1 count and bitmaps of an existing tensor (C % 8 == 0;
+//                   stats_scalar_kernel for other widths)
 //   dwconv_kernel   depthwise k x k convolution + epilogue (MobileNetV2 layers)
 //   maxpool_kernel  k x k max pooling
 //   avgpool_kernel  global average pooling
@@ -124,7 +125,8 @@ __device__ __forceinline__ void cta_done(const OccDev& o, const uint32_t* s_acc,
   for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x)
 
 // ---------------------------------------------------------------------------
-// Eq. 1 count and bitmaps of an existing tensor.  A work item is a 128-row
+// Eq. 1 count and bitmaps of a tensor of any width (the RGB input of a
+// network among them; stats_kernel below takes C % 8 == 0).  A work item is a 128-row
 // block x a chunk of up to kStatsChunk 64-column tiles; the next tile's loads
 // are issued before the current one is reduced.  Block masks are owned by
 // their item (plain stores); a row's bitmap word is stored whole when one
@@ -154,9 +156,9 @@ __device__ __forceinline__ void stats_load(const __nv_bfloat16* __restrict__ x, 
   }
 }
 
-__global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloat16* __restrict__ x,
-                                                                int64_t R, int C, OccDev o_param,
-                                                                int chunk) {
+__global__ void __launch_bounds__(kTileThreads, 3) stats_scalar_kernel(const __nv_bfloat16* __restrict__ x,
+                                                                       int64_t R, int C, OccDev o_param,
+                                                                       int chunk) {
   const OccDev o = o_param;  // registers, not parameter-space loads
   extern __shared__ uint32_t s_acc[];  // [C] when acc
   __shared__ uint32_t s_cnt[8 * 64];
@@ -262,6 +264,149 @@ __global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloa
     }
   }
   cta_done(o, s_acc, acc);
+}
+
+// ---------------------------------------------------------------------------
+// Eq. 1 count and bitmaps of a [R, C] tensor with C % 8 == 0, streamed with no
+// barrier per tile.  The 128 x 64 tiles are numbered column tile first
+// (L = ct * row_blocks + rb) and each CTA takes one contiguous range of them,
+// so that it stays on one column tile for long runs: its column counts stay
+// in registers (two 16-bit counters per 32-bit word) and reach global memory
+// once per run (a barrier reduction, one atomic per column).  Per tile and
+// row, the non-zero test is branch-free on pairs of bf16 values; row bits come
+// from a ballot (the row's word stored whole when the tensor has one column
+// tile, else OR-ed in); each warp ORs its block-column mask words into global
+// memory.  Two register buffers alternate, so the next tile's loads are in
+// flight while a tile is reduced.
+constexpr int kStatsRunTiles = 8192;  // tiles per run: 4 rows each, under the 16-bit counters' 65535
+
+// bit 15 / bit 31 set where the low / high bf16 of w is non-zero (any bit but the sign)
+__device__ __forceinline__ uint32_t nz_pairs(uint32_t w) {
+  return ((w & 0x7FFF7FFFu) + 0x7FFF7FFFu) & 0x80008000u;
+}
+
+__global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloat16* __restrict__ x,
+                                                                int64_t R, int C, OccDev o_param) {
+  const OccDev o = o_param;  // registers, not parameter-space loads
+  __shared__ uint32_t s_cnt[8 * 64];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
+  const int ctn = (C + 63) / 64;
+  const int64_t nrb = (R + 127) / 128;
+  const int64_t P = nrb * ctn;
+  const int64_t L0 = (int64_t)blockIdx.x * P / gridDim.x, L1 = ((int64_t)blockIdx.x + 1) * P / gridDim.x;
+  const bool own_row = ctn == 1;  // the row's bitmap word is this tile's bit alone
+  pdl_wait();
+  pdl_trigger();
+  int64_t Ln = L0;  // next tile to load
+  auto load = [&](uint4 (&u)[4]) {
+    if (Ln < L1) {
+      const int ct = (int)(Ln / nrb);
+      const int64_t row0 = (Ln - (int64_t)ct * nrb) * 128;
+      const int c0 = ct * 64 + cg * 8;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int64_t r = row0 + rs + 32 * i;
+        u[i] = (r < R && c0 < C) ? __ldg(reinterpret_cast<const uint4*>(x + r * C + c0))
+                                 : make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
+    ++Ln;
+  };
+  uint32_t cnt[4] = {0u, 0u, 0u, 0u};  // columns cg*8 + 2w (low half), + 2w + 1 (high half)
+  auto flush = [&](int ct) {
+    uint32_t c8[8];
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      c8[2 * w] = cnt[w] & 0xFFFFu;
+      c8[2 * w + 1] = cnt[w] >> 16;
+      cnt[w] = 0u;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      c8[j] += __shfl_xor_sync(0xffffffffu, c8[j], 8);
+      c8[j] += __shfl_xor_sync(0xffffffffu, c8[j], 16);
+    }
+    if (lane < 8) {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) s_cnt[warp * 64 + lane * 8 + j] = c8[j];
+    }
+    __syncthreads();
+    if (threadIdx.x < 64) {
+      uint32_t c = 0u;
+#pragma unroll
+      for (int w = 0; w < kTileThreads / 32; ++w) c += s_cnt[w * 64 + threadIdx.x];
+      if (c) atomicAdd(&o.col_nnz[ct * 64 + threadIdx.x], c);  // 0 for columns past C
+      uint32_t sum = c;
+#pragma unroll
+      for (int sh = 16; sh > 0; sh >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, sh);
+      if (lane == 0 && sum) {
+        atomicAdd(&o.tile_nnz[ct], sum);
+        atomicAdd(o.nnz, (unsigned long long)sum);
+      }
+    }
+    __syncthreads();
+  };
+  int run_ct = L0 < L1 ? (int)(L0 / nrb) : 0;
+  int run_tiles = 0;
+  auto tile = [&](uint4 (&u)[4], int64_t L) {
+    const int ct = (int)(L / nrb);
+    const int64_t row0 = (L - (int64_t)ct * nrb) * 128;
+    if (ct != run_ct || run_tiles == kStatsRunTiles) {  // the same for every thread
+      flush(run_ct);
+      run_ct = ct;
+      run_tiles = 0;
+    }
+    ++run_tiles;
+    uint32_t n[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      n[i][0] = nz_pairs(u[i].x);
+      n[i][1] = nz_pairs(u[i].y);
+      n[i][2] = nz_pairs(u[i].z);
+      n[i][3] = nz_pairs(u[i].w);
+    }
+    load(u);  // the tile two ahead
+    uint32_t o4[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        cnt[w] += n[i][w] >> 15;
+        o4[w] |= n[i][w];
+      }
+      const uint32_t b = __ballot_sync(0xffffffffu, (n[i][0] | n[i][1] | n[i][2] | n[i][3]) != 0u);
+      const int64_t r = row0 + rs + 32 * i;
+      if ((lane & 7) == 0 && r < R) {
+        const bool nzr = ((b >> lane) & 0xFFu) != 0u;
+        if (own_row) o.row_bm[r] = nzr ? 1ull : 0ull;
+        else if (nzr) atomicOr(&o.row_bm[r * o.W64 + (ct >> 6)], 1ull << (ct & 63));
+      }
+    }
+    // block-column mask: this thread's 8 columns over its 4 rows, then OR-ed over
+    // the warp's lanes of the same 32 columns; lanes 0 and 4 hold the two words
+    const uint32_t m8 = ((o4[0] >> 15) & 1u) | ((o4[0] >> 30) & 2u) | ((o4[1] >> 13) & 4u) |
+                        ((o4[1] >> 28) & 8u) | ((o4[2] >> 11) & 16u) | ((o4[2] >> 26) & 32u) |
+                        ((o4[3] >> 9) & 64u) | ((o4[3] >> 24) & 128u);
+    uint32_t v = m8 << ((cg & 3) * 8);
+    v |= __shfl_xor_sync(0xffffffffu, v, 1);
+    v |= __shfl_xor_sync(0xffffffffu, v, 2);
+    v |= __shfl_xor_sync(0xffffffffu, v, 8);
+    v |= __shfl_xor_sync(0xffffffffu, v, 16);
+    if ((lane & 27) == 0 && v) {  // lanes 0 and 4
+      const int w = ct * 2 + (lane >> 2);
+      if (w < o.C32) atomicOr(&o.blk_mask[(row0 >> 7) * o.C32 + w], v);
+    }
+  };
+  uint4 ua[4], ub[4];
+  load(ua);
+  load(ub);
+  for (int64_t L = L0; L < L1; ++L) {
+    tile(ua, L);
+    if (++L >= L1) break;
+    tile(ub, L);
+  }
+  flush(run_ct);
 }
 
 // ---------------------------------------------------------------------------
@@ -860,18 +1005,24 @@ int stats_chunk(int64_t R, int C) {
 }  // namespace
 
 bool stats_writes_rows_whole(int64_t R, int C) {
-  const int ctn = (C + 63) / 64;
-  return ctn <= stats_chunk(R, C);
+  (void)R;
+  return C <= 64;  // one column tile: both kernels store each row's word whole
 }
 
 cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev& o, cudaStream_t s) {
   if (R <= 0 || C <= 0) return cudaSuccess;
+  if (C % 8 == 0) {
+    const int64_t tiles = ((R + 127) / 128) * ((C + 63) / 64);
+    const int64_t cap = 3LL * device_sm_count();  // the resident CTAs (3 per SM) split the tiles
+    const unsigned grid = (unsigned)(tiles < cap ? tiles : cap);
+    return launch_kernel(stats_kernel, dim3(grid), dim3(kTileThreads), 0, s, x, R, C, o);
+  }
   const int chunk = stats_chunk(R, C);
   const int64_t items = ((R + 127) / 128) * ((((C + 63) / 64) + chunk - 1) / chunk);
   const int64_t cap = 3LL * device_sm_count();  // the resident CTAs (3 per SM) loop over the items
   const unsigned grid = (unsigned)(items < cap ? items : cap);
   const size_t smem = C <= kMaxAccCols ? sizeof(uint32_t) * (size_t)C : 0;
-  return launch_kernel(stats_kernel, dim3(grid), dim3(kTileThreads), smem, s, x, R, C, o, chunk);
+  return launch_kernel(stats_scalar_kernel, dim3(grid), dim3(kTileThreads), smem, s, x, R, C, o, chunk);
 }
 
 cudaError_t launch_clear(const ClearArgs& a, cudaStream_t s) {

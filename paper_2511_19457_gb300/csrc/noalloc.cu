@@ -117,14 +117,19 @@ extern "C" sparoa_status sparoa_gemm_noalloc(void* stream, const void* x, int64_
   OccDev xo;
   carve(b + kCtrlBytes, M, K, &xo);
   {
-    // control words and the Eq. 1 counters (which start the occupancy block);
-    // the stats kernel writes the block masks whole, and the row bitmaps too
-    // unless K is wide
+    // control words, the Eq. 1 counters (which start the occupancy block) and
+    // the block masks; the row bitmaps too unless the stats kernel writes them
+    // whole (K <= 64)
     ClearArgs z = {};
+    const int64_t blk_words = ((M + 127) / 128) * ((K + 31) / 32);
     z.p[0] = reinterpret_cast<uint32_t*>(b);
-    const char* end = stats_writes_rows_whole(M, (int)K) ? reinterpret_cast<char*>(xo.row_bm)
-                                                         : reinterpret_cast<char*>(xo.blk_mask);
-    z.words[0] = (int64_t)((end - b) / 4);
+    if (stats_writes_rows_whole(M, (int)K)) {
+      z.words[0] = (int64_t)((reinterpret_cast<char*>(xo.row_bm) - b) / 4);
+      z.p[1] = xo.blk_mask;
+      z.words[1] = blk_words;
+    } else {
+      z.words[0] = (int64_t)((reinterpret_cast<char*>(xo.blk_mask) - b) / 4) + blk_words;
+    }
     if (launch_clear(z, s) != cudaSuccess) return SPAROA_ERR_CUDA;
   }
 

@@ -136,10 +136,10 @@ cudaError_t launch_select(const __nv_bfloat16* x, int N, int T, int D, int index
 // ----------------------------------------------------------------------------
 // Memory-bound kernels (128-row x 64-channel tiles, occupancy fused)
 // ----------------------------------------------------------------------------
-// Eq. 1 statistics and bitmaps of x viewed as [R, C].  The block masks are
-// written whole, and so are the row bitmaps when stats_writes_rows_whole(R, C);
-// the counters (nnz, col_nnz, tile_nnz), and otherwise the row bitmaps, are
-// accumulated and must be zero on entry.
+// Eq. 1 statistics and bitmaps of x viewed as [R, C].  The row bitmaps are
+// written whole when stats_writes_rows_whole(R, C) (one 64-column tile); the
+// counters (nnz, col_nnz, tile_nnz), the block masks, and otherwise the row
+// bitmaps, are accumulated and must be zero on entry.
 constexpr int kStatsWholeRowCols = 512;
 bool stats_writes_rows_whole(int64_t R, int C);
 cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev& o, cudaStream_t s);
