@@ -280,9 +280,11 @@ __global__ void __launch_bounds__(kTileThreads, 3) stats_scalar_kernel(const __n
 // flight while a tile is reduced.
 constexpr int kStatsRunTiles = 8192;  // tiles per run: 4 rows each, under the 16-bit counters' 65535
 
-// bit 15 / bit 31 set where the low / high bf16 of w is non-zero (any bit but the sign)
+// bit 0 / bit 16 set where the low / high bf16 of w is non-zero (any bit but
+// the sign): adding 0x7FFF to a 15-bit magnitude carries into bit 15 exactly
+// when the magnitude is not zero, and never out of its 16-bit half
 __device__ __forceinline__ uint32_t nz_pairs(uint32_t w) {
-  return ((w & 0x7FFF7FFFu) + 0x7FFF7FFFu) & 0x80008000u;
+  return (((w & 0x7FFF7FFFu) + 0x7FFF7FFFu) >> 15) & 0x00010001u;
 }
 
 __global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloat16* __restrict__ x,
@@ -296,22 +298,32 @@ __global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloa
   const int64_t P = nrb * ctn;
   const int64_t L0 = (int64_t)blockIdx.x * P / gridDim.x, L1 = ((int64_t)blockIdx.x + 1) * P / gridDim.x;
   const bool own_row = ctn == 1;  // the row's bitmap word is this tile's bit alone
+  // (column tile, row block) of the first tile; later ones by stepping (no
+  // 64-bit division per tile)
+  const int ct0 = L0 < L1 ? (int)(L0 / nrb) : 0;
+  const int64_t rb0 = L0 - (int64_t)ct0 * nrb;
   pdl_wait();
   pdl_trigger();
-  int64_t Ln = L0;  // next tile to load
+  int64_t Ln = L0;  // next tile to load, at (l_ct, l_rb)
+  int l_ct = ct0;
+  int64_t l_rb = rb0;
   auto load = [&](uint4 (&u)[4]) {
     if (Ln < L1) {
-      const int ct = (int)(Ln / nrb);
-      const int64_t row0 = (Ln - (int64_t)ct * nrb) * 128;
-      const int c0 = ct * 64 + cg * 8;
+      const int64_t r0 = l_rb * 128 + rs;
+      const int c0 = l_ct * 64 + cg * 8;
+      const __nv_bfloat16* p = x + r0 * C + c0;
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        const int64_t r = row0 + rs + 32 * i;
-        u[i] = (r < R && c0 < C) ? __ldg(reinterpret_cast<const uint4*>(x + r * C + c0))
-                                 : make_uint4(0u, 0u, 0u, 0u);
+        u[i] = (r0 + 32 * i < R && c0 < C) ? __ldg(reinterpret_cast<const uint4*>(p))
+                                           : make_uint4(0u, 0u, 0u, 0u);
+        p += 32 * (int64_t)C;
       }
     }
     ++Ln;
+    if (++l_rb == nrb) {
+      l_rb = 0;
+      ++l_ct;
+    }
   };
   uint32_t cnt[4] = {0u, 0u, 0u, 0u};  // columns cg*8 + 2w (low half), + 2w + 1 (high half)
   auto flush = [&](int ct) {
@@ -347,11 +359,17 @@ __global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloa
     }
     __syncthreads();
   };
-  int run_ct = L0 < L1 ? (int)(L0 / nrb) : 0;
+  int run_ct = ct0;
   int run_tiles = 0;
-  auto tile = [&](uint4 (&u)[4], int64_t L) {
-    const int ct = (int)(L / nrb);
-    const int64_t row0 = (L - (int64_t)ct * nrb) * 128;
+  int t_ct = ct0;  // the tile being reduced
+  int64_t t_rb = rb0;
+  auto tile = [&](uint4 (&u)[4]) {
+    const int ct = t_ct;
+    const int64_t row0 = t_rb * 128;
+    if (++t_rb == nrb) {
+      t_rb = 0;
+      ++t_ct;
+    }
     if (ct != run_ct || run_tiles == kStatsRunTiles) {  // the same for every thread
       flush(run_ct);
       run_ct = ct;
@@ -367,14 +385,14 @@ __global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloa
       n[i][3] = nz_pairs(u[i].w);
     }
     load(u);  // the tile two ahead
-    uint32_t o4[4] = {0u, 0u, 0u, 0u};
+    uint32_t o4[4];
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      cnt[w] += (n[0][w] + n[1][w]) + (n[2][w] + n[3][w]);  // at most 4 per 16-bit half
+      o4[w] = (n[0][w] | n[1][w]) | (n[2][w] | n[3][w]);
+    }
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-#pragma unroll
-      for (int w = 0; w < 4; ++w) {
-        cnt[w] += n[i][w] >> 15;
-        o4[w] |= n[i][w];
-      }
       const uint32_t b = __ballot_sync(0xffffffffu, (n[i][0] | n[i][1] | n[i][2] | n[i][3]) != 0u);
       const int64_t r = row0 + rs + 32 * i;
       if ((lane & 7) == 0 && r < R) {
@@ -385,9 +403,9 @@ __global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloa
     }
     // block-column mask: this thread's 8 columns over its 4 rows, then OR-ed over
     // the warp's lanes of the same 32 columns; lanes 0 and 4 hold the two words
-    const uint32_t m8 = ((o4[0] >> 15) & 1u) | ((o4[0] >> 30) & 2u) | ((o4[1] >> 13) & 4u) |
-                        ((o4[1] >> 28) & 8u) | ((o4[2] >> 11) & 16u) | ((o4[2] >> 26) & 32u) |
-                        ((o4[3] >> 9) & 64u) | ((o4[3] >> 24) & 128u);
+    const uint32_t m8 = (o4[0] & 1u) | ((o4[0] >> 15) & 2u) | ((o4[1] << 2) & 4u) | ((o4[1] >> 13) & 8u) |
+                        ((o4[2] << 4) & 16u) | ((o4[2] >> 11) & 32u) | ((o4[3] << 6) & 64u) |
+                        ((o4[3] >> 9) & 128u);
     uint32_t v = m8 << ((cg & 3) * 8);
     v |= __shfl_xor_sync(0xffffffffu, v, 1);
     v |= __shfl_xor_sync(0xffffffffu, v, 2);
@@ -402,9 +420,9 @@ __global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloa
   load(ua);
   load(ub);
   for (int64_t L = L0; L < L1; ++L) {
-    tile(ua, L);
+    tile(ua);
     if (++L >= L1) break;
-    tile(ub, L);
+    tile(ub);
   }
   flush(run_ct);
 }
