@@ -592,18 +592,6 @@ __global__ void __launch_bounds__(kTileThreads) dw3_kernel(const DwArgs a_param,
   pdl_wait();
   pdl_trigger();
   if (a.path_out && blockIdx.x == 0 && threadIdx.x == 0) *a.path_out = 3;
-  // every channel's weights and affine, once per CTA
-  for (int idx = threadIdx.x; idx < 9 * Cp; idx += kTileThreads) {
-    const int c = idx / 9, t = idx - (idx / 9) * 9;
-    s_wf[t * Cp + c] = c < a.C ? __bfloat162float(a.w[(int64_t)c * 9 + t]) : 0.f;
-  }
-  for (int c = threadIdx.x; c < Cp; c += kTileThreads) {
-    float scv = 1.f, shv = 0.f;
-    if (c < a.C) epi_affine(a.ep, a.C, c, scv, shv);
-    s_sc[c] = scv;
-    s_sh[c] = shv;
-  }
-  __syncthreads();
   const int ctn = (a.C + 63) / 64;
   const int tiles_h = (a.Ho + kDwTH - 1) / kDwTH, tiles_w = (a.Wo + kDwTW - 1) / kDwTW;
   const int nsp = a.N * tiles_h * tiles_w;
@@ -654,7 +642,59 @@ __global__ void __launch_bounds__(kTileThreads) dw3_kernel(const DwArgs a_param,
     cp_async_commit();
   };
   Step cur = make_step(blockIdx.x, -1);
-  if (NB == 2 && cur.item < items) stage(cur, 0);
+  if (cur.item < items) stage(cur, 0);
+  // weights and affine of channels [cb, ce) into shared memory: 8 independent
+  // weight loads per thread before their stores, the affine 4 channels at a time
+  auto stage_weights = [&](int cb, int ce) {
+    const int nw = 9 * (ce - cb);
+    for (int base = threadIdx.x; base < nw; base += 8 * kTileThreads) {
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int idx = base + u * kTileThreads;
+        const int gi = cb * 9 + idx;
+        v[u] = (idx < nw && gi / 9 < a.C) ? __bfloat162float(a.w[gi]) : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int idx = base + u * kTileThreads;
+        if (idx < nw) {
+          const int gi = cb * 9 + idx;
+          const int c = gi / 9, t = gi - (gi / 9) * 9;
+          s_wf[t * Cp + c] = v[u];
+        }
+      }
+    }
+    for (int c0 = cb + (int)threadIdx.x; c0 < ce; c0 += 4 * kTileThreads) {
+      float scv[4], shv[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int c = c0 + u * kTileThreads;
+        scv[u] = 1.f;
+        shv[u] = 0.f;
+        if (c < a.C) epi_affine(a.ep, a.C, c, scv[u], shv[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int c = c0 + u * kTileThreads;
+        if (c < ce) {
+          s_sc[c] = scv[u];
+          s_sh[c] = shv[u];
+        }
+      }
+    }
+  };
+  // while the first input tile is in flight: every channel when the CTA runs
+  // all slices of its pixel tiles or more than one item, else its one item's
+  // slice
+  int w_ct = -1;  // slice whose weights are staged (-1: all)
+  if (own || items > (int64_t)gridDim.x) {
+    stage_weights(0, Cp);
+  } else if (cur.item < items) {
+    stage_weights(cur.ct * 64, cur.ct * 64 + 64);
+    w_ct = cur.ct;
+  }
+  __syncthreads();
   for (int sj = 0; cur.item < items; ++sj) {
     const Step nxt = next_step(cur);
     const int buf = NB == 2 ? (sj & 1) : 0;
@@ -667,8 +707,12 @@ __global__ void __launch_bounds__(kTileThreads) dw3_kernel(const DwArgs a_param,
         cp_async_wait<0>();
       }
     } else {
-      stage(cur, 0);
+      if (sj > 0) stage(cur, 0);  // the first step's tile was issued before the weights
       cp_async_wait<0>();
+    }
+    if (w_ct >= 0 && cur.ct != w_ct) {  // one slice staged, another needed (the same for every thread)
+      stage_weights(cur.ct * 64, cur.ct * 64 + 64);
+      w_ct = cur.ct;
     }
     __syncthreads();
     const __nv_bfloat16* s_in = s_in0 + buf * IH * IW * 64;
