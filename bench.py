@@ -157,10 +157,20 @@ def barrier(world: int):
         dist.barrier()
 
 
-def kernel_source_hash():
+# The sources a captured kernel is compiled from: its own file and the shared
+# device headers.  A capture stays valid while these are unchanged.
+KERNEL_SOURCES = {
+    "conv3_kernel_8x56x56x64": ["k_conv3.cu"],
+    "stats_kernel_25088x64": ["k_tiles.cu"],
+    "igemm_kernel_4096x3072x768": ["k_igemm.cu"],
+}
+COMMON_SOURCES = ["sparoa_dev.cuh", "sparoa_kernels.h"]
+
+
+def kernel_source_hash(key: str) -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2511_19457_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
+    for f in COMMON_SOURCES + KERNEL_SOURCES[key]:
         with open(os.path.join(csrc, f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -175,7 +185,7 @@ def ncu_traffic(key: str):
     with open(path) as f:
         d = json.load(f)
     e = d.get(key)
-    if not e or e.get("kernel_source_sha") != kernel_source_hash():
+    if not e or key not in KERNEL_SOURCES or e.get("kernel_source_sha") != kernel_source_hash(key):
         return None
     return e.get("dram_bytes_per_launch")
 
