@@ -45,7 +45,7 @@ extern "C" {
 typedef enum {
     SPAROA_OK = 0,
     SPAROA_ERR_INVALID_ARG = 1,  /* null pointer, bad size, misaligned pointer  */
-    SPAROA_ERR_UNSUPPORTED = 2,  /* valid request this build does not implement */
+    SPAROA_ERR_UNSUPPORTED = 2,  /* valid request the library does not implement */
     SPAROA_ERR_OOM = 3,          /* workspace allocation failed                 */
     SPAROA_ERR_CUDA = 4,         /* a CUDA runtime/driver call failed           */
     SPAROA_ERR_TIMEOUT = 5       /* a kernel's bounded wait ran out             */
