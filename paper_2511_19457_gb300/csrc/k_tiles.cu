@@ -943,47 +943,67 @@ __global__ void __launch_bounds__(kTileThreads)
 }
 
 // ---------------------------------------------------------------------------
+// Global average pooling [N, HW, C] -> [N, C] (C % 8 == 0): one CTA per (image,
+// 64-channel slice).  Lane l of warp w sums pixels 4 w + l / 8 + 32 k of the 8
+// channels 8 (l % 8) .. + 7, so every load of the CTA is in flight at once;
+// the 32 pixel partial sums of a channel meet by shuffles and in shared
+// memory, and threads 0..63 finish one channel each: the mean, its bf16 value
+// and the output occupancy (atomics into the cleared block: row bit, column,
+// tile and total counts, block-column mask words).
 __global__ void __launch_bounds__(kTileThreads)
     avgpool_kernel(const __nv_bfloat16* __restrict__ x, int N, int HW, int C,
                    __nv_bfloat16* __restrict__ y, OccDev o_param, int emit) {
   const OccDev o = o_param;
-  __shared__ uint32_t s_cnt[8 * 64];
-  extern __shared__ uint32_t s_acc[];  // [C] when acc (dynamic)
-  const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
-  const bool acc = emit && C <= kMaxAccCols;
-  acc_init(s_acc, C, acc);
+  __shared__ float s_part[8 * 64];  // [warp][channel of the slice]
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int cg = lane & 7, pq = warp * 4 + (lane >> 3);  // channel group, pixel lane 0..31
+  const int ctn = (C + 63) / 64;
+  const int n = (int)(blockIdx.x / ctn), ct = (int)(blockIdx.x - (blockIdx.x / ctn) * ctn);
+  const int c0 = ct * 64 + cg * 8;
   pdl_wait();
   pdl_trigger();
-  TileEmit e;
-  e.init();
-  SPAROA_TILE_LOOP((int64_t)N, C) {
-    const int64_t row0 = (tile / ctn) * 128;
-    const int col0 = (int)(tile % ctn) * 64;
-    const int c0 = col0 + cg * 8;
-    for (int i = 0; i < 4; ++i) {
-      const int64_t n = row0 + rs + 32 * i;
-      uint32_t mask = 0;
-      if (n < N && c0 < C) {
-        float a8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        const __nv_bfloat16* p = x + n * (int64_t)HW * C + c0;
-#pragma unroll 8
-        for (int q = 0; q < HW; ++q) {  // unrolled: eight pixels' loads in flight
-          float f[8];
-          unpack8(__ldg(reinterpret_cast<const uint4*>(p + (int64_t)q * C)), f);
+  float a8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  if (c0 < C) {
+    const __nv_bfloat16* p = x + (int64_t)n * HW * C + c0;
+    for (int q = pq; q < HW; q += 32) {
+      float f[8];
+      unpack8(__ldg(reinterpret_cast<const uint4*>(p + (int64_t)q * C)), f);
 #pragma unroll
-          for (int j = 0; j < 8; ++j) a8[j] += f[j];
-        }
-#pragma unroll
-        for (int j = 0; j < 8; ++j) a8[j] = a8[j] / (float)HW;
-        const uint4 u = pack8(a8);
-        *reinterpret_cast<uint4*>(y + n * C + c0) = u;
-        mask = nz_mask8(u);
-      }
-      if (emit) e.row(mask, n, col0, o);
+      for (int j = 0; j < 8; ++j) a8[j] += f[j];
     }
-    if (emit) e.tile_done(row0, col0, o, s_cnt, s_acc, acc);
   }
-  if (emit) cta_done(o, s_acc, acc);
+  // lanes cg, cg + 8, cg + 16, cg + 24 of a warp hold the same channels
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    a8[j] += __shfl_xor_sync(0xffffffffu, a8[j], 8);
+    a8[j] += __shfl_xor_sync(0xffffffffu, a8[j], 16);
+  }
+  if (lane < 8) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) s_part[warp * 64 + lane * 8 + j] = a8[j];
+  }
+  __syncthreads();
+  if (threadIdx.x < 64) {  // two full warps
+    const int c = ct * 64 + (int)threadIdx.x;
+    float sum = 0.f;
+#pragma unroll
+    for (int w = 0; w < kTileThreads / 32; ++w) sum += s_part[w * 64 + threadIdx.x];
+    const __nv_bfloat16 b = __float2bfloat16_rn(sum / (float)HW);
+    const bool live = c < C;
+    if (live) y[(int64_t)n * C + c] = b;
+    const bool nz = live && (__bfloat16_as_ushort(b) & 0x7FFFu) != 0u;
+    if (emit) {
+      const uint32_t word = __ballot_sync(0xffffffffu, nz);  // this warp's 32 columns
+      if (nz) atomicAdd(&o.col_nnz[c], 1u);
+      if (lane == 0 && word) {
+        const int w = ct * 2 + (int)(threadIdx.x >> 5);
+        if (w < o.C32) atomicOr(&o.blk_mask[(int64_t)(n >> 7) * o.C32 + w], word);
+        atomicAdd(&o.tile_nnz[ct], (uint32_t)__popc(word));
+        atomicAdd(o.nnz, (unsigned long long)__popc(word));
+        atomicOr(&o.row_bm[(int64_t)n * o.W64 + (ct >> 6)], 1ull << (ct & 63));
+      }
+    }
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -1154,8 +1174,11 @@ cudaError_t launch_maxpool(const __nv_bfloat16* x, int N, int H, int W, int C, i
 cudaError_t launch_avgpool(const __nv_bfloat16* x, int N, int HW, int C, __nv_bfloat16* y,
                            const OccDev& o, int emit, cudaStream_t s) {
   if (N <= 0) return cudaSuccess;
-  return launch_kernel(avgpool_kernel, dim3(tile_grid(N, C)), dim3(kTileThreads), acc_smem(emit, C),
-                       s, x, N, HW, C, y, o, emit);
+  if (C % 8) return cudaErrorInvalidValue;
+  const int64_t ctas = (int64_t)N * ((C + 63) / 64);
+  if (ctas >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;
+  return launch_kernel(avgpool_kernel, dim3((unsigned)ctas), dim3(kTileThreads), 0, s, x, N, HW, C, y, o,
+                       emit);
 }
 
 cudaError_t launch_bn_act(const __nv_bfloat16* x, int64_t R, int C, const EpiDev& ep,
