@@ -1,11 +1,14 @@
-// Memory-bound kernels of the path, all on the same 128-row x 64-channel tile:
-// 256 threads, thread t owns channels [8*(t%8), 8*(t%8)+8) of the tile (one
-// 16-byte vector) in rows t/8 + 32*i, i = 0..3.  Each kernel fuses the
-// occupancy emission of its output (Eq. 1 count and bitmaps, Sec. 3.1) so the
-// next operator's dispatch reads them without another pass over HBM.
+// Memory-bound kernels of the path.  Most work on 128-row x 64-channel tiles
+// with 256 threads, thread t owning channels [8*(t%8), 8*(t%8)+8) of the tile
+// (one 16-byte vector) in rows t/8 + 32*i, i = 0..3; the 3x3 depthwise and the
+// global average pool lay their threads out as their comments say.  Each
+// kernel fuses the occupancy emission of its output (Eq. 1 count and bitmaps,
+// Sec. 3.1) so the next operator's dispatch reads them without another pass
+// over HBM.
 //   stats_kernel    Eq. 1 count and bitmaps of an existing tensor (C % 8 == 0;
 //                   stats_scalar_kernel for other widths)
-//   dwconv_kernel   depthwise k x k convolution + epilogue (MobileNetV2 layers)
+//   dw3_kernel      depthwise 3x3, stride 1 or 2, on 2-D output tiles (MobileNetV2
+//                   layers); dwconv_kernel for other depthwise shapes
 //   maxpool_kernel  k x k max pooling
 //   avgpool_kernel  global average pooling
 //   bn_act_kernel   stand-alone bias / batch norm / residual / activation
