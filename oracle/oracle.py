@@ -12,6 +12,13 @@ rounds every operator output to bf16, the storage type of an activation.
 Tensors are numpy arrays: bf16 values travel as their uint16 bit patterns.
 
 Citations are to sections and equations of the SparOA paper (arXiv 2511.19457).
+
+Pins: every operator is pinned by tests/test_oracle_pins.py and
+tests/test_oracle_vit_pins.py (closed forms, brute force, textbook values,
+Table 2's MAC counts).  ``run_graph``'s chained output is the composition of
+those operators with bf16 rounding between them; networks with random weights
+have no published outputs, so beyond that composition its parity is
+unpinned ("parity unpinned").
 """
 from __future__ import annotations
 
