@@ -5,6 +5,8 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <map>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -14,9 +16,53 @@
 namespace sparoa {
 namespace {
 thread_local bool t_pdl = true;
+
+// Per-device launch facts: SM count, and per kernel the dynamic shared memory
+// it has been opted in to on that device.
+struct DeviceFacts {
+  int sms = 0;
+  std::map<const void*, size_t> optin;
+};
+std::mutex g_facts_mu;
+std::map<int, DeviceFacts> g_facts;
+
+int current_device() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    dev = 0;
+  }
+  return dev;
+}
 }  // namespace
 bool pdl_enabled() { return t_pdl; }
 void set_pdl_enabled(bool on) { t_pdl = on; }
+
+int device_sm_count() {
+  const int dev = current_device();
+  std::lock_guard<std::mutex> lock(g_facts_mu);
+  DeviceFacts& f = g_facts[dev];
+  if (f.sms <= 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) {
+      cudaGetLastError();
+      return 152;  // grid sizing only; not remembered, so the next call asks again
+    }
+    f.sms = n;
+  }
+  return f.sms;
+}
+
+cudaError_t smem_optin(const void* func, size_t bytes) {
+  const int dev = current_device();
+  std::lock_guard<std::mutex> lock(g_facts_mu);
+  size_t& have = g_facts[dev].optin[func];
+  if (bytes <= have) return cudaSuccess;
+  const cudaError_t e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  if (e != cudaSuccess) return e;
+  have = bytes;
+  return cudaSuccess;
+}
 }  // namespace sparoa
 
 using namespace sparoa;

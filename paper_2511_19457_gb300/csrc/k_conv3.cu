@@ -453,12 +453,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 template <int CO>
 cudaError_t launch_co(const CUtensorMap& tX, const CUtensorMap& tW, const IgemmArgs& a,
                       const Conv3Geo& g, int smem, cudaStream_t s) {
-  static int attr = 0;
-  if (smem > attr) {
-    cudaError_t e = cudaFuncSetAttribute(conv3_kernel<CO>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    attr = smem;
-  }
+  cudaError_t e0 = smem_optin(reinterpret_cast<const void*>(conv3_kernel<CO>), (size_t)smem);
+  if (e0 != cudaSuccess) return e0;
   const int tiles = g.N * g.tiles_per_img;
   const int grid = tiles < device_sm_count() ? tiles : device_sm_count();
   cudaError_t e = launch_kernel(conv3_kernel<CO>, dim3(grid), dim3(kThreads), (size_t)smem, s, tX, tW, a, g);

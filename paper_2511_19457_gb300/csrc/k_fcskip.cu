@@ -243,13 +243,10 @@ cudaError_t launch_fcskip(const FcSkipArgs& a, cudaStream_t s) {
   if (a.M <= 0 || a.N <= 0) return cudaSuccess;
   if (a.K % 8 != 0 || a.N % 8 != 0 || a.K > kMaxWin * kKW) return cudaErrorInvalidValue;
   const size_t smem = FcSmem::kBytes + (size_t)a.K * sizeof(short);
-  static size_t attr = 0;
   // opt in above the 48 KB default, which also counts the static shared memory
-  if (smem > 40 * 1024 && smem > attr) {
-    cudaError_t e = cudaFuncSetAttribute(fcskip_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+  if (smem > 40 * 1024) {
+    cudaError_t e = smem_optin(reinterpret_cast<const void*>(fcskip_kernel), smem);
     if (e != cudaSuccess) return e;
-    attr = smem;
   }
   dim3 grid((a.N + kTN - 1) / kTN, (a.M + kTM - 1) / kTM);
   return launch_kernel(fcskip_kernel, grid, dim3(kThreads), smem, s, a);

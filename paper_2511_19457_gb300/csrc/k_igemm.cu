@@ -926,30 +926,13 @@ bool make_tmap_nhwc(CUtensorMap* m, const void* base, int n, int h, int w, int c
   return r == CUDA_SUCCESS;
 }
 
-int num_sms() {
-  static int n = 0;
-  if (!n) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-      n = 152;
-  }
-  return n;
-}
-
 template <int BN, int BK>
 cudaError_t launch_cfg(const IgemmArgs& a, const CUtensorMap& tA, const CUtensorMap& tB,
                        const CUtensorMap& tY, int64_t tiles, cudaStream_t s) {
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(igemm_kernel<BN, BK>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         Cfg<BN, BK>::kSmem);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  cudaError_t e0 = smem_optin(reinterpret_cast<const void*>(igemm_kernel<BN, BK>), (size_t)Cfg<BN, BK>::kSmem);
+  if (e0 != cudaSuccess) return e0;
   const int64_t units = tiles * (a.ksplit > 1 ? a.ksplit : 1);
-  const int64_t grid = units < num_sms() ? units : num_sms();
+  const int64_t grid = units < device_sm_count() ? units : device_sm_count();
   cudaError_t e = launch_kernel(igemm_kernel<BN, BK>, dim3((unsigned)grid), dim3(kThreads),
                                 (size_t)Cfg<BN, BK>::kSmem, s, tA, tB, tY, a);
   if (e != cudaSuccess) return e;
@@ -959,7 +942,6 @@ cudaError_t launch_cfg(const IgemmArgs& a, const CUtensorMap& tA, const CUtensor
 }  // namespace
 
 PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() { return get_encode(); }
-int device_sm_count() { return num_sms(); }
 
 void choose_spatial_tile(IgemmArgs& a) {
   int64_t best = -1;
@@ -1000,7 +982,7 @@ void choose_spatial_tile(IgemmArgs& a) {
 static int k_block(const IgemmArgs& a) { return (a.conv == 2 ? (a.Cp % 64 == 0) : (a.Ktot > 32)) ? 64 : 32; }
 
 void choose_tiles(const IgemmArgs& a, int64_t mtiles, int* bn_out, int* ks_out) {
-  const int sms = num_sms();
+  const int sms = device_sm_count();
   int bn = a.N > 64 ? 128 : 64;
   int64_t tiles = mtiles * ((a.N + bn - 1) / bn);
   if (bn == 128) {

@@ -1151,13 +1151,10 @@ cudaError_t launch_dwconv(const DwArgs& a, cudaStream_t s) {
     const int64_t items = inner ? nsp : ntiles;
     const unsigned grid = (unsigned)(items < cap ? items : cap);
     auto kern = a.stride == 1 ? dw3_kernel<1> : dw3_kernel<2>;
-    static size_t attr1 = 0, attr2 = 0;
-    size_t& attr = a.stride == 1 ? attr1 : attr2;
     // opt in above the 48 KB default, which also counts the static shared memory
-    if (smem > 40 * 1024 && smem > attr) {
-      cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (smem > 40 * 1024) {
+      cudaError_t e = smem_optin(reinterpret_cast<const void*>(kern), smem);
       if (e != cudaSuccess) return e;
-      attr = smem;
     }
     return launch_kernel(kern, dim3(grid), dim3(kTileThreads), smem, s, a, inner);
   }

@@ -370,12 +370,9 @@ template <int HD>
 cudaError_t launch_attention_hd(const __nv_bfloat16* qkv, int N, int T, int heads, __nv_bfloat16* y,
                                 cudaStream_t s) {
   const size_t smem = attention_smem(T, HD);
-  static size_t attr = 0;
-  if (smem > 40 * 1024 && smem > attr) {
-    cudaError_t e = cudaFuncSetAttribute(attention_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+  if (smem > 40 * 1024) {
+    cudaError_t e = smem_optin(reinterpret_cast<const void*>(attention_kernel<HD>), smem);
     if (e != cudaSuccess) return e;
-    attr = smem;
   }
   // split the query tiles while the (image, head) pairs leave resident CTA
   // slots (3 per SM) empty, down to one tile per warp

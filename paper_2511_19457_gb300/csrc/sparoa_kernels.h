@@ -85,8 +85,14 @@ struct IgemmArgs {
 // Picks the N tile and the K split, encodes the tensor maps and launches.
 cudaError_t launch_igemm(const IgemmArgs& a, cudaStream_t s);
 
-// Streaming multiprocessors of the current device (cached per process).
+// Streaming multiprocessors of the current device (cached per device).
 int device_sm_count();
+
+// Opt `func` in to `bytes` of dynamic shared memory on the current device.
+// The attribute belongs to the device, so the largest size set so far is
+// remembered per (device, kernel); the record is guarded by a mutex, so host
+// threads may launch concurrently.
+cudaError_t smem_optin(const void* func, size_t bytes);
 
 // conv = 2: the bw x bh x bn (= 128) output tile with the fewest padded pixels.
 void choose_spatial_tile(IgemmArgs& a);
