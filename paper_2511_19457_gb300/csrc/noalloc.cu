@@ -77,7 +77,7 @@ extern "C" sparoa_status sparoa_gemm_noalloc(void* stream, const void* x, int64_
   auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
   if (!al16(x) || !al16(W) || !al16(y) || (W_kn && !al16(W_kn))) return SPAROA_ERR_INVALID_ARG;
   if (y_dtype != SPAROA_BF16 && y_dtype != SPAROA_F32) return SPAROA_ERR_INVALID_ARG;
-  if (ep && (ep->act < 0 || ep->act > 2 || (ep->residual && !al16(ep->residual))))
+  if (ep && (ep->act < 0 || ep->act > 3 || (ep->residual && !al16(ep->residual))))
     return SPAROA_ERR_INVALID_ARG;
   sparoa_thresholds t;
   if (thr) {
