@@ -31,3 +31,30 @@ def assert_occ_equal(occ_dev: dict, st, what=""):
     assert np.array_equal(occ_dev["tile_nnz"], st.tile_nnz), f"{what}: tile_nnz"
     assert np.array_equal(occ_dev["row_bm"], st.row_bm), f"{what}: row_bm"
     assert np.array_equal(occ_dev["blk_mask"], st.blk_mask), f"{what}: blk_mask"
+
+
+def perturbed_chain_error(ops, x_bits, shape, ref_last_f64, rel=2.0 ** -24, seed=1):
+    """Sensitivity of a graph's chained output to the smallest rounding error
+    any fp32 kernel makes.  The oracle walks the graph again, but every
+    operator's fp64 output is multiplied by (1 + u * rel), u ~ U(-1, 1) per
+    element (rel = 2^-24: at most one fp32 rounding of the result), before
+    the bf16 rounding that stores it.  Returns (max |err| / max |ref|,
+    relative Frobenius error) of that walk's bf16 output against
+    ``ref_last_f64``, the unperturbed walk's fp64 output of the last operator."""
+    from oracle import oracle as orc
+    rng = np.random.default_rng(seed)
+    values = {0: (np.asarray(x_bits), tuple(shape))}
+    last = None
+    for i, op in enumerate(ops):
+        xin, xs = values[op["input"]]
+        res = values[op["residual"]][0] if op.get("residual", -1) >= 0 else None
+        r = orc.run_op(op, xin, xs, res)
+        y = r.out_f64 * (1.0 + rel * rng.uniform(-1.0, 1.0, size=r.out_f64.shape))
+        bits = orc.f64_to_bf16(y).reshape(r.out_shape)
+        values[i + 1] = (bits, r.out_shape)
+        last = bits
+    got = ((np.asarray(last, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32)
+           .astype(np.float64).reshape(-1))
+    ref = np.asarray(ref_last_f64, dtype=np.float64).reshape(-1)
+    err = np.abs(got - ref)
+    return err.max() / np.abs(ref).max(), np.linalg.norm(got - ref) / np.linalg.norm(ref)

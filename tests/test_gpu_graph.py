@@ -4,8 +4,9 @@ Teacher forcing: every operator is checked on exactly the bf16 tensor the GPU
 fed it (its input read back from the library's workspace), so that Eq. 1
 counts, bitmaps and dispatch decisions are compared bit for bit and each
 operator's output within the float tolerance.  The chained run (oracle fed only
-the graph input) is compared at the end with a looser bound, since bf16
-storage rounding at each of 20-50 operator boundaries compounds.
+the graph input) is compared at the end within the float tolerance, or within
+twice the network's own sensitivity to one fp32 rounding per operator where
+that is larger, with decision flips near the sparsity threshold reported.
 """
 import numpy as np
 import pytest
@@ -14,7 +15,7 @@ import torch
 from oracle import oracle as orc
 from paper_2511_19457_gb300 import calibrate as cal
 from paper_2511_19457_gb300 import synth
-from tests._parity import assert_close, assert_occ_equal
+from tests._parity import FRO_REL, MAX_REL, assert_close, assert_occ_equal, perturbed_chain_error
 
 pytestmark = pytest.mark.gpu
 
@@ -95,11 +96,31 @@ def test_graph_batch8_resnet_forced_paths(sp):
 
 @pytest.mark.parametrize("name", ["resnet18", "mobilenet_v2"])
 def test_graph_chained_end_to_end(sp, name):
+    """The oracle fed only the graph input, walking its own values.
+
+    Each operator's output is rounded to bf16 on both sides, so a difference in
+    the last fp32 bit before that rounding can move a stored value by one bf16
+    step, and the network carries it on.  How far that goes is a property of
+    the network, measured here with the oracle alone: its walk with every
+    operator output perturbed by at most one fp32 rounding (2^-24 relative).
+    The device's chained output must be within the path's float tolerance or,
+    where the network's own sensitivity exceeds it, within twice that
+    sensitivity.  Operators whose dispatch decision differs between the two
+    walks (a zero fraction within rounding of s_thr) are reported, not failed
+    on: both paths compute the same operator."""
     ops, xb, shape, recs, outs, occs = _run(sp, name, batch=1)
     ref = orc.run_graph(ops, xb, shape)
+    flips = [i for i, (r, o) in enumerate(zip(recs, ref)) if int(r.stats.path) != o.path]
     got = synth.bits_to_f32(outs[-1][0]).astype(np.float64)
-    # per-op parity is the bar; the chained drift of bf16 storage is bounded loosely
-    assert_close(got, ref[-1].out_f64, max_rel=8e-2, fro_rel=3e-2, what=f"{name} chained logits")
+    want = ref[-1].out_f64.reshape(-1)
+    err = np.abs(got - want)
+    s_max, s_fro = perturbed_chain_error(ops, xb, shape, want)
+    max_rel, fro_rel = max(MAX_REL, 2 * s_max), max(FRO_REL, 2 * s_fro)
+    print(f"{name} chained: max|err|/max|ref| = {err.max() / np.abs(want).max():.3e}, "
+          f"rel Frobenius = {np.linalg.norm(got - want) / np.linalg.norm(want):.3e}; "
+          f"oracle under one fp32 rounding per op: {s_max:.3e}, {s_fro:.3e}; "
+          f"bounds {max_rel:.3e}, {fro_rel:.3e}; decision flips at ops {flips}")
+    assert_close(got, want, max_rel=max_rel, fro_rel=fro_rel, what=f"{name} chained logits")
 
 
 def _mixed_table():
