@@ -55,6 +55,8 @@ def parse_args():
                         "of the committed calibration table")
     p.add_argument("--calib-out", default=None, help="calibrate: write the thresholds table here")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-extras", action="store_true",
+                   help="conv workload: skip the other configurations' sub-records")
     return p.parse_args()
 
 
@@ -257,7 +259,8 @@ def conv_config():
     return {"workload": "conv3x3 s1 p1 NHWC bf16 [8,56,56,64]->64, BN+ReLU epilogue; "
                         "Eq.1 stats + threshold dispatch + next-op occupancy",
             "global_batch": 8, "seq_len": None, "parallelism": "replicas",
-            "thresholds": {"s_thr": 0.5, "c_thr_flops_per_byte": 32.0}}
+            "thresholds": {"s_thr": 0.5, "c_thr_flops_per_byte": 32.0},
+            "l2": f"GPU arm: {NBUF} rotating input/output sets (257 MB > 129 MB L2)"}
 
 
 # ---------------------------------------------------------------------------
@@ -283,6 +286,15 @@ def time_graph(g, replays):
     e1.record()
     torch.cuda.synchronize()
     return e0.elapsed_time(e1)
+
+
+def time_graph_per_replay(g, min_replays=50, min_s=0.2, max_replays=20000):
+    """ms per replay over at least `min_replays` replays and `min_s` seconds
+    (a short probe sizes the run); independent of the bench's --steps."""
+    probe = time_graph(g, 5) / 5
+    reps = max(min_replays, int(math.ceil(min_s * 1e3 / max(probe, 1e-6))))
+    reps = min(reps, max_replays)
+    return time_graph(g, reps) / reps, reps
 
 
 def run_conv(args, rank, local_rank, world, peaks):
@@ -358,14 +370,18 @@ def run_conv(args, rank, local_rank, world, peaks):
     barrier(world)
     ms = max_over_ranks(ms, world, dev)
 
-    # per-kernel durations (same launches, same buffers), measured live
-    reps = max(1, min(200, args.steps // NBUF))
+    # per-kernel durations (same launches, same buffers), measured live over
+    # >= 50 replays and >= 0.2 s whatever --steps is
     g_stats = graph_of(stats, NBUF)
     g_conv = graph_of(conv, NBUF)
     g_stats.replay()
     g_conv.replay()
-    stats_us = time_graph(g_stats, reps) * 1e3 / (reps * NBUF)
-    conv_us = time_graph(g_conv, reps) * 1e3 / (reps * NBUF)
+    clocks.mark()
+    ms_r, stats_reps = time_graph_per_replay(g_stats)
+    stats_us = ms_r * 1e3 / NBUF
+    ms_r, conv_reps = time_graph_per_replay(g_conv)
+    conv_us = ms_r * 1e3 / NBUF
+    clocks.mark()
     clocks.stop()
 
     # end to end through the public API: every step copies its input from pinned
@@ -422,14 +438,15 @@ def run_conv(args, rank, local_rank, world, peaks):
     value = total_flops / (ms * 1e-3) / 1e12
     e2e_value = flops * e2e_steps * world / (e2e_ms * 1e-3) / 1e12
     cfg = conv_config()
-    cfg.update({"path": path, "rho": st.sparsity, "occupied_k_fraction": occ_frac,
-                "l2": f"rotating {NBUF} input/output sets ({NBUF * 2 * R * C * 2 / 1e6:.0f} MB > 129 MB L2)",
-                "cuda_graph": True, "parallelism": f"replicas x{world}"})
+    detail = {"path": path, "rho": st.sparsity, "occupied_k_fraction": occ_frac,
+              "rotating_sets_mb": round(NBUF * 2 * R * C * 2 / 1e6), "cuda_graph": True,
+              "replicas": world, "kernel_timing_replays": {"stats": stats_reps * NBUF,
+                                                           "conv": conv_reps * NBUF}}
     line = {"metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded; stands in for ImageNet activations)", "config": cfg,
-            "roofline": roof, "stats_kernel": stats_kernel,
+            "workload_detail": detail, "roofline": roof, "stats_kernel": stats_kernel,
             "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": R * C * 2,
                     "d2h_bytes_per_step": R * Co * 2, "steps": e2e_steps,
                     "copies": "pinned host <-> device on two side streams, overlapping compute"},
@@ -469,6 +486,216 @@ def conv_occupied_fraction(occ, N, H, W, C, k=3, pad=1):
                 total += any_t.shape[0]
                 occupied += int(any_t[:, (b * 32) // 64].sum())
     return occupied / total if total else 1.0
+
+
+def fc_record(ctx, dev, peaks):
+    """The single FC operator [64, 512] x [512, 512]^T (column-sparse ReLU
+    input, fp32 output): one step = stats + dispatch + the chosen kernel, over
+    rotating input / output sets; the FC call alone (its kernels, no stats)
+    timed separately for its roofline (HBM-bound: occupied weight rows + x + y)."""
+    import torch
+
+    from paper_2511_19457_gb300 import sparoa as sp
+    from paper_2511_19457_gb300 import synth
+    d = synth.fc_layer(seed=0)
+    M, K, N = d["M"], d["K"], d["N"]
+    xs = [sp.bits_to_device(d["x"]).view(M, K).clone() for _ in range(NBUF)]
+    w = sp.bits_to_device(d["w"]).view(N, K)
+    wkn = sp.bits_to_device(d["w_kn"]).view(K, N)
+    bias = torch.from_numpy(d["bias"]).to(dev)
+    ys = [torch.empty(M, N, dtype=torch.float32, device=dev) for _ in range(NBUF)]
+    xo = [sp.OccupancyBuffer(M, K) for _ in range(NBUF)]
+
+    def stats(j):
+        sp.sparoa_op_stats(ctx, xs[j], (M, K), occ=xo[j], host=False)
+
+    def gemm(j):
+        sp.sparoa_gemm(ctx, xs[j], w, ys[j], W_kn=wkn, bias=bias, x_occ=xo[j])
+
+    st = sp.sparoa_gemm(ctx, xs[0], w, ys[0], W_kn=wkn, bias=bias, host=True)
+    for j in range(NBUF):
+        stats(j)
+        gemm(j)
+    g_step = graph_of(lambda j: (stats(j), gemm(j)), NBUF)
+    g_gemm = graph_of(gemm, NBUF)
+    g_step.replay()
+    g_gemm.replay()
+    step_ms, _ = time_graph_per_replay(g_step)
+    gemm_ms, _ = time_graph_per_replay(g_gemm)
+    step_us, gemm_us = step_ms * 1e3 / NBUF, gemm_ms * 1e3 / NBUF
+    kocc = int((xs[0].float().abs().sum(0) != 0).sum().item())
+    flops = 2 * M * K * N
+    alg_bytes = (kocc * N * 2 + M * K * 2 + M * N * 4) if st.path == sp.PATH_SKIP else (N * K + M * K) * 2 + M * N * 4
+    ach = alg_bytes / (gemm_us * 1e-6) / 1e9
+    return {"workload": "fc [64,512]x[512,512]^T fp32 out, ReLU input with whole columns zeroed "
+                        "(p=0.4), s_thr 0.5",
+            "path": PATH_NAME.get(int(st.path)), "rho": st.sparsity, "occupied_k": kocc,
+            "step_us": step_us, "step_tflops": flops / (step_us * 1e-6) / 1e12,
+            "roofline": {"bound": "hbm", "kernel": "sparoa_gemm call (dispatch + chosen FC kernel)",
+                         "kernel_us": gemm_us, "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": ach / peaks["hbm_gbs"], "algorithmic_bytes": alg_bytes,
+                         "note": "weights shared by the rotating sets (L2-resident across calls)"}}
+
+
+def graphs_record(ctx, steps=30):
+    """ResNet-18 at batch 1 / 8 / 32 and MobileNetV2 at batch 1 / 32 through
+    sparoa_run_graph (CUDA graph, L2 flushed before every timed replay)."""
+    out = {}
+    for name, batch in [("resnet18", 1), ("resnet18", 8), ("resnet18", 32),
+                        ("mobilenet_v2", 1), ("mobilenet_v2", 32)]:
+        ms, recs = time_graph_workload(ctx, name, batch, steps, 3)
+        flops = sum(r.stats.flops for r in recs)
+        paths = [int(r.stats.path) for r in recs]
+        out[f"{name}_b{batch}"] = {
+            "images_per_s": batch / (ms * 1e-3), "ms_per_batch": ms,
+            "effective_tflops": flops / (ms * 1e-3) / 1e12,
+            "ops": {"dense": paths.count(1), "zero_skip": paths.count(2), "depthwise": paths.count(3),
+                    "other": paths.count(0)},
+            "decisions": [(int(r.stats.numel), int(r.stats.nnz), float(r.stats.flops_per_byte),
+                           int(r.stats.macs_eq2), int(r.stats.path)) for r in recs]}
+    return out
+
+
+def ops_cfg4_record(ctx, dev, peaks):
+    """Dense tcgen05 path at MobileNetV2's (batch 32) stem, expansion,
+    projection, last pointwise and classifier shapes: the conv / FC call with
+    the dense path forced, input occupancy measured beforehand, rotating
+    input / output sets larger than L2."""
+    import torch
+
+    from paper_2511_19457_gb300 import sparoa as sp
+    gen = torch.Generator(device=dev).manual_seed(1)
+    tc = peaks["bf16_tflops"]
+    rows = []
+    shapes = [("stem 3x3 s2", 32, 224, 224, 3, 32, 3, 2, 1),
+              ("expand 1x1", 32, 56, 56, 24, 144, 1, 1, 0),
+              ("project 1x1", 32, 56, 56, 144, 24, 1, 1, 0),
+              ("expand 1x1", 32, 28, 28, 32, 192, 1, 1, 0),
+              ("project 1x1", 32, 14, 14, 384, 64, 1, 1, 0),
+              ("expand 1x1", 32, 14, 14, 64, 384, 1, 1, 0),
+              ("last 1x1", 32, 7, 7, 320, 1280, 1, 1, 0)]
+    for tag, N, H, W, C, Co, k, s_, p_ in shapes:
+        Ho, Wo = (H + 2 * p_ - k) // s_ + 1, (W + 2 * p_ - k) // s_ + 1
+        in_b = N * H * W * C * 2
+        nb = max(2, min(40, int(3 * 129e6 / (in_b + N * Ho * Wo * Co * 2)) + 1))
+        w = (torch.randn(Co, k, k, C, device=dev, generator=gen) / math.sqrt(k * k * C)).to(torch.bfloat16)
+        xs = []
+        for _ in range(nb):
+            v = torch.randn(N, H, W, C, device=dev, generator=gen).clamp_min_(0.0)
+            xs.append(v.to(torch.bfloat16))
+        ys = [torch.empty(N, Ho, Wo, Co, dtype=torch.bfloat16, device=dev) for _ in range(nb)]
+        xo = [sp.OccupancyBuffer(N * H * W, C) for _ in range(nb)]
+        for j in range(nb):
+            sp.sparoa_op_stats(ctx, xs[j], (N, H, W, C), occ=xo[j], host=False)
+        dense = sp.thresholds(force_path=sp.PATH_DENSE)
+        call = lambda j: sp.sparoa_conv2d(ctx, xs[j], w, ys[j], stride=s_, pad=p_, act=sp.ACT_RELU6,
+                                          thr=dense, x_occ=xo[j])
+        for j in range(nb):
+            call(j)
+        g = graph_of(call, nb)
+        g.replay()
+        ms, _ = time_graph_per_replay(g)
+        us = ms * 1e3 / nb
+        flops = 2.0 * N * Ho * Wo * Co * C * k * k
+        rule = sp.sparoa_conv2d(ctx, xs[0], w, ys[0], stride=s_, pad=p_, act=sp.ACT_RELU6, host=True)
+        ach = flops / (us * 1e-6) / 1e12
+        rows.append({"op": f"{tag} [{N},{H},{W},{C}]->{Co}", "us": round(us, 2), "bound": "tensor",
+                     "achieved": round(ach, 1), "unit": "TFLOP/s", "peak": tc, "frac": round(ach / tc, 4),
+                     "flop_per_byte": round(float(rule.flops_per_byte), 1),
+                     "rule_path": PATH_NAME.get(int(rule.path)), "rotating_sets": nb})
+        del xs, ys, xo, g
+        torch.cuda.empty_cache()
+    return rows
+
+
+def mlp_sweep_record(ctx, dev, rhos=None, structures=("unstructured", "block32", "token")):
+    """The MLP down projection h [M, 3072] x W2 [768, 3072]^T at M in {256,
+    1024, 4096}: forced-dense and forced-zero-skip time per zero fraction rho
+    and zero structure, the crossover rho (the smallest rho from which
+    zero-skip is faster at every larger rho of the grid), and what the rule
+    (s_thr 0.5, c_thr 32) picks on the measured count.  Each point's input is
+    drawn once (seeded) and copied into rotating sets larger than L2."""
+    import torch
+
+    from paper_2511_19457_gb300 import sparoa as sp
+    from paper_2511_19457_gb300 import synth
+    wts = synth.mlp_weights(seed=0)
+    w2 = sp.bits_to_device(wts["w2"]).view(768, 3072)
+    rhos = rhos or [round(0.05 * i, 2) for i in range(20)]
+    table, cross = [], {}
+    for M in (256, 1024, 4096):
+        nb = max(2, int(3 * 129e6 / (M * 3072 * 2 + M * 768 * 2)) + 1)
+        ys = [torch.empty(M, 768, dtype=torch.bfloat16, device=dev) for _ in range(nb)]
+        for structure in structures:
+            wins = []
+            for rho in rhos:
+                h0 = sp.bits_to_device(synth.mlp_hidden(M, rho, structure, seed=M)).view(M, 3072)
+                hs = [h0] + [h0.clone() for _ in range(nb - 1)]
+                occ = [sp.OccupancyBuffer(M, 3072) for _ in range(nb)]
+                for j in range(nb):
+                    sp.sparoa_op_stats(ctx, hs[j], (M, 3072), occ=occ[j], host=False)
+                times = {}
+                for force in (1, 2):
+                    thr = sp.thresholds(force_path=force)
+                    g = graph_of(lambda j: sp.sparoa_gemm(ctx, hs[j], w2, ys[j], thr=thr, x_occ=occ[j]), nb)
+                    g.replay()
+                    ms, _ = time_graph_per_replay(g, min_replays=10, min_s=0.02)
+                    times[force] = ms * 1e3 / nb
+                rule = sp.sparoa_gemm(ctx, hs[0], w2, ys[0], x_occ=occ[0], host=True)
+                table.append({"M": M, "structure": structure, "rho": rho, "nnz": int(rule.nnz),
+                              "dense_us": round(times[1], 2), "skip_us": round(times[2], 2),
+                              "rule_path": PATH_NAME.get(int(rule.path))})
+                wins.append(times[2] < times[1])
+                del hs, occ
+            crossover = None
+            for i in range(len(rhos) - 1, -1, -1):
+                if not wins[i]:
+                    break
+                crossover = rhos[i]
+            cross[f"M{M}_{structure}"] = crossover
+        del ys
+        torch.cuda.empty_cache()
+    return {"workload": "MLP down projection [M,3072]x[768,3072]^T, bf16, M in {256,1024,4096}",
+            "crossover_rho": cross, "rule": {"s_thr": 0.5, "c_thr": 32.0, "flop_per_byte": 768.0},
+            "table": table}
+
+
+def other_configs(ctx, dev, peaks):
+    """The other configurations of the metric, as sub-records of the default
+    line: the FC operator, the two CNNs at batch 1 / 8 / 32, MobileNetV2's
+    dense-path shapes and the MLP sparsity sweep."""
+    out = {}
+    for key, fn in [("fc", lambda: fc_record(ctx, dev, peaks)),
+                    ("graphs", lambda: graphs_record(ctx)),
+                    ("mobilenet_v2_dense_ops", lambda: ops_cfg4_record(ctx, dev, peaks)),
+                    ("mlp_sweep", lambda: mlp_sweep_record(ctx, dev))]:
+        t0 = time.perf_counter()
+        try:
+            out[key] = fn()
+        except Exception as e:  # a failed sub-record must not lose the headline line
+            out[key] = {"error": f"{type(e).__name__}: {e}"}
+        out.setdefault("seconds", {})[key] = round(time.perf_counter() - t0, 1)
+    return out
+
+
+def oracle_rule_check(extra):
+    """The oracle's threshold rule on the counts the device measured (the
+    CPU-baseline leg): agreement of every recorded dispatch decision."""
+    from oracle import oracle as orc
+    n = agree = 0
+    sweep = extra.get("mlp_sweep", {})
+    for row in sweep.get("table", []):
+        want = orc.decide(row["M"] * 3072, row["nnz"], 768.0, 3072 * 768, 0.5, 32.0)
+        n += 1
+        agree += int(PATH_NAME.get(want) == row["rule_path"])
+    for rec in extra.get("graphs", {}).values():
+        if not isinstance(rec, dict):
+            continue
+        for numel, nnz, fpb, macs, path in rec.get("decisions", []):
+            if path in (1, 2):
+                n += 1
+                agree += int(orc.decide(numel, nnz, fpb, macs, 0.5, 32.0) == path)
+    return {"decisions_checked": n, "agree": agree}
 
 
 def run_fc(args, rank, local_rank, world, peaks):
@@ -946,8 +1173,21 @@ def main():
     peaks = measured_peaks()
     if args.workload == "conv":
         line = run_conv(args, rank, local_rank, world, peaks)
+        if world == 1 and not args.no_extras:
+            import torch
+
+            from paper_2511_19457_gb300 import sparoa as sp
+            ctx = sp.Context(local_rank)
+            line["other_configs"] = other_configs(ctx, torch.device("cuda", local_rank), peaks)
+            ctx.close()
         if rank == 0 and not args.no_cpu_baseline:
             line["cpu_baseline"] = cpu_baseline_conv()
+            if "other_configs" in line:
+                line["cpu_baseline"]["oracle_rule_check"] = oracle_rule_check(line["other_configs"])
+        if "other_configs" in line:
+            for rec in line["other_configs"].get("graphs", {}).values():
+                if isinstance(rec, dict):
+                    rec.pop("decisions", None)
     elif args.workload in ("resnet18", "mobilenet_v2", "vit_b16"):
         line = run_graph_workload(args, rank, local_rank, world, peaks, args.workload)
     elif args.workload == "fc":
