@@ -240,6 +240,46 @@ sparoa_status occ_clear(sparoa_ctx* ctx, const sparoa_occupancy& o, bool rows_wh
   return SPAROA_OK;
 }
 
+// Word ranges that clear an occupancy block (rows_whole: all but the row
+// bitmaps).  A block carved by sparoa_occupancy_init is contiguous and takes
+// one range (two with rows_whole); any other block one range per field.
+void occ_ranges(const sparoa_occupancy& o, bool rows_whole, std::vector<std::pair<uint32_t*, int64_t>>* out) {
+  const OccLayout l = occ_layout(o.R, o.C);
+  char* base = reinterpret_cast<char*>(o.nnz);
+  const int64_t T = (o.C + 63) / 64, W64 = (T + 63) / 64, RB = (o.R + 127) / 128, C32 = (o.C + 31) / 32;
+  const bool contiguous = reinterpret_cast<char*>(o.col_nnz) == base + l.col &&
+                          reinterpret_cast<char*>(o.tile_nnz) == base + l.tile &&
+                          reinterpret_cast<char*>(o.row_bm) == base + l.row &&
+                          reinterpret_cast<char*>(o.blk_mask) == base + l.blk;
+  if (contiguous) {
+    if (rows_whole) {
+      out->push_back({reinterpret_cast<uint32_t*>(base), (int64_t)(l.row / 4)});
+      out->push_back({o.blk_mask, (int64_t)((l.total - l.blk) / 4)});
+    } else {
+      out->push_back({reinterpret_cast<uint32_t*>(base), (int64_t)(l.total / 4)});
+    }
+    return;
+  }
+  out->push_back({reinterpret_cast<uint32_t*>(o.nnz), 2});
+  out->push_back({o.col_nnz, o.C});
+  out->push_back({o.tile_nnz, T});
+  if (!rows_whole) out->push_back({reinterpret_cast<uint32_t*>(o.row_bm), 2 * o.R * W64});
+  out->push_back({o.blk_mask, RB * C32});
+}
+
+// Clear the given word ranges, five per launch.
+sparoa_status clear_ranges(sparoa_ctx* ctx, const std::vector<std::pair<uint32_t*, int64_t>>& rg) {
+  for (size_t i = 0; i < rg.size(); i += 5) {
+    ClearArgs a = {};
+    for (size_t k = 0; k < 5 && i + k < rg.size(); ++k) {
+      a.p[k] = rg[i + k].first;
+      a.words[k] = rg[i + k].second;
+    }
+    SP_CUDA(launch_clear(a, ctx->stream));
+  }
+  return SPAROA_OK;
+}
+
 // Split-K scratch offered to the implicit-GEMM kernel: 65536 arrival counters
 // (zeroed once when allocated; every launch leaves them zero) and 64 MiB of
 // fp32 partial tiles.  Allocated with the context.
@@ -866,11 +906,21 @@ sparoa_status sparoa_conv2d(sparoa_ctx* ctx, const void* x, int64_t N, int64_t H
   const Work wk = conv_work(N, H, W, C_in, C_out, kh, kw, Ho, Wo, groups);
   sparoa_occupancy xo;
   const bool need_x_occ = !depthwise || host_out;
-  if (need_x_occ) {
-    if (x_occ) xo = *x_occ;
-    else if (N > 0) SP_TRY(measure(ctx, x, N * H * W, C_in, &xo));
+  if (need_x_occ && !x_occ && N > 0) {
+    // the input's occupancy is measured into context scratch: one clear
+    // launch for it and the output's block, then the statistics
+    const int64_t R = N * H * W;
+    SP_TRY(ensure(ctx, ctx->occ, occ_layout(R, C_in).total));
+    occ_carve(ctx->occ.p, R, C_in, &xo);
+    std::vector<std::pair<uint32_t*, int64_t>> rg;
+    occ_ranges(xo, stats_writes_rows_whole(R, (int)C_in), &rg);
+    if (y_occ) occ_ranges(*y_occ, false, &rg);
+    SP_TRY(clear_ranges(ctx, rg));
+    SP_CUDA(launch_stats(static_cast<const __nv_bfloat16*>(x), R, (int)C_in, to_dev(xo), ctx->stream));
+  } else {
+    if (need_x_occ && x_occ) xo = *x_occ;
+    if (y_occ) SP_TRY(occ_clear(ctx, *y_occ));
   }
-  if (y_occ) SP_TRY(occ_clear(ctx, *y_occ));
   if (N > 0) {
     if (depthwise) {
       DwArgs a;

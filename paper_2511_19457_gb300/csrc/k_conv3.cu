@@ -14,19 +14,20 @@
 // start address moved by (r * Wp + s) whole rows (the swizzle is a function of
 // the absolute shared-memory address, so a row-aligned move keeps it).  All
 // 9 taps x C/16 MMAs of a tile read one slab; the weights [tap][channel block]
-// [C_out][64] (same layout) are loaded once per CTA.  Compared with gathering A per (tap, channel block), the shared-memory
-// traffic per tile drops about tenfold.
+// [C_out][64] (same layout) are loaded once per CTA.
 //
 // Dispatch and zero skipping as in the implicit-GEMM kernel (Sec. 3 rule
 // evaluated on the device; Sec. 2.1 zero-valued products skipped): on the
-// zero-skip path the producers OR the input row bitmaps of each tap's 128
-// shifted pixels, and the MMA warp leaves out the (tap, 64-channel tile) MMAs
-// whose activations are all zero.  Epilogue: bias / batch norm / residual /
-// activation, bf16 store, output occupancy.
+// zero-skip path one warp reads the input's 128-row block-column masks over
+// the whole input rows each tap row of a tile touches, and the MMA warp
+// leaves out the taps of a tap row whose activations are all zero there.
+// Epilogue: bias / batch norm / residual / activation, bf16 store, output
+// occupancy (column counts kept in registers across tiles, row flags of the
+// two column halves combined at one 64-thread barrier per lane quarter).
 //
-// Warp roles (416 threads, persistent CTAs): warps 0-3 producers (thread 0
-// issues TMA; all compute skip masks), warps 4-11 epilogue (two per TMEM lane
-// quarter, 32 columns each), warp 12 MMA.
+// Warp roles (416 threads, persistent CTAs): warp 0 lane 0 issues the slab
+// TMA loads, warp 1 computes the skip masks, warps 4-11 epilogue (two per TMEM
+// lane quarter, 32 columns each), warp 12 MMA.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -43,20 +44,17 @@ namespace {
 // of the 3x3 window must fit: R * Wp >= (Wp - 1) + 2 * Wp + 2 + 128.
 int slab_rows(int Wp) { return 3 + (129 + Wp - 1) / Wp; }
 int block_stride(int Wp) { return (128 * Wp * slab_rows(Wp) + 1023) / 1024 * 1024; }
+constexpr int kCtlBytes = 2048;  // barriers, flags, masks, row flags, column affine and counts
 int conv3_smem(int C, int Co, int W) {
-  const int ctl = 512 + 2 * Co * 4 + 4 * Co * 4 + Co * 4 + 16 + 1024 * 8;
-  return 9 * C * Co * 2 + 2 * (C / 64) * block_stride(W + 2) + ctl + 1024;
+  return 9 * C * Co * 2 + 2 * (C / 64) * block_stride(W + 2) + kCtlBytes + 1024;
 }
-}  // namespace
-
-namespace {
 
 constexpr int kEpiWarps = 8;                      // two per TMEM lane quarter, 32 columns each
 constexpr int kEpiThreads = 32 * kEpiWarps;
 constexpr int kMmaWarp = 4 + kEpiWarps;
 constexpr int kThreads = 32 * (kMmaWarp + 1);     // 4 producer warps, epilogue warps, MMA warp
 constexpr int kBM = 128;
-constexpr int kMaxPos = 1024;  // slab positions for the skip masks
+constexpr int kMaxPos = 1024;  // slab positions (bounds the slab size)
 
 struct Conv3Geo {
   int N, H, W, C, Co, Wp, R, tiles_per_img, chunk_stride, slab_bytes, w_bytes;
@@ -79,6 +77,104 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const void* tmap, uint
       : "memory");
 }
 
+// Two fp32 values to a bf16 pair (round to nearest even), `lo` in the low
+// half; with relu, negative results become zero in the same instruction.
+template <bool RELU>
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  uint32_t d;
+  if (RELU)
+    asm("cvt.rn.relu.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  else
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  return d;
+}
+
+// Bits 0 and 1 of the result: the low / high bf16 of w is non-zero (not +-0).
+__device__ __forceinline__ uint32_t nz_pair(uint32_t w) {
+  const uint32_t t = ((w & 0x7FFF7FFFu) + 0x7FFF7FFFu) & 0x80008000u;
+  return ((t >> 15) & 1u) | (t >> 30);
+}
+
+// Occupied tap rows of tile t (zero-skip path), from the input's 128-row
+// block-column masks: tap row r of the tile reads input rows
+// [oh_first + r - 1, oh_last + r - 1] of its image, and is occupied unless
+// every 128-row block covering those whole rows is all zero in all channels.
+// Executed by one whole warp; returns the 9-bit tap mask (bit 3 r + s).
+__device__ __forceinline__ uint32_t conv3_tap_mask(const Conv3Geo& G, const uint32_t* in_blk, int in_C32,
+                                                   int t, int lane) {
+  const int img = t / G.tiles_per_img;
+  const int q0 = (t - img * G.tiles_per_img) * kBM;
+  const int oh_first = q0 / G.Wp;
+  int oh_last = (q0 + kBM - 1) / G.Wp;
+  if (oh_last > G.H - 1) oh_last = G.H - 1;
+  const int64_t base = (int64_t)img * G.H * G.W;
+  const int lo_row = oh_first - 1 < 0 ? 0 : oh_first - 1;
+  const int hi_row = oh_last + 1 > G.H - 1 ? G.H - 1 : oh_last + 1;
+  const int64_t B_lo = (base + (int64_t)lo_row * G.W) >> 7;
+  const int64_t B_hi = (base + (int64_t)hi_row * G.W + G.W - 1) >> 7;
+  const int nb = (int)(B_hi - B_lo + 1);
+  if (nb > 32) return 0x1FFu;  // wider than one warp's reach: keep every tap
+  bool nz = false;
+  if (lane < nb) {
+    const uint32_t* wd = in_blk + (B_lo + lane) * in_C32;
+    for (int k = 0; k < in_C32; ++k) nz |= wd[k] != 0u;
+  }
+  const uint32_t occ = __ballot_sync(0xffffffffu, nz);
+  uint32_t mask = 0u;
+#pragma unroll
+  for (int r = 0; r < 3; ++r) {
+    const int ih_lo = oh_first + r - 1 < 0 ? 0 : oh_first + r - 1;
+    const int ih_hi = oh_last + r - 1 > G.H - 1 ? G.H - 1 : oh_last + r - 1;
+    if (ih_lo > ih_hi) continue;
+    const int b0 = (int)(((base + (int64_t)ih_lo * G.W) >> 7) - B_lo);
+    const int b1 = (int)(((base + (int64_t)ih_hi * G.W + G.W - 1) >> 7) - B_lo);
+    const uint32_t span = (b1 - b0 + 1 >= 32) ? 0xffffffffu : ((1u << (b1 - b0 + 1)) - 1u);
+    if ((occ >> b0) & span) mask |= 7u << (3 * r);
+  }
+  return mask;
+}
+
+// The per-tile MMAs: 9 taps x 4 k-steps of 128 x CO x 16, the A operand the
+// slab shifted by the tap's row offset.  `tapmask` leaves out taps whose
+// activations are all zero; accumulate flags are compile-time constants (the
+// first issued MMA of the tile is peeled).
+template <int CO>
+__device__ __forceinline__ void conv3_issue(uint32_t d, uint64_t adesc0, uint64_t bdesc0, int Wp, uint32_t tapmask) {
+  constexpr uint32_t idesc = idesc_bf16_f32(kBM, CO);
+  if (tapmask == 0x1FFu) {
+    tc_mma_bf16(d, adesc0, bdesc0, idesc, 0u);
+#pragma unroll
+    for (int i = 1; i < 36; ++i) {
+      const int tap = i >> 2, ks = i & 3;
+      tc_mma_bf16(d, adesc0 + (uint64_t)((((tap / 3) * Wp + (tap % 3)) * 128) >> 4) + (uint64_t)(2 * ks),
+                  bdesc0 + (uint64_t)((tap * CO * 128) >> 4) + (uint64_t)(2 * ks), idesc, 1u);
+    }
+    return;
+  }
+  if (tapmask == 0u) {
+    // no occupied tap: tap 0's activations are all zero, so one
+    // non-accumulating MMA on them writes the zero accumulator
+    tc_mma_bf16(d, adesc0, bdesc0, idesc, 0u);
+    return;
+  }
+  const int ftap = __ffs((int)tapmask) - 1;
+  {
+    const uint64_t ad = adesc0 + (uint64_t)((((ftap / 3) * Wp + (ftap % 3)) * 128) >> 4);
+    const uint64_t bd = bdesc0 + (uint64_t)((ftap * CO * 128) >> 4);
+    tc_mma_bf16(d, ad, bd, idesc, 0u);
+#pragma unroll
+    for (int ks = 1; ks < 4; ++ks) tc_mma_bf16(d, ad + (uint64_t)(2 * ks), bd + (uint64_t)(2 * ks), idesc, 1u);
+  }
+#pragma unroll
+  for (int tap = 1; tap < 9; ++tap) {
+    if (tap <= ftap || !((tapmask >> tap) & 1u)) continue;
+    const uint64_t ad = adesc0 + (uint64_t)((((tap / 3) * Wp + (tap % 3)) * 128) >> 4);
+    const uint64_t bd = bdesc0 + (uint64_t)((tap * CO * 128) >> 4);
+#pragma unroll
+    for (int ks = 0; ks < 4; ++ks) tc_mma_bf16(d, ad + (uint64_t)(2 * ks), bd + (uint64_t)(2 * ks), idesc, 1u);
+  }
+}
+
 template <int CO>
 __global__ void __launch_bounds__(kThreads, 1)
     conv3_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
@@ -91,30 +187,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t sSlab = sW + (uint32_t)G.w_bytes;      // 2 slabs
   uint8_t* ctl = smem + G.w_bytes + 2 * G.slab_bytes;
   const uint32_t sCtl = sSlab + 2u * (uint32_t)G.slab_bytes;
-  // control block: bars(8 each): w, slab_full[2], slab_empty[2], accf[2], acce[2]
+  // control block: mbarriers (8 bytes each) w (+ 8 spare), full[2], empty[2], accf[2],
+  // acce[2], mask[2]; then flags, masks, row flags, column affine and counts
   const uint32_t bar_w = sCtl;
-  const uint32_t bar_full = sCtl + 8;
-  const uint32_t bar_empty = sCtl + 24;
-  const uint32_t bar_accf = sCtl + 40;
-  const uint32_t bar_acce = sCtl + 56;
-  const uint32_t bar_mask = sCtl + 80;  // [2] zero-skip: the 128 mask threads of a slab's tile are done
-  volatile int* s_abort = reinterpret_cast<volatile int*>(ctl + 72);
-  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(ctl + 76);
-  uint32_t* s_tapm = reinterpret_cast<uint32_t*>(ctl + 128);  // [3] 9-bit occupied-tap masks
-  float* s_scale = reinterpret_cast<float*>(ctl + 512);                          // [CO]
-  float* s_shift = s_scale + CO;                                                 // [CO]
-  uint32_t* s_cnt = reinterpret_cast<uint32_t*>(s_shift + CO);                   // [4][CO]
-  uint32_t* s_acc = s_cnt + 4 * CO;                                              // [CO]
-  uint8_t* s_pos = reinterpret_cast<uint8_t*>(s_acc + CO);  // [kMaxPos] 1 = input pixel has a non-zero
-  unsigned long long* s_rowbm = reinterpret_cast<unsigned long long*>(s_pos + kMaxPos);  // [128]
+  const uint32_t bar_full = sCtl + 72;
+  const uint32_t bar_empty = sCtl + 88;
+  const uint32_t bar_accf = sCtl + 104;
+  const uint32_t bar_acce = sCtl + 120;
+  const uint32_t bar_mask = sCtl + 136;
+  volatile int* s_abort = reinterpret_cast<volatile int*>(ctl + 152);
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(ctl + 156);
+  uint32_t* s_tapm = reinterpret_cast<uint32_t*>(ctl + 160);          // [2] 9-bit occupied-tap masks
+  uint8_t* s_rowf = ctl + 256;                                         // [3][2][128] row has a non-zero
+  float* s_scale = reinterpret_cast<float*>(ctl + 1024);              // [CO]
+  float* s_shift = s_scale + CO;                                       // [CO]
+  uint32_t* s_acc = reinterpret_cast<uint32_t*>(s_shift + CO);         // [CO] non-zeros per column
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int N = G.N, H = G.H, W = G.W, C = G.C, Wp = G.Wp;
   const int tiles = N * G.tiles_per_img;
-  const int act = P.ep.act;
-  const __nv_bfloat16* const residual = P.ep.residual;
-  const unsigned long long* const in_rowbm = P.in_rowbm;
-  const int in_W64 = P.in_W64;
   uint32_t* const err = P.err;
   const int emit = P.emit;
 
@@ -123,7 +214,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(bar_w, 1u);
     for (int b = 0; b < 2; ++b) {
       mbar_init(bar_full + 8 * b, 1u);
-      mbar_init(bar_mask + 8 * b, 128u);
+      mbar_init(bar_mask + 8 * b, 1u);
       mbar_init(bar_empty + 8 * b, 1u);
       mbar_init(bar_accf + 8 * b, 1u);
       mbar_init(bar_acce + 8 * b, (uint32_t)kEpiThreads);
@@ -134,6 +225,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tmap(&tmW);
   }
   if (warp == kMmaWarp) tmem_alloc(smem_u32(s_tmem), (uint32_t)(2 * CO));
+  if (warp >= 4 && warp < kMmaWarp)
+    for (int c = threadIdx.x - 128; c < CO; c += kEpiThreads) s_acc[c] = 0u;
   // the first tile's slab origin (arithmetic on the parameters only)
   const int t_first = blockIdx.x;
   const int img_first = t_first / G.tiles_per_img;
@@ -141,175 +234,107 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_wait();
   pdl_trigger();
   if (threadIdx.x == 0 && t_first < tiles) {
-    // The first slab and the weights go out before anything else: the slab
-    // comes from HBM and gates the first MMAs.  Either path needs them.
+    // The weights (the same 72 KB for every CTA, from L2) go out first, then
+    // the first tile's slab.
+    mbar_arrive_expect_tx(bar_w, (uint32_t)(9 * (C / 64) * CO * 128));
+    for (int tap = 0; tap < 9; ++tap)
+      for (int cb = 0; cb < C / 64; ++cb)
+        tma_load_3d(sW + (uint32_t)((tap * (C / 64) + cb) * CO * 128), &tmW, bar_w, cb * 64, tap, 0);
     mbar_arrive_expect_tx(bar_full, (uint32_t)(C / 64 * 128 * Wp * G.R));
     for (int cb = 0; cb < C / 64; ++cb)
       tma_load_4d(sSlab + (uint32_t)(cb * G.chunk_stride), &tmX, bar_full, cb * 64, -1, oh0_first - 1,
                   img_first);
-    mbar_arrive_expect_tx(bar_w, (uint32_t)G.w_bytes);
-    for (int tap = 0; tap < 9; ++tap)
-      for (int cb = 0; cb < C / 64; ++cb)
-        tma_load_3d(sW + (uint32_t)((tap * (C / 64) + cb) * CO * 128), &tmW, bar_w, cb * 64, tap, 0);
   }
   const int path = decide_path(P.disp);
   record_path(P.disp, path);
   const bool skip = path == 2;
-  if (warp >= 4 && warp < kMmaWarp) {
-    const int et = threadIdx.x - 128;
-    for (int c = et; c < CO; c += kEpiThreads) s_acc[c] = 0u;
-    for (int i = et; i < kBM; i += kEpiThreads) s_rowbm[i] = 0ull;
-  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *s_tmem;
 
-  if (warp < 4) {
-    // -------------------------------------------------------------- producers
-    const int t_ = threadIdx.x;
-    int j = 0;
-    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++j) {
-      if (!skip && warp != 0) break;  // dense path: warp 0 walks the tiles, lane 0 streams the slabs
-      const int b = j & 1;
-      const int mb = j % 3;  // mask buffer: the MMAs of tile j - 3 are issued by now
-      const int img = t / G.tiles_per_img;
-      const int q0 = (t - img * G.tiles_per_img) * kBM;
-      const int oh0 = q0 / Wp;
-      // the slab first, so that its load overlaps the mask computation below
-      bool ok = true;
-      if (t_ == 0 && j > 0) {  // the first slab went out with the weights
-        ok = mbar_wait(bar_empty + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutEmpty);
-        if (ok) {
-          const uint32_t dst = sSlab + (uint32_t)(b * G.slab_bytes);
-          mbar_arrive_expect_tx(bar_full + 8 * b, (uint32_t)(C / 64 * 128 * Wp * G.R));
-          for (int cb = 0; cb < C / 64; ++cb)
-            tma_load_4d(dst + (uint32_t)(cb * G.chunk_stride), &tmX, bar_full + 8 * b, cb * 64, -1,
-                        oh0 - 1, img);
+  if (warp == 0) {
+    // -------------------------------------------------------------- slab loads
+    if (lane == 0) {
+      int j = 1;
+      for (int t = blockIdx.x + gridDim.x; t < tiles; t += gridDim.x, ++j) {
+        const int b = j & 1;
+        if (!mbar_wait(bar_empty + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutEmpty))
+          break;
+        const int img = t / G.tiles_per_img;
+        const int oh0 = (t - img * G.tiles_per_img) * kBM / Wp;
+        const uint32_t dst = sSlab + (uint32_t)(b * G.slab_bytes);
+        mbar_arrive_expect_tx(bar_full + 8 * b, (uint32_t)(C / 64 * 128 * Wp * G.R));
+        for (int cb = 0; cb < C / 64; ++cb)
+          tma_load_4d(dst + (uint32_t)(cb * G.chunk_stride), &tmX, bar_full + 8 * b, cb * 64, -1, oh0 - 1, img);
+      }
+    }
+  } else if (warp == 1) {
+    // -------------------------------------------------------------- skip masks
+    if (skip) {
+      int j = 0;
+      for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++j) {
+        const int b = j & 1;
+        bool ok = true;
+        // mask buffer b was read by the MMA issue of tile j - 2, before that
+        // tile's commit to the slab-empty barrier
+        if (lane == 0 && j >= 2)
+          ok = mbar_wait(bar_empty + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutEmpty);
+        if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) break;
+        const uint32_t m = conv3_tap_mask(G, P.in_blk, P.in_C32, t, lane);
+        if (lane == 0) {
+          s_tapm[b] = m;
+          mbar_arrive(bar_mask + 8 * b);
         }
       }
-      if (skip) {
-        // zero-skip masks of this tile: per tap, OR of the row bitmaps of the
-        // tile's 128 shifted pixels (the mask buffer of tile j - 3 is free: the
-        // empty-slot wait of tile j - 1 saw those MMAs complete)
-        // One 64-channel block (C == 64): a pixel's row bitmap word is its bit 0.
-        // All of this thread's bitmap loads are issued before any is used.
-        const int npos = G.R * Wp < kMaxPos ? G.R * Wp : kMaxPos;
-        uint32_t nzb = 0u;  // bit k: slab position t_ + 128 k is a non-zero pixel
-#pragma unroll
-        for (int k = 0; k < kMaxPos / 128; ++k) {
-          const int pp = t_ + 128 * k;
-          const int prr = pp / Wp;
-          const int pr = oh0 - 1 + prr, pc = pp - prr * Wp - 1;  // input pixel of slab position pp
-          unsigned long long w = 0ull;
-          if (pp < npos && pr >= 0 && pr < H && pc >= 0 && pc < W)
-            w = in_rowbm[(((int64_t)img * H + pr) * W + pc) * in_W64];
-          nzb |= (uint32_t)(w & 1ull) << k;
-        }
-#pragma unroll
-        for (int k = 0; k < kMaxPos / 128; ++k)
-          if (t_ + 128 * k < npos) s_pos[t_ + 128 * k] = (uint8_t)((nzb >> k) & 1u);
-        if (t_ == 0) s_tapm[mb] = 0u;
-        named_bar_sync(1, 128);
-        const int qoff = q0 - oh0 * Wp;
-        const bool rvalid = q0 + t_ < H * Wp;
-        uint32_t tb = 0u;  // bit tap: this output position reads a non-zero pixel under that tap
-#pragma unroll
-        for (int tap = 0; tap < 9; ++tap) {
-          const int pp = qoff + t_ + (tap / 3) * Wp + (tap % 3);
-          if (rvalid && pp < kMaxPos && s_pos[pp]) tb |= 1u << tap;
-        }
-        tb = __reduce_or_sync(0xffffffffu, tb);
-        if (lane == 0 && tb) atomicOr(&s_tapm[mb], tb);
-      }
-      if (!skip) {
-        if (__shfl_sync(0xffffffffu, ok ? 1 : 0, 0) == 0) break;
-        continue;
-      }
-      // all masks written (and s_pos free for the next tile); uniform abort decision
-      if (named_bar_or(1, 128, !ok)) break;
-      mbar_arrive(bar_mask + 8 * b);  // this tile's masks are written
     }
   } else if (warp == kMmaWarp) {
     // -------------------------------------------------------------- MMA issue
-    // The whole warp walks the tiles so that it stays converged between tiles;
-    // lane 0 waits, issues the MMAs and commits.
-    constexpr uint32_t idesc = idesc_bf16_f32(kBM, CO);
-    bool ok = true;
-    if (lane == 0) ok = mbar_wait(bar_w, 0u, err, s_abort, kErrTimeoutFull);
-    ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-    tc_fence_after();
-    int j = 0;
-    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++j) {
-      const int b = j & 1;
-      if (lane == 0) {
-        ok = mbar_wait(bar_acce + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutAcc) &&
-             mbar_wait(bar_full + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutFull) &&
-             (!skip || mbar_wait(bar_mask + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutFull));
-      }
-      if (lane == 0 && ok) {
+    if (lane == 0) {
+      int j = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++j) {
+        const int b = j & 1;
+        ok = mbar_wait_spin(bar_acce + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutAcc) &&
+             mbar_wait_spin(bar_full + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutFull) &&
+             (!skip || mbar_wait_spin(bar_mask + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutFull));
+        if (!ok) break;
+        tc_fence_after();
         const int q0 = (t - (t / G.tiles_per_img) * G.tiles_per_img) * kBM;
         const int qoff = q0 - (q0 / Wp) * Wp;
-        tc_fence_after();
         const uint32_t d = tmem + (uint32_t)(b * CO);
         const uint32_t slab = sSlab + (uint32_t)(b * G.slab_bytes);
-        // descriptors of tap 0 / channel block 0 / k-step 0; the others differ only
-        // in the start-address field (byte offset >> 4), which never carries out
+        // descriptors of tap 0 / k-step 0; the others differ only in the
+        // start-address field (byte offset >> 4), which never carries out
         const uint64_t adesc0 = smem_desc_kmajor<64>(slab + (uint32_t)(qoff * 128));
         const uint64_t bdesc0 = smem_desc_kmajor<64>(sW);
-        // Occupied taps as a 9-bit mask (one 64-channel block: C == 64). The
-        // lane issuing MMAs is slow at anything else, so the dense case is a
-        // straight run of 36 MMAs and the zero-skip case one branch per tap;
-        // every accumulate flag is a constant (the first occupied tap's first
-        // k-step is the only non-accumulating MMA).
-        uint32_t tapmask = skip ? s_tapm[j % 3] : 0x1FFu;
-        if (tapmask == 0x1FFu) {
-          tc_mma_bf16(d, adesc0, bdesc0, idesc, 0u);
-#pragma unroll
-          for (int i = 1; i < 36; ++i) {
-            const int tap = i >> 2, ks = i & 3;
-            tc_mma_bf16(d, adesc0 + (uint64_t)((((tap / 3) * Wp + (tap % 3)) * 128) >> 4) + (uint64_t)(2 * ks),
-                        bdesc0 + (uint64_t)((tap * CO * 128) >> 4) + (uint64_t)(2 * ks), idesc, 1u);
-          }
-        } else if (tapmask == 0u) {
-          // no tap is occupied: tap 0's activations are all zero, so one
-          // non-accumulating MMA on them writes the zero accumulator
-          tc_mma_bf16(d, adesc0, bdesc0, idesc, 0u);
-        } else {
-          const int ftap = __ffs((int)tapmask) - 1;
-          tapmask &= ~(1u << ftap);
-          {
-            const uint64_t ad = adesc0 + (uint64_t)((((ftap / 3) * Wp + (ftap % 3)) * 128) >> 4);
-            const uint64_t bd = bdesc0 + (uint64_t)((ftap * CO * 128) >> 4);
-            tc_mma_bf16(d, ad, bd, idesc, 0u);
-#pragma unroll
-            for (int ks = 1; ks < 4; ++ks)
-              tc_mma_bf16(d, ad + (uint64_t)(2 * ks), bd + (uint64_t)(2 * ks), idesc, 1u);
-          }
-#pragma unroll
-          for (int tap = 0; tap < 9; ++tap) {
-            if (!((tapmask >> tap) & 1u)) continue;  // all-zero activations, or the peeled tap
-            const uint64_t ad = adesc0 + (uint64_t)((((tap / 3) * Wp + (tap % 3)) * 128) >> 4);
-            const uint64_t bd = bdesc0 + (uint64_t)((tap * CO * 128) >> 4);
-#pragma unroll
-            for (int ks = 0; ks < 4; ++ks)
-              tc_mma_bf16(d, ad + (uint64_t)(2 * ks), bd + (uint64_t)(2 * ks), idesc, 1u);
-          }
+        const uint32_t tapmask = skip ? s_tapm[b] : 0x1FFu;
+        if (j == 0) {
+          ok = mbar_wait_spin(bar_w, 0u, err, s_abort, kErrTimeoutFull);
+          if (!ok) break;
+          tc_fence_after();
         }
-        tc_commit(bar_empty + 8 * b);  // slab free once these MMAs are done
+        conv3_issue<CO>(d, adesc0, bdesc0, Wp, tapmask);
+        tc_commit(bar_empty + 8 * b);  // slab and mask buffer free once these MMAs are done
         tc_commit(bar_accf + 8 * b);
       }
-      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      // TMEM is freed below only after the epilogue has read the last two
+      // accumulators (the waits a further two tiles would make)
+      for (int k = 0; k < 2 && ok; ++k, ++j)
+        ok = mbar_wait(bar_acce + 8 * (j & 1), (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutAcc);
     }
-  } else {
+  } else if (warp >= 4) {
     // -------------------------------------------------------------- epilogue
     // warp w reads TMEM lanes 32 (w % 4).. (its quarter of the tile's rows) and
-    // the 32 accumulator columns 32 ((w - 4) / 4)..
+    // the 32 accumulator columns 32 ((w - 4) / 4)..; the two warps of a lane
+    // quarter meet at one 64-thread named barrier per tile (id 3 + quarter)
     const int q = warp & 3, r = q * 32 + lane, et = threadIdx.x - 128;
-    const int c0 = ((warp - 4) >> 2) * 32;
+    const int hf = (warp - 4) >> 2;
+    const int c0 = hf * 32;
+    const int pair_bar = 3 + q;
     const OccDev o = P.out_occ;
-    const bool acc_smem = emit != 0;
-    const bool affine = P.ep.bias != nullptr || P.ep.bn != nullptr;  // else the column affine is 1, 0
+    const int act = P.ep.act;
+    const __nv_bfloat16* const residual = P.ep.residual;
     // the column affine, read here rather than before the CTA barrier so that
     // its global loads do not hold up the first MMAs
     for (int c = et; c < CO; c += kEpiThreads) {
@@ -319,6 +344,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       s_shift[c] = sh;
     }
     named_bar_sync(2, kEpiThreads);
+    // this warp's 32 columns of the affine stay in registers for every tile
+    float sc[32], sh[32];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float4 a = reinterpret_cast<const float4*>(s_scale + c0)[i];
+      const float4 bq = reinterpret_cast<const float4*>(s_shift + c0)[i];
+      sc[4 * i] = a.x; sc[4 * i + 1] = a.y; sc[4 * i + 2] = a.z; sc[4 * i + 3] = a.w;
+      sh[4 * i] = bq.x; sh[4 * i + 1] = bq.y; sh[4 * i + 2] = bq.z; sh[4 * i + 3] = bq.w;
+    }
+    uint32_t colcnt = 0u;    // non-zeros of column c0 + lane over this warp's rows of every tile
+    int64_t prev_m = -1;     // the previous tile's output row of this thread (its row flag is pending)
     int j = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++j) {
       const int b = j & 1;
@@ -328,116 +364,100 @@ __global__ void __launch_bounds__(kThreads, 1)
       const bool mvalid = oh < H && ow < W;
       const int64_t m = ((int64_t)img * H + oh) * W + ow;
       const bool ok = mbar_wait(bar_accf + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutAcc);
-      // the same abort decision for every epilogue warp (one that left alone
-      // would strand the others at the occupancy barrier)
-      if (named_bar_or(2, kEpiThreads, !ok)) break;
+      // the pair agrees on an abort, and the row flags of the previous tile
+      // (written before this barrier by both warps) can be combined after it
+      if (named_bar_or(pair_bar, 64, !ok)) break;
+      if (emit && hf == 0 && prev_m >= 0) {
+        const int fb = (j - 1) % 3;
+        o.row_bm[prev_m * o.W64] = (s_rowf[(fb * 2 + 0) * 128 + r] | s_rowf[(fb * 2 + 1) * 128 + r]) ? 1ull : 0ull;
+      }
       tc_fence_after();
-      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * CO);
-      const int blk = mvalid ? (int)(m >> 7) : -1;
-      const uint32_t grp = __match_any_sync(0xffffffffu, blk);
-      const bool leader = (__ffs(grp) - 1) == lane;
-      unsigned long long tl = 0ull;
-      {
-        uint32_t raw[32];
-        tmem_ld32_nowait(tbase + (uint32_t)c0, raw);
-        tmem_wait_ld32(raw);
-        uint32_t nzw = 0u;
+      uint32_t raw[32];
+      tmem_ld32_nowait(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * CO + c0), raw);
+      tmem_wait_ld32(raw);
+      float v[32];
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int cc = c0 + h * 16;
-          float v[16];
-          if (affine) {
-#pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) {
-              const float4 sc = reinterpret_cast<const float4*>(s_scale + cc)[q4];
-              const float4 sh = reinterpret_cast<const float4*>(s_shift + cc)[q4];
-              v[4 * q4 + 0] = fmaf(__uint_as_float(raw[h * 16 + 4 * q4 + 0]), sc.x, sh.x);
-              v[4 * q4 + 1] = fmaf(__uint_as_float(raw[h * 16 + 4 * q4 + 1]), sc.y, sh.y);
-              v[4 * q4 + 2] = fmaf(__uint_as_float(raw[h * 16 + 4 * q4 + 2]), sc.z, sh.z);
-              v[4 * q4 + 3] = fmaf(__uint_as_float(raw[h * 16 + 4 * q4 + 3]), sc.w, sh.w);
-            }
-          } else {
-#pragma unroll
-            for (int jj = 0; jj < 16; ++jj) v[jj] = __uint_as_float(raw[h * 16 + jj]);
-          }
-          if (residual && mvalid) {
-            const uint4* rp = reinterpret_cast<const uint4*>(residual + m * G.Co + cc);
-            const uint4 r0 = rp[0], r1 = rp[1];
-            const __nv_bfloat162* h0 = reinterpret_cast<const __nv_bfloat162*>(&r0);
-            const __nv_bfloat162* h1 = reinterpret_cast<const __nv_bfloat162*>(&r1);
-#pragma unroll
-            for (int jj = 0; jj < 4; ++jj) {
-              const float2 a0 = __bfloat1622float2(h0[jj]);
-              const float2 a1 = __bfloat1622float2(h1[jj]);
-              v[2 * jj] += a0.x;
-              v[2 * jj + 1] += a0.y;
-              v[8 + 2 * jj] += a1.x;
-              v[8 + 2 * jj + 1] += a1.y;
-            }
-          }
-          if (act == 1) {
-#pragma unroll
-            for (int jj = 0; jj < 16; ++jj) v[jj] = v[jj] > 0.f ? v[jj] : 0.f;
-          } else if (act == 2) {
-#pragma unroll
-            for (int jj = 0; jj < 16; ++jj) v[jj] = v[jj] > 0.f ? (v[jj] < 6.f ? v[jj] : 6.f) : 0.f;
-          } else if (act == 3) {
-#pragma unroll
-            for (int jj = 0; jj < 16; ++jj) v[jj] = gelu_f(v[jj]);
-          }
-          uint32_t pk[8];
-#pragma unroll
-          for (int jj = 0; jj < 8; ++jj) {
-            const __nv_bfloat162 h2 = __floats2bfloat162_rn(v[2 * jj], v[2 * jj + 1]);
-            pk[jj] = *reinterpret_cast<const uint32_t*>(&h2);
-            nzw |= ((pk[jj] & 0x7FFFu) ? 1u : 0u) << (h * 16 + 2 * jj);
-            nzw |= ((pk[jj] & 0x7FFF0000u) ? 1u : 0u) << (h * 16 + 2 * jj + 1);
-          }
-          if (mvalid) {
-            uint4* yp = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(P.y) + m * G.Co + cc);
-            yp[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            yp[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-          }
-        }
-        if (!mvalid) nzw = 0u;
-        if (emit) {
-          if (nzw) tl |= 1ull << ((c0 >> 6) & 63);
-          const uint32_t bits = __reduce_or_sync(grp, nzw);
-          const int word = c0 >> 5;
-          if (leader && blk >= 0 && bits) atomicOr(&o.blk_mask[blk * o.C32 + word], bits);
-          s_cnt[q * CO + c0 + lane] = __popc(warp_transpose32(nzw));
-        }
-      }
+      for (int i = 0; i < 32; ++i) v[i] = fmaf(__uint_as_float(raw[i]), sc[i], sh[i]);
       tc_fence_before();
-      mbar_arrive(bar_acce + 8 * b);
-      if (emit) {
-        // both column halves of a row meet in shared memory; the tile owns its
-        // output rows, so the half-0 thread stores the word once
-        if (tl) atomicOr(&s_rowbm[r], tl);
-        named_bar_sync(2, kEpiThreads);
-        if (c0 == 0) {
-          const unsigned long long v = s_rowbm[r];
-          s_rowbm[r] = 0ull;
-          if (mvalid) o.row_bm[m * o.W64] = v;
+      mbar_arrive(bar_acce + 8 * b);  // the accumulator is in registers
+      if (residual && mvalid) {
+        const uint4* rp = reinterpret_cast<const uint4*>(residual + m * G.Co + c0);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const uint4 rv = rp[k];
+          const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&rv);
+#pragma unroll
+          for (int jj = 0; jj < 4; ++jj) {
+            const float2 a = __bfloat1622float2(h[jj]);
+            v[8 * k + 2 * jj] += a.x;
+            v[8 * k + 2 * jj + 1] += a.y;
+          }
         }
-        for (int c = et; c < CO; c += kEpiThreads)
-          s_acc[c] += s_cnt[c] + s_cnt[CO + c] + s_cnt[2 * CO + c] + s_cnt[3 * CO + c];
-        named_bar_sync(2, kEpiThreads);
       }
+      uint32_t pk[16];
+      if (act == 1) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) pk[i] = pack_bf16x2<true>(v[2 * i], v[2 * i + 1]);
+      } else {
+        if (act == 2) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = fminf(fmaxf(v[i], 0.f), 6.f);
+        } else if (act == 3) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = gelu_f(v[i]);
+        }
+#pragma unroll
+        for (int i = 0; i < 16; ++i) pk[i] = pack_bf16x2<false>(v[2 * i], v[2 * i + 1]);
+      }
+      if (mvalid) {
+        uint4* yp = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(P.y) + m * G.Co + c0);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) yp[k] = make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
+      }
+      if (emit) {
+        uint32_t nzw = 0u;  // bit i: column c0 + i of this row is non-zero
+#pragma unroll
+        for (int i = 0; i < 16; ++i) nzw |= nz_pair(pk[i]) << (2 * i);
+        if (!mvalid) nzw = 0u;
+        // block-column mask: the warp's 32 positions cover at most two
+        // 128-row blocks of the output (the first and the last valid row's)
+        const int blk = mvalid ? (int)(m >> 7) : -1;
+        const uint32_t vmask = __ballot_sync(0xffffffffu, mvalid);
+        if (vmask) {
+          const int lo = __shfl_sync(0xffffffffu, blk, __ffs(vmask) - 1);
+          const int hi = __shfl_sync(0xffffffffu, blk, 31 - __clz(vmask));
+          const uint32_t b_lo = __reduce_or_sync(0xffffffffu, blk == lo ? nzw : 0u);
+          const uint32_t b_hi = hi != lo ? __reduce_or_sync(0xffffffffu, blk == hi ? nzw : 0u) : 0u;
+          if (lane == 0 && b_lo) atomicOr(&o.blk_mask[lo * o.C32 + (c0 >> 5)], b_lo);
+          if (lane == 1 && b_hi) atomicOr(&o.blk_mask[hi * o.C32 + (c0 >> 5)], b_hi);
+        }
+        colcnt += __popc(warp_transpose32(nzw));
+        s_rowf[((j % 3) * 2 + hf) * 128 + r] = nzw ? 1 : 0;
+      }
+      prev_m = mvalid ? m : -1;
     }
-    if (emit && acc_smem) {
-      unsigned long long total = 0ull;
-      for (int cb0 = 0; cb0 < CO; cb0 += kEpiThreads) {
-        const int c = cb0 + et;
-        const uint32_t cnt = c < CO ? s_acc[c] : 0u;
-        if (cnt) atomicAdd(&o.col_nnz[c], cnt);
+    // the last tile's row flags
+    named_bar_sync(pair_bar, 64);
+    if (emit && hf == 0 && prev_m >= 0) {
+      const int fb = (j - 1) % 3;
+      o.row_bm[prev_m * o.W64] = (s_rowf[(fb * 2 + 0) * 128 + r] | s_rowf[(fb * 2 + 1) * 128 + r]) ? 1ull : 0ull;
+    }
+    if (emit) {
+      // column counts: the four lane quarters meet in shared memory, then one
+      // atomic per column, per 64-column tile and for the total
+      if (colcnt) atomicAdd(&s_acc[c0 + lane], colcnt);
+      named_bar_sync(2, kEpiThreads);
+      if (et < CO) {
+        const uint32_t cnt = s_acc[et];
+        if (cnt) atomicAdd(&o.col_nnz[et], cnt);
         uint32_t sum = cnt;
 #pragma unroll
-        for (int s = 16; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
-        total += sum;
-        if (lane == 0 && sum) atomicAdd(&o.tile_nnz[c >> 6], sum);
+        for (int sft = 16; sft > 0; sft >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, sft);
+        if (lane == 0 && sum) {
+          atomicAdd(&o.tile_nnz[et >> 6], sum);
+          atomicAdd(o.nnz, (unsigned long long)sum);
+        }
       }
-      if (lane == 0 && total) atomicAdd(o.nnz, total);
     }
   }
 
