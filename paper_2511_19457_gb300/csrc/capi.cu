@@ -91,6 +91,8 @@ struct sparoa_ctx {
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;  // its fork / join with `stream`
   uint32_t* d_err() const { return reinterpret_cast<uint32_t*>(small.p); }
   int32_t* d_path() const { return reinterpret_cast<int32_t*>(reinterpret_cast<char*>(small.p) + 16); }
+  // Eq. 1 count of an FC input that the fused small-FC kernel measures itself
+  uint64_t* d_count() const { return reinterpret_cast<uint64_t*>(reinterpret_cast<char*>(small.p) + 32); }
 };
 
 namespace {
@@ -453,11 +455,51 @@ struct GemmPlan {
   DispatchDev disp;
 };
 
-sparoa_status run_gemm(sparoa_ctx* ctx, const GemmPlan& g, cudaStream_t stream, int ws_slot = -1) {
+// count_out: the input's Eq. 1 count is not known yet; the fused small-FC
+// kernel measures it into count_out (which g.disp.in_nnz points at).
+sparoa_status run_gemm(sparoa_ctx* ctx, const GemmPlan& g, cudaStream_t stream, int ws_slot = -1,
+                       unsigned long long* count_out = nullptr) {
   const bool small_skip = g.M <= 128 && g.W_kn != nullptr && g.K <= 8192 && (g.N % 8) == 0;
+  // small inputs: statistics, dispatch and either path's product in one kernel
+  const bool fused = small_skip && fcsmall_supported((int)g.M, (int)g.K, (int)g.N);
   const int force = g.disp.force;
   OccDev yo{};
   if (g.yo) yo = to_dev(*g.yo);
+  if (fused) {
+    // both paths of a small FC in one launch (count, dispatch, product)
+    FcSkipArgs f;
+    f.x = static_cast<const __nv_bfloat16*>(g.x);
+    f.w_kn = static_cast<const __nv_bfloat16*>(g.W_kn);
+    f.M = (int)g.M;
+    f.K = (int)g.K;
+    f.N = (int)g.N;
+    f.ep = g.ep;
+    f.y = g.y;
+    f.y_f32 = g.y_f32;
+    f.disp = g.disp;
+    f.out_occ = yo;
+    f.emit = g.yo ? 1 : 0;
+    f.nnz_out = count_out;
+    SP_CUDA(launch_fcsmall(f, stream));
+    return SPAROA_OK;
+  }
+  if (small_skip && force != 1) {
+    FcSkipArgs f;
+    f.x = static_cast<const __nv_bfloat16*>(g.x);
+    f.w_kn = static_cast<const __nv_bfloat16*>(g.W_kn);
+    f.M = (int)g.M;
+    f.K = (int)g.K;
+    f.N = (int)g.N;
+    f.in_blk = g.xo.blk_mask;
+    f.in_C32 = (int)((g.K + 31) / 32);
+    f.ep = g.ep;
+    f.y = g.y;
+    f.y_f32 = g.y_f32;
+    f.disp = g.disp;
+    f.out_occ = yo;
+    f.emit = g.yo ? 1 : 0;
+    SP_CUDA(launch_fcskip(f, stream));
+  }
   if (!(small_skip && force == 2)) {
     IgemmArgs a;
     a.M = (int)g.M;
@@ -478,23 +520,6 @@ sparoa_status run_gemm(sparoa_ctx* ctx, const GemmPlan& g, cudaStream_t stream, 
     a.err = ctx->d_err();
     SP_TRY(offer_splitk(ctx, &a, ws_slot));
     SP_CUDA(launch_igemm(a, stream));
-  }
-  if (small_skip && force != 1) {
-    FcSkipArgs f;
-    f.x = static_cast<const __nv_bfloat16*>(g.x);
-    f.w_kn = static_cast<const __nv_bfloat16*>(g.W_kn);
-    f.M = (int)g.M;
-    f.K = (int)g.K;
-    f.N = (int)g.N;
-    f.in_blk = g.xo.blk_mask;
-    f.in_C32 = (int)((g.K + 31) / 32);
-    f.ep = g.ep;
-    f.y = g.y;
-    f.y_f32 = g.y_f32;
-    f.disp = g.disp;
-    f.out_occ = yo;
-    f.emit = g.yo ? 1 : 0;
-    SP_CUDA(launch_fcskip(f, stream));
   }
   return SPAROA_OK;
 }
@@ -758,8 +783,20 @@ sparoa_status sparoa_gemm(sparoa_ctx* ctx, const void* x, int64_t M, int64_t K, 
   p.y = y;
   p.y_f32 = y_dtype == SPAROA_F32;
   p.yo = y_occ;
-  if (x_occ) p.xo = *x_occ;
-  else SP_TRY(measure(ctx, x, M, K, &p.xo));
+  // a small input with its [K, N] weights is measured by the fused FC kernel
+  // itself (count only); otherwise by the statistics kernel
+  const bool fused_count = !x_occ && M > 0 && M <= 128 && W_kn && K <= 8192 &&
+                           fcsmall_supported((int)M, (int)K, (int)N);
+  if (x_occ) {
+    p.xo = *x_occ;
+  } else if (fused_count) {
+    memset(&p.xo, 0, sizeof(p.xo));
+    p.xo.nnz = ctx->d_count();
+    p.xo.R = M;
+    p.xo.C = K;
+  } else {
+    SP_TRY(measure(ctx, x, M, K, &p.xo));
+  }
   if (y_occ) SP_TRY(occ_clear(ctx, *y_occ));
   p.disp.in_nnz = reinterpret_cast<const unsigned long long*>(p.xo.nnz);
   p.disp.numel = (unsigned long long)(M * K);
@@ -767,7 +804,9 @@ sparoa_status sparoa_gemm(sparoa_ctx* ctx, const void* x, int64_t M, int64_t K, 
   p.disp.fpb_ok = intensity_ok(t, w);
   p.disp.force = t.force_path;
   p.disp.path_out = ctx->d_path();
-  if (M > 0) SP_TRY(run_gemm(ctx, p, ctx->stream));
+  if (M > 0)
+    SP_TRY(run_gemm(ctx, p, ctx->stream, -1,
+                    fused_count ? reinterpret_cast<unsigned long long*>(ctx->d_count()) : nullptr));
   if (!host_out) return SPAROA_OK;
   uint64_t nnz = 0;
   int32_t path = 0;

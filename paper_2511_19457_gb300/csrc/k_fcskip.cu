@@ -237,6 +237,311 @@ __global__ void __launch_bounds__(kThreads) fcskip_kernel(const FcSkipArgs a) {
   }
 }
 
+// ---------------------------------------------------------------------------
+// Fused small FC: statistics, dispatch and the zero-skip product in one launch
+// ---------------------------------------------------------------------------
+// For inputs small enough to sit in shared memory whole (M <= 128 rows,
+// M * (K + 8) * 2 bytes within kSmallXBytes) every CTA loads x once and
+// derives from it what the separate statistics kernel would: the Eq. 1
+// non-zero count (Sec. 3.1) and which columns hold a non-zero.  All CTAs reach
+// the same decision (Sec. 3 rule); on the zero-skip path each CTA multiplies
+// the occupied columns of x by the matching rows of W_kn for its 16 output
+// columns on the tensor cores (mma.sync m16n8k16, fp32 accumulation), the
+// columns compacted into dense k-steps of 16 (Sec. 2.1: zero activations
+// take no part); on the dense path every column takes part.  A 128-row
+// tcgen05 tile would be mostly empty at these sizes, so both paths of a
+// small FC run here, in one launch.  CTA 0 writes the count and the path
+// for the host record.
+constexpr int kSmallTN = 16;
+constexpr size_t kSmallXBytes = 160 * 1024;
+
+__device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr)
+               : "memory");
+}
+
+constexpr int kSmallThreads = 1024;  // 32 warps: short dependency chains per warp
+constexpr int kSmallWarps = kSmallThreads / 32;
+
+struct SmallGeo {
+  int xpitch;   // bf16 elements per staged x row: K + 8 (column K stays zero)
+  int mp8;      // rows staged: M rounded up to 8 (the extra rows zero)
+  int kc;       // compacted K bound: K rounded up to 16
+  size_t x_off, any_off, w_off, red_off, col_off, misc_off, bytes;
+};
+
+__host__ __device__ inline SmallGeo small_geo(int M, int K) {
+  SmallGeo g;
+  g.xpitch = K + 8;
+  g.mp8 = (M + 7) / 8 * 8;
+  g.kc = (K + 15) / 16 * 16;
+  g.x_off = 0;
+  g.any_off = ((size_t)g.mp8 * g.xpitch * 2 + 15) / 16 * 16;          // [K / 2] u32: pair occupancy
+  g.w_off = (g.any_off + (size_t)(K / 2) * 4 + 15) / 16 * 16;        // [kc][16] bf16: W rows taken
+  g.red_off = g.w_off + (size_t)g.kc * kSmallTN * 2;                 // [32][16][16] fp32 partial sums
+  g.col_off = g.red_off + (size_t)kSmallWarps * 16 * kSmallTN * 4;   // [kc] columns taken
+  g.misc_off = (g.col_off + (size_t)g.kc * 2 + 15) / 16 * 16;
+  g.bytes = g.misc_off + 256;  // count, path, per-warp counts [32], per-column output counts [16]
+  return g;
+}
+
+__global__ void __launch_bounds__(kSmallThreads) fcsmall_kernel(const FcSkipArgs a) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  const int M = a.M, K = a.K, N = a.N;
+  const SmallGeo G = small_geo(M, K);
+  __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(smem + G.x_off);
+  uint32_t* s_any = reinterpret_cast<uint32_t*>(smem + G.any_off);
+  __nv_bfloat16* wc = reinterpret_cast<__nv_bfloat16*>(smem + G.w_off);
+  float* red = reinterpret_cast<float*>(smem + G.red_off);
+  short* s_col = reinterpret_cast<short*>(smem + G.col_off);
+  uint32_t* s_cnt32 = reinterpret_cast<uint32_t*>(smem + G.misc_off);  // x's non-zeros
+  int* s_path = reinterpret_cast<int*>(smem + G.misc_off + 8);
+  int* s_wsum = reinterpret_cast<int*>(smem + G.misc_off + 16);     // [32]
+  uint32_t* s_cnt = reinterpret_cast<uint32_t*>(smem + G.misc_off + 144);  // [16]
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int n0 = blockIdx.x * kSmallTN;
+  const int KP = K / 2;  // column pairs
+
+  for (int i = tid; i < KP; i += kSmallThreads) s_any[i] = 0u;
+  if (tid == 0) *s_cnt32 = 0u;
+  if (tid < kSmallTN) s_cnt[tid] = 0u;
+  pdl_wait();
+  pdl_trigger();
+  // the epilogue's column affine, fetched now: thread t < 4 Mp takes row
+  // t / 4 and the four columns n0 + 4 (t % 4) ..
+  float e_sc[4], e_sh[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int n = n0 + (tid & 3) * 4 + j;
+    e_sc[j] = 1.f;
+    e_sh[j] = 0.f;
+    if (n < N) epi_affine(a.ep, N, n, e_sc[j], e_sh[j]);
+  }
+  // 1. x whole into shared memory (16-byte copies, all in flight); rows
+  //    M .. mp8 - 1 and column K zero
+  const uint32_t xs_u32 = smem_u32(xs);
+  const int chunks = K / 8;
+  for (int idx = tid; idx < M * chunks; idx += kSmallThreads) {
+    const int r = idx / chunks, c = idx - (idx / chunks) * chunks;
+    cp_async_16(xs_u32 + (uint32_t)((r * G.xpitch + c * 8) * 2), a.x + (int64_t)r * K + c * 8, 16u);
+  }
+  cp_async_commit();
+  for (int idx = tid; idx < (G.mp8 - M) * (chunks + 1); idx += kSmallThreads) {
+    const int r = M + idx / (chunks + 1), c = idx - (idx / (chunks + 1)) * (chunks + 1);
+    *reinterpret_cast<uint4*>(xs + r * G.xpitch + c * 8) = make_uint4(0u, 0u, 0u, 0u);
+  }
+  for (int r = tid; r < M; r += kSmallThreads)
+    *reinterpret_cast<uint4*>(xs + r * G.xpitch + K) = make_uint4(0u, 0u, 0u, 0u);
+  cp_async_wait<0>();
+  __syncthreads();
+
+  // 2. Eq. 1 count and occupied column pairs: unit = (pair, 8 rows); the
+  //    non-zero bits of a bf16 pair land on bits 15 / 31
+  const uint32_t* x32 = reinterpret_cast<const uint32_t*>(xs);
+  const int pitch32 = G.xpitch / 2;
+  uint32_t cnt = 0u;
+  const int units = KP * (G.mp8 / 8);
+  for (int u = tid; u < units; u += kSmallThreads) {
+    const int oct = u / KP, cp = u - oct * KP;
+    const uint32_t* col = x32 + oct * 8 * pitch32 + cp;
+    uint32_t wv[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) wv[i] = col[i * pitch32];
+    uint32_t any = 0u;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t t = ((wv[i] & 0x7FFF7FFFu) + 0x7FFF7FFFu) & 0x80008000u;
+      any |= t;
+      cnt += __popc(t);
+    }
+    if (any) atomicOr(&s_any[cp], any);
+  }
+#pragma unroll
+  for (int sft = 16; sft > 0; sft >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, sft);
+  if (lane == 0 && cnt) atomicAdd(s_cnt32, cnt);  // M * K < 2^31: a 32-bit count
+  __syncthreads();
+
+  // 3. the rule (every CTA reaches the same decision)
+  const unsigned long long nnz = *s_cnt32;
+  if (tid == 0) {
+    int path;
+    if (a.disp.force == 1) path = 1;
+    else if (a.disp.force == 2) path = 2;
+    else {
+      const double numel = (double)((unsigned long long)M * (unsigned long long)K);
+      const double zeros = numel - (double)nnz;
+      path = zeros >= __dmul_rn(a.disp.s_thr, numel) ? 2 : (a.disp.fpb_ok ? 1 : 2);
+    }
+    *s_path = path;
+    if (blockIdx.x == 0) {
+      if (a.nnz_out) *a.nnz_out = nnz;
+      if (a.disp.path_out) *a.disp.path_out = path;
+    }
+  }
+  __syncthreads();
+  const int path = *s_path;
+
+  // 4. the columns that take part, in increasing order: every column on the
+  //    dense path; on the zero-skip path the occupied ones, numbered from the
+  //    warps' ballots and a prefix over the warps, a pass of 1024 pairs at a
+  //    time
+  int nocc = 0;
+  if (path == 2) {
+    for (int pass0 = 0; pass0 < KP; pass0 += kSmallThreads) {
+      const int cp = pass0 + tid;
+      const uint32_t any = cp < KP ? s_any[cp] : 0u;
+      const bool f_lo = (any >> 15) & 1u, f_hi = any >> 31;
+      const uint32_t b_lo = __ballot_sync(0xffffffffu, f_lo), b_hi = __ballot_sync(0xffffffffu, f_hi);
+      const uint32_t lt = (1u << lane) - 1u;
+      if (lane == 0) s_wsum[warp] = __popc(b_lo) + __popc(b_hi);
+      __syncthreads();
+      // exclusive prefix of the 32 warps' counts: one load per lane, a scan
+      // by shuffles
+      const int wv = s_wsum[lane];
+      int incl = wv;
+#pragma unroll
+      for (int sft = 1; sft < 32; sft <<= 1) {
+        const int t2 = __shfl_up_sync(0xffffffffu, incl, sft);
+        if (lane >= sft) incl += t2;
+      }
+      const int total = __shfl_sync(0xffffffffu, incl, 31);
+      int off = nocc + __shfl_sync(0xffffffffu, incl - wv, warp) + __popc(b_lo & lt) + __popc(b_hi & lt);
+      if (f_lo) s_col[off++] = (short)(2 * cp);
+      if (f_hi) s_col[off] = (short)(2 * cp + 1);
+      nocc += total;
+      __syncthreads();  // s_wsum is reused by the next pass
+    }
+  } else {
+    for (int k = tid; k < K; k += kSmallThreads) s_col[k] = (short)k;
+    nocc = K;
+  }
+  const int kc = (nocc + 15) / 16 * 16;
+  for (int k = nocc + tid; k < kc; k += kSmallThreads) s_col[k] = (short)K;  // the zero column
+  __syncthreads();
+  // W rows of the columns taken: W_kn[col][n0 .. n0 + 16), zero for the padding
+  for (int idx = tid; idx < kc * 2; idx += kSmallThreads) {
+    const int kk = idx >> 1, h = idx & 1;
+    const int col = s_col[kk];
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (col < K && n0 + h * 8 + 8 <= N) v = __ldg(reinterpret_cast<const uint4*>(a.w_kn + (int64_t)col * N + n0 + h * 8));
+    *reinterpret_cast<uint4*>(wc + kk * kSmallTN + h * 8) = v;
+  }
+  __syncthreads();
+
+  // 5. tensor-core product over the k-steps of 16 taken columns: warp w takes
+  //    row group w % RG (16 rows) and every KS-th k-step from w / RG
+  const int RG = (M + 15) / 16;
+  const int KS = kSmallWarps / RG;
+  const int rg = warp % RG, ks0 = warp / RG;
+  const int g = lane >> 2, tq = lane & 3;
+  const int Mp = RG * 16;
+  if (ks0 < KS) {
+    float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    const int r0 = rg * 16 + g, r1 = r0 + 8;
+    const bool v0 = r0 < M, v1 = r1 < M;
+    const __nv_bfloat16* xr0 = xs + (v0 ? r0 : 0) * G.xpitch;
+    const __nv_bfloat16* xr1 = xs + (v1 ? r1 : 0) * G.xpitch;
+    const uint32_t w_lane = smem_u32(wc) + (uint32_t)(((lane & 15) * kSmallTN + (lane >> 4) * 8) * 2);
+    for (int k0 = ks0 * 16; k0 < kc; k0 += KS * 16) {
+      const uint32_t p01 = *reinterpret_cast<const uint32_t*>(s_col + k0 + 2 * tq);
+      const uint32_t p23 = *reinterpret_cast<const uint32_t*>(s_col + k0 + 2 * tq + 8);
+      const int c0 = (int)(p01 & 0xFFFFu), c1 = (int)(p01 >> 16);
+      const int c2 = (int)(p23 & 0xFFFFu), c3 = (int)(p23 >> 16);
+      uint32_t af[4];
+      af[0] = v0 ? ((uint32_t)__bfloat16_as_ushort(xr0[c0]) | ((uint32_t)__bfloat16_as_ushort(xr0[c1]) << 16)) : 0u;
+      af[1] = v1 ? ((uint32_t)__bfloat16_as_ushort(xr1[c0]) | ((uint32_t)__bfloat16_as_ushort(xr1[c1]) << 16)) : 0u;
+      af[2] = v0 ? ((uint32_t)__bfloat16_as_ushort(xr0[c2]) | ((uint32_t)__bfloat16_as_ushort(xr0[c3]) << 16)) : 0u;
+      af[3] = v1 ? ((uint32_t)__bfloat16_as_ushort(xr1[c2]) | ((uint32_t)__bfloat16_as_ushort(xr1[c3]) << 16)) : 0u;
+      uint32_t b0, b1, b2, b3;
+      ldsm_x4_t(w_lane + (uint32_t)(k0 * kSmallTN * 2), b0, b1, b2, b3);
+      mma_16816(acc[0], af, b0, b1);
+      mma_16816(acc[1], af, b2, b3);
+    }
+    // partial sums of this k-step group: red[ks][row][16]
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      float* rb = red + ((size_t)ks0 * Mp + rg * 16) * kSmallTN + j * 8 + 2 * tq;
+      rb[g * kSmallTN] = acc[j][0];
+      rb[g * kSmallTN + 1] = acc[j][1];
+      rb[(g + 8) * kSmallTN] = acc[j][2];
+      rb[(g + 8) * kSmallTN + 1] = acc[j][3];
+    }
+  }
+  __syncthreads();
+
+  // 6. epilogue: thread t < 4 Mp = (row t / 4, columns n0 + 4 (t % 4) ..)
+  const OccDev o = a.out_occ;
+  if (tid < Mp * 4) {
+    const int row = tid >> 2, cq = tid & 3;
+    const int64_t m = row;
+    float v4[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int k2 = 0; k2 < KS; ++k2) {
+      const float4 pv = *reinterpret_cast<const float4*>(red + ((size_t)k2 * Mp + row) * kSmallTN + cq * 4);
+      v4[0] += pv.x;
+      v4[1] += pv.y;
+      v4[2] += pv.z;
+      v4[3] += pv.w;
+    }
+    uint32_t bits = 0u;
+    if (row < M) {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int n = n0 + cq * 4 + j;
+        if (n >= N) continue;
+        float v = fmaf(v4[j], e_sc[j], e_sh[j]);
+        if (a.ep.residual) v += __bfloat162float(a.ep.residual[m * N + n]);
+        v = epi_act(v, a.ep.act);
+        if (a.y_f32) {
+          reinterpret_cast<float*>(a.y)[m * N + n] = v;
+        } else {
+          const __nv_bfloat16 ob = __float2bfloat16_rn(v);
+          reinterpret_cast<__nv_bfloat16*>(a.y)[m * N + n] = ob;
+          if (bf16_nz(__bfloat16_as_ushort(ob))) bits |= 1u << j;
+        }
+      }
+    }
+    if (a.emit) {
+      // the row's 16 columns are held by 4 consecutive threads (one warp)
+      uint32_t rb16 = bits << (cq * 4);
+      rb16 |= __shfl_xor_sync(0xffffffffu, rb16, 1);
+      rb16 |= __shfl_xor_sync(0xffffffffu, rb16, 2);
+      if (cq == 0 && rb16 && row < M) atomicOr(&o.row_bm[m * o.W64 + (n0 >> 12)], 1ull << ((n0 >> 6) & 63));
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if ((bits >> j) & 1u) atomicAdd(&s_cnt[cq * 4 + j], 1u);
+      const uint32_t wbits = __reduce_or_sync(0xffffffffu, rb16);
+      const int w = n0 >> 5;
+      if (lane == 0 && wbits && w < o.C32) atomicOr(&o.blk_mask[w], wbits << (n0 & 31));
+    }
+  }
+  if (a.emit) {
+    __syncthreads();
+    if (tid < kSmallTN) {
+      const uint32_t c = s_cnt[tid];
+      const int n = n0 + tid;
+      if (c && n < N) atomicAdd(&o.col_nnz[n], c);
+    }
+    if (tid == 0) {
+      uint32_t sum = 0u;
+      for (int j = 0; j < kSmallTN; ++j) sum += s_cnt[j];
+      if (sum) {
+        atomicAdd(&o.tile_nnz[n0 >> 6], sum);
+        atomicAdd(o.nnz, (unsigned long long)sum);
+      }
+    }
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_fcskip(const FcSkipArgs& a, cudaStream_t s) {
@@ -250,6 +555,23 @@ cudaError_t launch_fcskip(const FcSkipArgs& a, cudaStream_t s) {
   }
   dim3 grid((a.N + kTN - 1) / kTN, (a.M + kTM - 1) / kTM);
   return launch_kernel(fcskip_kernel, grid, dim3(kThreads), smem, s, a);
+}
+
+bool fcsmall_supported(int M, int K, int N) {
+  return M > 0 && M <= 128 && K % 8 == 0 && N % 8 == 0 && K < 32760 &&
+         (size_t)M * (K + 8) * 2 <= kSmallXBytes && small_geo(M, K).bytes <= 220 * 1024;
+}
+
+cudaError_t launch_fcsmall(const FcSkipArgs& a, cudaStream_t s) {
+  if (a.M <= 0 || a.N <= 0) return cudaSuccess;
+  if (!fcsmall_supported(a.M, a.K, a.N)) return cudaErrorInvalidValue;
+  const size_t smem = small_geo(a.M, a.K).bytes;
+  if (smem > 40 * 1024) {
+    cudaError_t e = smem_optin(reinterpret_cast<const void*>(fcsmall_kernel), smem);
+    if (e != cudaSuccess) return e;
+  }
+  dim3 grid((a.N + kSmallTN - 1) / kSmallTN);
+  return launch_kernel(fcsmall_kernel, grid, dim3(kSmallThreads), smem, s, a);
 }
 
 }  // namespace sparoa

@@ -266,6 +266,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int KS = P.ksplit > 1 ? P.ksplit : 1;
   const int units = tiles * KS;
 
+  if (P.dense_only) {
+    // launched next to the fused small-FC kernel, which handles the zero-skip
+    // path: decide first, and leave before any set-up when it is not ours
+    pdl_wait();
+    if (decide_path(P.disp) == 2) {
+      pdl_trigger();
+      return;
+    }
+  }
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(bar_full + 8 * s, p.conv == 1 ? 129u : 1u);

@@ -118,8 +118,17 @@ struct FcSkipArgs {
   DispatchDev disp{};
   OccDev out_occ{};
   int emit = 0;
+  unsigned long long* nnz_out = nullptr;  // fcsmall: where CTA 0 writes x's Eq. 1 count
 };
 cudaError_t launch_fcskip(const FcSkipArgs& a, cudaStream_t s);
+
+// Fused statistics + dispatch + FC for an x that fits shared memory whole
+// (M <= 128): counts x's non-zeros and occupied columns itself, writes the
+// count to nnz_out (nullable) and the path to disp.path_out, and multiplies
+// on the tensor cores (mma.sync) the occupied columns (zero-skip path) or all
+// of them (dense path).
+bool fcsmall_supported(int M, int K, int N);
+cudaError_t launch_fcsmall(const FcSkipArgs& a, cudaStream_t s);
 
 // ----------------------------------------------------------------------------
 // Vision-transformer operators (k_vit.cu)
