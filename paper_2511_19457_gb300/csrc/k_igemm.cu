@@ -209,7 +209,8 @@ __device__ __forceinline__ UnitGeo unit_geo(const Geo& p, int u, int KS, int kbl
 template <int BN, int BK>
 __global__ void __launch_bounds__(kThreads, 1)
     igemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                 const __grid_constant__ CUtensorMap tmY, const IgemmArgs P) {
+                 const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmA32,
+                 const __grid_constant__ CUtensorMap tmB32, const IgemmArgs P) {
   using C = Cfg<BN, BK>;
   const Geo p = make_geo(P);
   const EpiDev ep = P.ep;
@@ -258,6 +259,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int kblocks = (p.Ktot + BK - 1) / BK;
+  const int kgroups = (p.Ktot + 31) / 32;  // 32-column groups of K (compacted zero-skip GEMM)
   const int nt = (p.N + BN - 1) / BN;
   const int mtiles = p.conv == 2 ? ((p.Nimg + p.bn - 1) / p.bn) * p.th * p.tw : (p.M + kBM - 1) / kBM;
   const int tiles = mtiles * nt;
@@ -288,6 +290,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_mbar_init();
     if (p.conv != 1) prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
+    if (p.conv == 0 && BK == 64) {
+      prefetch_tmap(&tmA32);
+      prefetch_tmap(&tmB32);
+    }
     if (!y_f32) prefetch_tmap(&tmY);
   }
   if (warp == kMmaWarp) tmem_alloc(smem_u32(s_tmem), C::kTmemCols);
@@ -313,6 +319,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const bool run = !(P.dense_only && path == 2);
   if (run) record_path(P.disp, path);
   const bool skip = (path == 2);
+  // zero-skip GEMM with 64-wide K blocks: stages hold two occupied 32-column
+  // groups each (compacted), loaded as 32-column boxes with the 64-byte swizzle
+  const bool compact = skip && p.conv == 0 && BK == 64 && kgroups <= kMaxKWords * 32;
 
   if (!run) {
     // nothing to do; fall through to the common exit (TMEM is freed there)
@@ -333,7 +342,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (skip) {
         // ---- occupied K blocks of this tile
         named_bar_sync(1, 128);  // thread 0 is done with the previous tile's bits
-        if (p.conv == 0) {
+        if (compact) {
+          // occupied 32-column groups of this unit's K range in the tile's
+          // 128-row block: one bit per group
+          const int g0 = 2 * kb0, g1 = 2 * kb1 < kgroups ? 2 * kb1 : kgroups;
+          const uint32_t* words = in_blk + (int64_t)(g.m0 >> 7) * in_C32;
+          for (int w0 = 0; w0 < kgroups && w0 < kMaxKWords * 32; w0 += 128) {
+            const int gi = w0 + r;
+            const bool occ = gi >= g0 && gi < g1 && words[gi] != 0u;
+            const uint32_t bits = __ballot_sync(0xffffffffu, occ);
+            if (lane == 0 && (w0 >> 5) + warp < kMaxKWords) s_kbits[(w0 >> 5) + warp] = bits;
+          }
+        } else if (p.conv == 0) {
           for (int w0 = 0; w0 < kblocks && w0 < kMaxKWords * 32; w0 += 128) {
             const int kb = w0 + r;
             // a K block covers BK / 32 words of the 128-row block-column mask
@@ -396,6 +416,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // last occupied block of this unit's K range; a range with none still
         // runs its first block (whose data is all zero)
         last = kb0;
+        if (compact) last = kb1 - 1;  // unused: the compacted loop tracks its own last stage
         for (int kb = kb1 - 1; kb > kb0; --kb) {
           if (kb >= kMaxKWords * 32 || ((s_kbits[kb >> 5] >> (kb & 31)) & 1u)) {
             last = kb;
@@ -404,7 +425,58 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (!ok) continue;  // keep the skip-mask barriers in step; issue nothing more
-      if (p.conv != 1) {
+      if (compact) {
+        if (r == 0) {
+          // pairs of occupied groups in increasing order; an odd last group
+          // takes a stage alone; a unit with none runs group g0 (all zero) so
+          // that its accumulator is written
+          const int g0 = 2 * kb0, g1 = 2 * kb1 < kgroups ? 2 * kb1 : kgroups;
+          int cnt = 0;
+          for (int wd = g0 >> 5; wd <= (g1 - 1) >> 5; ++wd) cnt += __popc(s_kbits[wd]);
+          const int nst = cnt ? (cnt + 1) / 2 : 1;
+          int slot = it % S;
+          uint32_t ph = (uint32_t)((it / S) & 1);
+          int st = 0, pend = -1;
+          auto issue = [&](int ga, int gb) -> bool {
+            if (it >= S && !mbar_wait(bar_empty + 8 * slot, ph ^ 1u, err, s_abort, kErrTimeoutEmpty)) return false;
+            const uint32_t fb = bar_full + 8 * slot;
+            const int nh = gb >= 0 ? 2 : 1;
+            stage_last[slot] = (st == nst - 1 ? 1 : 0) | (nh == 1 ? 2 : 0);
+            mbar_arrive_expect_tx(fb, (uint32_t)(nh * (kBM * 64 + BN * 64)));
+            tma_load_2d(sA + slot * C::kAStage, &tmA32, fb, ga * 32, g.m0);
+            tma_load_2d(sB + slot * C::kBStage, &tmB32, fb, ga * 32, g.n0);
+            if (nh == 2) {
+              tma_load_2d(sA + slot * C::kAStage + kBM * 64, &tmA32, fb, gb * 32, g.m0);
+              tma_load_2d(sB + slot * C::kBStage + BN * 64, &tmB32, fb, gb * 32, g.n0);
+            }
+            ++st;
+            ++it;
+            if (++slot == S) {
+              slot = 0;
+              ph ^= 1u;
+            }
+            return true;
+          };
+          if (cnt == 0) {
+            ok = issue(g0, -1);
+          } else {
+            for (int wd = g0 >> 5; wd <= (g1 - 1) >> 5 && ok; ++wd) {
+              uint32_t bits = s_kbits[wd];
+              while (bits && ok) {
+                const int gi = wd * 32 + __ffs(bits) - 1;
+                bits &= bits - 1u;
+                if (pend < 0) {
+                  pend = gi;
+                } else {
+                  ok = issue(pend, gi);
+                  pend = -1;
+                }
+              }
+            }
+            if (ok && pend >= 0) ok = issue(pend, -1);
+          }
+        }
+      } else if (p.conv != 1) {
         if (r == 0) {
           // The issuing lane is slow at anything but issuing: ring slot, phase
           // and the (tap, channel block) of each K block advance incrementally,
@@ -517,9 +589,32 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           tc_fence_after();
-          const bool last = stage_last[slot] != 0;
+          const int sflags = stage_last[slot];
+          const bool last = (sflags & 1) != 0;
           const uint32_t a = sA + slot * C::kAStage;
           const uint32_t bb = sB + slot * C::kBStage;
+          if (compact) {
+            // one or two 32-column groups, each 128 (A) / BN (B) rows of 64
+            // bytes with the 64-byte swizzle: two k-steps of 16 per group
+            const uint64_t a0 = smem_desc_sw64(a), b0 = smem_desc_sw64(bb);
+            if (first) tc_mma_bf16(d, a0, b0, idesc, 0u);
+            else tc_mma_bf16(d, a0, b0, idesc, 1u);
+            tc_mma_bf16(d, a0 + 2, b0 + 2, idesc, 1u);
+            if (!(sflags & 2)) {
+              const uint64_t a1 = smem_desc_sw64(a + kBM * 64), b1 = smem_desc_sw64(bb + BN * 64);
+              tc_mma_bf16(d, a1, b1, idesc, 1u);
+              tc_mma_bf16(d, a1 + 2, b1 + 2, idesc, 1u);
+            }
+            first = false;
+            tc_commit(bar_empty + 8 * slot);
+            ++it;
+            if (++slot == S) {
+              slot = 0;
+              ph ^= 1u;
+            }
+            if (last) break;
+            continue;
+          }
           // k-steps advance the start-address field by 32 B (2 units); the
           // accumulate flags are constants on both branches (a per-MMA flag
           // computed at run time roughly halves the issue rate)
@@ -937,13 +1032,14 @@ bool make_tmap_nhwc(CUtensorMap* m, const void* base, int n, int h, int w, int c
 
 template <int BN, int BK>
 cudaError_t launch_cfg(const IgemmArgs& a, const CUtensorMap& tA, const CUtensorMap& tB,
-                       const CUtensorMap& tY, int64_t tiles, cudaStream_t s) {
+                       const CUtensorMap& tY, const CUtensorMap& tA32, const CUtensorMap& tB32,
+                       int64_t tiles, cudaStream_t s) {
   cudaError_t e0 = smem_optin(reinterpret_cast<const void*>(igemm_kernel<BN, BK>), (size_t)Cfg<BN, BK>::kSmem);
   if (e0 != cudaSuccess) return e0;
   const int64_t units = tiles * (a.ksplit > 1 ? a.ksplit : 1);
   const int64_t grid = units < device_sm_count() ? units : device_sm_count();
   cudaError_t e = launch_kernel(igemm_kernel<BN, BK>, dim3((unsigned)grid), dim3(kThreads),
-                                (size_t)Cfg<BN, BK>::kSmem, s, tA, tB, tY, a);
+                                (size_t)Cfg<BN, BK>::kSmem, s, tA, tB, tY, tA32, tB32, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
@@ -1056,20 +1152,27 @@ cudaError_t launch_igemm(const IgemmArgs& a_in, cudaStream_t s) {
     if (!okY) return cudaErrorInvalidValue;
   }
   if (a.conv == 1) tA = tB;  // unused by the gather producers
+  // 32-column boxes (64-byte swizzle) of the compacted zero-skip GEMM
+  CUtensorMap tA32 = tB, tB32 = tB;
+  if (a.conv == 0 && bk == 64) {
+    if (!make_tmap_2d(&tA32, a.x, (uint64_t)a.M, (uint64_t)a.Ktot, 32, kBM) ||
+        !make_tmap_2d(&tB32, a.w, (uint64_t)a.N, (uint64_t)a.Ktot, 32, (uint32_t)bn))
+      return cudaErrorInvalidValue;
+  }
   const int64_t tiles = mtiles * ((a.N + bn - 1) / bn);
   if (bk == 64) {
     switch (bn) {
-      case 64: return launch_cfg<64, 64>(a, tA, tB, tY, tiles, s);
-      case 128: return launch_cfg<128, 64>(a, tA, tB, tY, tiles, s);
-      case 192: return launch_cfg<192, 64>(a, tA, tB, tY, tiles, s);
-      default: return launch_cfg<256, 64>(a, tA, tB, tY, tiles, s);
+      case 64: return launch_cfg<64, 64>(a, tA, tB, tY, tA32, tB32, tiles, s);
+      case 128: return launch_cfg<128, 64>(a, tA, tB, tY, tA32, tB32, tiles, s);
+      case 192: return launch_cfg<192, 64>(a, tA, tB, tY, tA32, tB32, tiles, s);
+      default: return launch_cfg<256, 64>(a, tA, tB, tY, tA32, tB32, tiles, s);
     }
   }
   switch (bn) {
-    case 64: return launch_cfg<64, 32>(a, tA, tB, tY, tiles, s);
-    case 128: return launch_cfg<128, 32>(a, tA, tB, tY, tiles, s);
-    case 192: return launch_cfg<192, 32>(a, tA, tB, tY, tiles, s);
-    default: return launch_cfg<256, 32>(a, tA, tB, tY, tiles, s);
+    case 64: return launch_cfg<64, 32>(a, tA, tB, tY, tA32, tB32, tiles, s);
+    case 128: return launch_cfg<128, 32>(a, tA, tB, tY, tA32, tB32, tiles, s);
+    case 192: return launch_cfg<192, 32>(a, tA, tB, tY, tA32, tB32, tiles, s);
+    default: return launch_cfg<256, 32>(a, tA, tB, tY, tA32, tB32, tiles, s);
   }
 }
 
