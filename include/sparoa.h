@@ -222,6 +222,23 @@ sparoa_status sparoa_set_overlap(sparoa_ctx *ctx, int32_t enable);
 /* Wait for the stream; report (and clear) a device-side timeout. */
 sparoa_status sparoa_sync(sparoa_ctx *ctx);
 
+/* Testing hooks for the failure paths (the paper has no counterpart).
+ *
+ * sparoa_set_wait_limit: SM clock cycles after which a tensor-core kernel's
+ * bounded waits give up (0 = the default, about a second).  A wait that runs
+ * out records an error bit in the context and lets every CTA unwind: it waits
+ * (bounded again) for the copies and MMAs it already issued, frees its tensor
+ * memory and exits; the next synchronising call returns SPAROA_ERR_TIMEOUT and
+ * the context stays usable.
+ * sparoa_set_fault: 1 = the tensor-core kernels' MMA issuer withholds its
+ * signal for the first accumulator of each CTA until the code is set back to
+ * 0, so that the epilogue's bounded wait runs out (no fault, trap or endless
+ * loop on the GPU); 2 = the next workspace allocation of the context fails
+ * (SPAROA_ERR_OOM), once; 0 = off.
+ * Errors: INVALID_ARG (ctx NULL, negative cycles, unknown code). */
+sparoa_status sparoa_set_wait_limit(sparoa_ctx *ctx, int64_t cycles);
+sparoa_status sparoa_set_fault(sparoa_ctx *ctx, int32_t code);
+
 /* Static description of a status code. */
 const char *sparoa_status_str(sparoa_status s);
 

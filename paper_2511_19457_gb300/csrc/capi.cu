@@ -87,6 +87,8 @@ struct sparoa_ctx {
   DevBuf splitk;      // split-K arrival counters (kept zero) + fp32 partial tiles
   std::vector<sparoa_occupancy> graph_occ;
   int overlap = 1;    // programmatic dependent launch between consecutive kernels
+  int64_t wait_limit = 0;  // SM cycles before a kernel's bounded wait gives up (0: default)
+  int fault = 0;           // error-path tests: 1 MMA signal withheld, 2 next allocation fails
   cudaStream_t aux = nullptr;                        // second stream of split execution
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;  // its fork / join with `stream`
   uint32_t* d_err() const { return reinterpret_cast<uint32_t*>(small.p); }
@@ -144,6 +146,10 @@ struct DeviceGuard {
 
 sparoa_status ensure(sparoa_ctx* ctx, DevBuf& b, size_t bytes) {
   if (bytes <= b.bytes) return SPAROA_OK;
+  if (ctx->fault == 2) {  // injected for the error-path tests: this allocation fails, once
+    ctx->fault = 0;
+    return fail(ctx, SPAROA_ERR_OOM, "workspace allocation of %zu bytes failed (injected)", bytes);
+  }
   if (b.p) {
     SP_CUDA(cudaStreamSynchronize(ctx->stream));
     cudaFree(b.p);
@@ -518,6 +524,8 @@ sparoa_status run_gemm(sparoa_ctx* ctx, const GemmPlan& g, cudaStream_t stream, 
     a.out_occ = yo;
     a.emit = g.yo ? 1 : 0;
     a.err = ctx->d_err();
+    a.wait_limit = ctx->wait_limit;
+    a.fault = ctx->fault == 1 ? kFaultSkipFirstAccCommit : 0;
     SP_TRY(offer_splitk(ctx, &a, ws_slot));
     SP_CUDA(launch_igemm(a, stream));
   }
@@ -569,6 +577,8 @@ sparoa_status run_conv(sparoa_ctx* ctx, const ConvPlan& c) {
   if (c.yo) a.out_occ = to_dev(*c.yo);
   a.emit = c.yo ? 1 : 0;
   a.err = ctx->d_err();
+  a.wait_limit = ctx->wait_limit;
+  a.fault = ctx->fault == 1 ? kFaultSkipFirstAccCommit : 0;
   if (!pointwise && conv3_supported(a)) {
     SP_CUDA(launch_conv3(a, ctx->stream));
     return SPAROA_OK;
@@ -682,6 +692,18 @@ sparoa_status sparoa_set_overlap(sparoa_ctx* ctx, int32_t enable) {
 sparoa_status sparoa_set_stream(sparoa_ctx* ctx, void* stream) {
   if (!ctx) return SPAROA_ERR_INVALID_ARG;
   ctx->stream = static_cast<cudaStream_t>(stream);
+  return SPAROA_OK;
+}
+
+sparoa_status sparoa_set_wait_limit(sparoa_ctx* ctx, int64_t cycles) {
+  if (!ctx || cycles < 0) return SPAROA_ERR_INVALID_ARG;
+  ctx->wait_limit = cycles;
+  return SPAROA_OK;
+}
+
+sparoa_status sparoa_set_fault(sparoa_ctx* ctx, int32_t code) {
+  if (!ctx || code < 0 || code > 2) return SPAROA_ERR_INVALID_ARG;
+  ctx->fault = code;
   return SPAROA_OK;
 }
 

@@ -195,9 +195,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t bar_accf = sCtl + 104;
   const uint32_t bar_acce = sCtl + 120;
   const uint32_t bar_mask = sCtl + 136;
+  const uint32_t bar_drain = sCtl + 168;  // after an abort: the MMAs issued so far are done
   volatile int* s_abort = reinterpret_cast<volatile int*>(ctl + 152);
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(ctl + 156);
   uint32_t* s_tapm = reinterpret_cast<uint32_t*>(ctl + 160);          // [2] 9-bit occupied-tap masks
+  int* s_slabs = reinterpret_cast<int*>(ctl + 176);                    // slabs issued (drain after an abort)
   uint8_t* s_rowf = ctl + 256;                                         // [3][2][128] row has a non-zero
   float* s_scale = reinterpret_cast<float*>(ctl + 1024);              // [CO]
   float* s_shift = s_scale + CO;                                       // [CO]
@@ -208,10 +210,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int tiles = N * G.tiles_per_img;
   uint32_t* const err = P.err;
   const int emit = P.emit;
+  const long long wlim = P.wait_limit > 0 ? P.wait_limit : kWaitLimitCycles;
 
   // on-chip prologue, overlapping the previous grid on the stream
   if (threadIdx.x == 0) {
     mbar_init(bar_w, 1u);
+    mbar_init(bar_drain, 1u);
     for (int b = 0; b < 2; ++b) {
       mbar_init(bar_full + 8 * b, 1u);
       mbar_init(bar_mask + 8 * b, 1u);
@@ -257,9 +261,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // -------------------------------------------------------------- slab loads
     if (lane == 0) {
       int j = 1;
+      *s_slabs = t_first < tiles ? 1 : 0;  // the first went out in the prologue
       for (int t = blockIdx.x + gridDim.x; t < tiles; t += gridDim.x, ++j) {
         const int b = j & 1;
-        if (!mbar_wait(bar_empty + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutEmpty))
+        if (!mbar_wait(bar_empty + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutEmpty, wlim))
           break;
         const int img = t / G.tiles_per_img;
         const int oh0 = (t - img * G.tiles_per_img) * kBM / Wp;
@@ -267,6 +272,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_arrive_expect_tx(bar_full + 8 * b, (uint32_t)(C / 64 * 128 * Wp * G.R));
         for (int cb = 0; cb < C / 64; ++cb)
           tma_load_4d(dst + (uint32_t)(cb * G.chunk_stride), &tmX, bar_full + 8 * b, cb * 64, -1, oh0 - 1, img);
+        *s_slabs = j + 1;
       }
     }
   } else if (warp == 1) {
@@ -279,7 +285,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // mask buffer b was read by the MMA issue of tile j - 2, before that
         // tile's commit to the slab-empty barrier
         if (lane == 0 && j >= 2)
-          ok = mbar_wait(bar_empty + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutEmpty);
+          ok = mbar_wait(bar_empty + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutEmpty, wlim);
         if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) break;
         const uint32_t m = conv3_tap_mask(G, P.in_blk, P.in_C32, t, lane);
         if (lane == 0) {
@@ -295,9 +301,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++j) {
         const int b = j & 1;
-        ok = mbar_wait_spin(bar_acce + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutAcc) &&
-             mbar_wait_spin(bar_full + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutFull) &&
-             (!skip || mbar_wait_spin(bar_mask + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutFull));
+        ok = mbar_wait_spin(bar_acce + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutAcc, wlim) &&
+             mbar_wait_spin(bar_full + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutFull, wlim) &&
+             (!skip || mbar_wait_spin(bar_mask + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutFull, wlim));
         if (!ok) break;
         tc_fence_after();
         const int q0 = (t - (t / G.tiles_per_img) * G.tiles_per_img) * kBM;
@@ -310,18 +316,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint64_t bdesc0 = smem_desc_kmajor<64>(sW);
         const uint32_t tapmask = skip ? s_tapm[b] : 0x1FFu;
         if (j == 0) {
-          ok = mbar_wait_spin(bar_w, 0u, err, s_abort, kErrTimeoutFull);
+          ok = mbar_wait_spin(bar_w, 0u, err, s_abort, kErrTimeoutFull, wlim);
           if (!ok) break;
           tc_fence_after();
         }
         conv3_issue<CO>(d, adesc0, bdesc0, Wp, tapmask);
         tc_commit(bar_empty + 8 * b);  // slab and mask buffer free once these MMAs are done
-        tc_commit(bar_accf + 8 * b);
+        // (the fault injection of the error-path tests leaves the first
+        // accumulator unsignalled: the epilogue's bounded wait runs out)
+        if (!(P.fault == kFaultSkipFirstAccCommit && j == 0)) tc_commit(bar_accf + 8 * b);
       }
       // TMEM is freed below only after the epilogue has read the last two
       // accumulators (the waits a further two tiles would make)
       for (int k = 0; k < 2 && ok; ++k, ++j)
-        ok = mbar_wait(bar_acce + 8 * (j & 1), (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutAcc);
+        ok = mbar_wait(bar_acce + 8 * (j & 1), (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutAcc, wlim);
     }
   } else if (warp >= 4) {
     // -------------------------------------------------------------- epilogue
@@ -363,7 +371,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int oh = qq / Wp, ow = qq - (qq / Wp) * Wp;
       const bool mvalid = oh < H && ow < W;
       const int64_t m = ((int64_t)img * H + oh) * W + ow;
-      const bool ok = mbar_wait(bar_accf + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutAcc);
+      const bool ok = mbar_wait(bar_accf + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutAcc, wlim);
       // the pair agrees on an abort, and the row flags of the previous tile
       // (written before this barrier by both warps) can be combined after it
       if (named_bar_or(pair_bar, 64, !ok)) break;
@@ -464,6 +472,24 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncwarp();  // lanes that finished early wait for their warp's working lane
   tc_fence_before();
   __syncthreads();
+  if (*s_abort) {
+    // a bounded wait ran out: before shared and tensor memory are released,
+    // the weights and the last slab of each buffer have landed and the MMAs
+    // issued so far are done (each wait bounded again)
+    if (threadIdx.x == 0 && t_first < tiles) {
+      mbar_drain(bar_w, 0u, wlim);
+      const int n = *s_slabs;
+      for (int k = 0; k < 2 && k < n; ++k) {
+        const int i = n - 1 - k;
+        mbar_drain(bar_full + 8 * (i & 1), (uint32_t)((i >> 1) & 1), wlim);
+      }
+    }
+    if (warp == kMmaWarp && lane == 0) {
+      tc_commit(bar_drain);
+      mbar_drain(bar_drain, 0u, wlim);
+    }
+    __syncthreads();
+  }
   if (warp == kMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, (uint32_t)(2 * CO));

@@ -69,7 +69,7 @@ struct Cfg {
   // 40 KB stage (4096 x 3072 x 768: 26.1 -> 22.3 us).  kFixed is everything
   // but the ring (barriers and flags of at most 12 stages) plus the 1024 bytes
   // of alignment slack.
-  static constexpr int kFixed = 2 * kStgBytes + (2 * 12 + 4) * 8 + (12 + 8) * 4 + 16 + kMaxKWords * 4 +
+  static constexpr int kFixed = 2 * kStgBytes + (2 * 12 + 5) * 8 + (12 + 8) * 4 + 16 + kMaxKWords * 4 +
                                 kMaxTaps * 8 + 4 * BN * 4 + 4 * BN * 4 + kMaxAccCols * 4 + kBM * 8 +
                                 (BN / 32) * 4 + 16 + 1024;
   static constexpr int kBudget =
@@ -81,7 +81,7 @@ struct Cfg {
   static constexpr int kBOff = kAOff + kStages * kAStage;
   static constexpr int kStgOff = kBOff + kStages * kBStage;          // 1024-aligned
   static constexpr int kBarOff = kStgOff + 2 * kStgBytes;
-  static constexpr int kNumBars = 2 * kStages + 4;                   // full, empty, accf[2], acce[2]
+  static constexpr int kNumBars = 2 * kStages + 5;                   // full, empty, accf[2], acce[2], drain
   static constexpr int kFlagOff = kBarOff + kNumBars * 8;
   static constexpr int kKBitsOff = (kFlagOff + (kStages + 8) * 4 + 15) & ~15;
   static constexpr int kTapOff = kKBitsOff + kMaxKWords * 4;
@@ -218,6 +218,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const __nv_bfloat16* const residual = P.ep.residual;
   const int y_f32 = P.y_f32;
   const int emit = P.emit;
+  const long long wlim = P.wait_limit > 0 ? P.wait_limit : kWaitLimitCycles;
   const __nv_bfloat16* const xin = P.x;
   const uint32_t* const in_blk = P.in_blk;
   const int in_C32 = P.in_C32;
@@ -237,10 +238,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t bar_empty = bar_full + 8 * S;   // + 8*s
   const uint32_t bar_accf = bar_empty + 8 * S;   // + 8*b
   const uint32_t bar_acce = bar_accf + 16;       // + 8*b
+  const uint32_t bar_drain = bar_acce + 16;      // after an abort: the MMAs issued so far are done
   int* flags = reinterpret_cast<int*>(smem + C::kFlagOff);
   int* stage_last = flags;                // [S]: 1 = last stage of its tile
   volatile int* s_abort = flags + S;      // CTA-wide abort request
   volatile int* s_last = flags + S + 2;   // [2] split K: this unit finishes its tile
+  int* s_issued = flags + S + 4;          // stages the producer filled (for the drain after an abort)
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(flags + S + 1);
   uint32_t* s_kbits = reinterpret_cast<uint32_t*>(smem + C::kKBitsOff);
   unsigned long long* s_tap = reinterpret_cast<unsigned long long*>(smem + C::kTapOff);
@@ -286,6 +289,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(bar_accf + 8 * b, 1u);
       mbar_init(bar_acce + 8 * b, (uint32_t)kEpiThreads);
     }
+    mbar_init(bar_drain, 1u);
     *s_abort = 0;
     fence_mbar_init();
     if (p.conv != 1) prefetch_tmap(&tmA);
@@ -438,7 +442,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint32_t ph = (uint32_t)((it / S) & 1);
           int st = 0, pend = -1;
           auto issue = [&](int ga, int gb) -> bool {
-            if (it >= S && !mbar_wait(bar_empty + 8 * slot, ph ^ 1u, err, s_abort, kErrTimeoutEmpty)) return false;
+            if (it >= S && !mbar_wait(bar_empty + 8 * slot, ph ^ 1u, err, s_abort, kErrTimeoutEmpty, wlim)) return false;
             const uint32_t fb = bar_full + 8 * slot;
             const int nh = gb >= 0 ? 2 : 1;
             stage_last[slot] = (st == nst - 1 ? 1 : 0) | (nh == 1 ? 2 : 0);
@@ -491,7 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool issue =
                 !(skip && kb != last && kb < kMaxKWords * 32 && !((s_kbits[kb >> 5] >> (kb & 31)) & 1u));
             if (issue) {
-              if (it >= S && !mbar_wait(eb0 + 8 * slot, ph ^ 1u, err, s_abort, kErrTimeoutEmpty)) {
+              if (it >= S && !mbar_wait(eb0 + 8 * slot, ph ^ 1u, err, s_abort, kErrTimeoutEmpty, wlim)) {
                 ok = false;
                 break;
               }
@@ -528,7 +532,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             continue;
           const int slot = it % S;
           const uint32_t ph = (uint32_t)((it / S) & 1);
-          if (!mbar_wait(bar_empty + 8 * slot, ph ^ 1u, err, s_abort, kErrTimeoutEmpty)) {
+          if (!mbar_wait(bar_empty + 8 * slot, ph ^ 1u, err, s_abort, kErrTimeoutEmpty, wlim)) {
             ok = false;
             break;
           }
@@ -562,6 +566,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+    if (r == 0) *s_issued = it;  // stages this CTA filled (TMA copies issued)
     if (p.conv == 1) {
       cp_async_wait<0>();
       fence_proxy_async_smem();
@@ -576,7 +581,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++j) {
         const int b = j & 1;
         if (!mbar_wait(bar_acce + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort,
-                       kErrTimeoutAcc))
+                       kErrTimeoutAcc, wlim))
           break;
         tc_fence_after();
         const uint32_t d = tmem + (uint32_t)b * C::kAccCols;
@@ -584,7 +589,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         int slot = it % S;
         uint32_t ph = (uint32_t)((it / S) & 1);
         while (true) {
-          if (!mbar_wait(bar_full + 8 * slot, ph, err, s_abort, kErrTimeoutFull)) {
+          if (!mbar_wait(bar_full + 8 * slot, ph, err, s_abort, kErrTimeoutFull, wlim)) {
             ok = false;
             break;
           }
@@ -638,7 +643,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (last) break;
         }
-        if (ok) tc_commit(bar_accf + 8 * b);
+        // (the fault injection of the error-path tests leaves the first
+        // accumulator unsignalled: the epilogue's bounded wait runs out)
+        if (ok && !(P.fault == kFaultSkipFirstAccCommit && j == 0)) tc_commit(bar_accf + 8 * b);
       }
     }
   } else {
@@ -685,7 +692,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         scb[c] = sc;
         shb[c] = sh;
       }
-      const bool ok = mbar_wait(bar_accf + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutAcc);
+      const bool ok = mbar_wait(bar_accf + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutAcc, wlim);
       // publishes the affine, and makes the abort decision the same for every
       // epilogue warp (a warp that left alone would strand the others at a barrier)
       if (named_bar_or(2, kEpiThreads, !ok)) break;
@@ -971,6 +978,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncwarp();  // lanes that finished early wait for their warp's working lane
   tc_fence_before();
   __syncthreads();
+  if (*s_abort) {
+    // a bounded wait ran out: before shared and tensor memory are released,
+    // the copies into the last stage of every ring slot have landed and the
+    // MMAs issued so far are done (each wait bounded again)
+    if (threadIdx.x == 0) {
+      const int issued = *s_issued;
+      for (int k = 0; k < S && k < issued; ++k) {
+        const int i = issued - 1 - k;
+        mbar_drain(bar_full + 8 * (i % S), (uint32_t)((i / S) & 1), wlim);
+      }
+    }
+    if (warp == kMmaWarp && lane == 0) {
+      tc_commit(bar_drain);
+      mbar_drain(bar_drain, 0u, wlim);
+    }
+    __syncthreads();
+  }
   if (warp == kMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, C::kTmemCols);

@@ -17,7 +17,8 @@
 
 namespace sparoa {
 
-// Bounded waits give up after about a second of SM clock cycles.
+// Bounded waits give up after about a second of SM clock cycles (the default;
+// a context can set another limit, which its kernels receive as a parameter).
 constexpr long long kWaitLimitCycles = 1ll << 31;
 
 enum ErrBits : uint32_t {
@@ -127,18 +128,19 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parit
 
 // Wait for the phase with the given parity to complete.  Waiting threads are
 // suspended by the hardware between polls (woken when the phase completes);
-// the cycle counter and the CTA abort flag are checked every 16 polls.  Gives up after kWaitLimitCycles
-// or once another role of the CTA raised *abort; then it records `bit` in
-// *err, raises *abort and returns false.
+// the cycle counter and the CTA abort flag are checked every 16 polls.  Gives
+// up after `limit` cycles (then it records `bit` in *err and raises *abort) or
+// once another role of the CTA raised *abort; either way it returns false.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t* err,
-                                          volatile int* abort, uint32_t bit) {
+                                          volatile int* abort, uint32_t bit,
+                                          long long limit = kWaitLimitCycles) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   for (uint32_t n = 1;; ++n) {
     if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
     if ((n & 15u) == 0u) {
       if (*abort) return false;
-      if (clock64() - t0 > kWaitLimitCycles) {
+      if (clock64() - t0 > limit) {
         atomicOr(err, bit);
         *abort = 1;
         return false;
@@ -164,14 +166,15 @@ __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
 // polls without being suspended between polls (a suspended thread is woken
 // some time after the phase completes), with the same limit and abort rule.
 __device__ __forceinline__ bool mbar_wait_spin(uint32_t bar, uint32_t parity, uint32_t* err,
-                                               volatile int* abort, uint32_t bit) {
+                                               volatile int* abort, uint32_t bit,
+                                               long long limit = kWaitLimitCycles) {
   if (mbar_test_wait(bar, parity)) return true;
   const long long t0 = clock64();
   for (uint32_t n = 1;; ++n) {
     if (mbar_test_wait(bar, parity)) return true;
     if ((n & 255u) == 0u) {
       if (*abort) return false;
-      if (clock64() - t0 > kWaitLimitCycles) {
+      if (clock64() - t0 > limit) {
         atomicOr(err, bit);
         *abort = 1;
         return false;
@@ -179,6 +182,24 @@ __device__ __forceinline__ bool mbar_wait_spin(uint32_t bar, uint32_t parity, ui
     }
   }
 }
+
+// After an abort: wait, at most `limit` cycles and whatever the abort flag
+// says, for a phase that asynchronous work already issued by this CTA (TMA
+// copies into its shared memory, MMAs into its tensor memory) completes, so
+// that the CTA does not release those resources while they are written.
+__device__ __forceinline__ bool mbar_drain(uint32_t bar, uint32_t parity, long long limit) {
+  if (mbar_test_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  for (uint32_t n = 1;; ++n) {
+    if (mbar_try_wait_sleep(bar, parity, 2000u)) return true;
+    if ((n & 15u) == 0u && clock64() - t0 > limit) return false;
+  }
+}
+
+// Fault injection for tests of the error paths (IgemmArgs::fault): the MMA
+// issuer never signals the first accumulator, so the epilogue's bounded wait
+// runs out and the call reports a timeout.
+constexpr int kFaultSkipFirstAccCommit = 1;
 
 // ---------------------------------------------------------------------------
 // TMA and cp.async

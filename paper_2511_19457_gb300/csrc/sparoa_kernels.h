@@ -72,6 +72,8 @@ struct IgemmArgs {
   OccDev out_occ{};
   int emit = 0;
   uint32_t* err = nullptr;
+  long long wait_limit = 0;          // cycles before a bounded wait gives up (0: the default)
+  int fault = 0;                     // error-path tests: kFaultSkipFirstAccCommit or 0
   // split K (set by launch_igemm from the scratch offered here): fp32 partial
   // tiles [tiles][ksplit][128][BN] in `ws` (ws_bytes), one zeroed arrival
   // counter per output tile in `ws_cnt` (ws_cnt_len), left zero again

@@ -85,6 +85,8 @@ _sig("sparoa_set_overlap", [_P, _I32])
 _sig("sparoa_graph_workspace", [_P, _P, _I32, _I64, _I64, _I64, _I64, ctypes.POINTER(ctypes.c_uint64)])
 _sig("sparoa_gemm_split", [_P, _P, _I64, _I64, _P, _P, _I64, _P, ctypes.c_double, _P, _I32, _P, _P])
 _sig("sparoa_sync", [_P])
+_sig("sparoa_set_wait_limit", [_P, ctypes.c_int64])
+_sig("sparoa_set_fault", [_P, ctypes.c_int32])
 _lib.sparoa_status_str.restype = ctypes.c_char_p
 _lib.sparoa_status_str.argtypes = [ctypes.c_int]
 _lib.sparoa_last_error.restype = ctypes.c_char_p
@@ -112,6 +114,7 @@ _sig("sparoa_gemm_noalloc", [_P, _P, _I64, _I64, _P, _P, _I64, ctypes.POINTER(Ep
                              ctypes.POINTER(Thresholds), _P, _I32, ctypes.POINTER(Stats)])
 
 EXPORTED = ["sparoa_create", "sparoa_destroy", "sparoa_set_stream", "sparoa_set_overlap", "sparoa_sync",
+            "sparoa_set_wait_limit", "sparoa_set_fault",
             "sparoa_status_str", "sparoa_last_error", "sparoa_occupancy_bytes",
             "sparoa_occupancy_init", "sparoa_op_stats", "sparoa_gemm", "sparoa_conv2d",
             "sparoa_maxpool2d", "sparoa_avgpool_global", "sparoa_bn_act", "sparoa_run_graph",
@@ -174,6 +177,15 @@ class Context:
     def set_overlap(self, enable: bool):
         """Programmatic dependent launch between consecutive kernels (default on)."""
         self._check(_lib.sparoa_set_overlap(self.h, 1 if enable else 0))
+
+    def set_wait_limit(self, cycles: int):
+        """SM cycles before a kernel's bounded wait gives up (0 = default)."""
+        self._check(_lib.sparoa_set_wait_limit(self.h, int(cycles)))
+
+    def set_fault(self, code: int):
+        """Error-path tests: 1 = withhold the first accumulator signal
+        (timeout), 2 = fail the next workspace allocation, 0 = off."""
+        self._check(_lib.sparoa_set_fault(self.h, int(code)))
 
 
 class OccupancyBuffer:
