@@ -431,6 +431,315 @@ __global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloa
 }
 
 // ---------------------------------------------------------------------------
+// Streamed element-wise producers: the stats kernel's tile order and
+// occupancy scheme (contiguous runs of column-tile-major 128 x 64 tiles per
+// CTA, column counts in 16-bit register halves flushed once per run, row bits
+// by ballot, block-column masks OR-ed per warp) with the tile's values made
+// and stored first.  No barrier per tile; the next tile's loads are in flight
+// while a tile is transformed.
+struct StreamEmit {
+  uint32_t cnt[4];  // columns cg*8 + 2w (low half) and + 2w + 1 (high half)
+  int run_ct, run_tiles;
+};
+
+__device__ __forceinline__ void stream_flush(StreamEmit& e, uint32_t* s_cnt, const OccDev& o) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t c8[8];
+#pragma unroll
+  for (int w = 0; w < 4; ++w) {
+    c8[2 * w] = e.cnt[w] & 0xFFFFu;
+    c8[2 * w + 1] = e.cnt[w] >> 16;
+    e.cnt[w] = 0u;
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    c8[j] += __shfl_xor_sync(0xffffffffu, c8[j], 8);
+    c8[j] += __shfl_xor_sync(0xffffffffu, c8[j], 16);
+  }
+  if (lane < 8) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) s_cnt[warp * 64 + lane * 8 + j] = c8[j];
+  }
+  __syncthreads();
+  if (threadIdx.x < 64) {
+    uint32_t c = 0u;
+#pragma unroll
+    for (int w = 0; w < kTileThreads / 32; ++w) c += s_cnt[w * 64 + threadIdx.x];
+    if (c) atomicAdd(&o.col_nnz[e.run_ct * 64 + threadIdx.x], c);  // 0 for columns past C
+    uint32_t sum = c;
+#pragma unroll
+    for (int sh = 16; sh > 0; sh >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, sh);
+    if (lane == 0 && sum) {
+      atomicAdd(&o.tile_nnz[e.run_ct], sum);
+      atomicAdd(o.nnz, (unsigned long long)sum);
+    }
+  }
+  __syncthreads();
+}
+
+// n[i][w]: nz_pairs of word w of this thread's row i (0 outside the tensor).
+// Called by every thread with the same tile sequence.
+__device__ __forceinline__ void stream_tile(StreamEmit& e, const uint32_t (&n)[4][4], int ct, int64_t row0,
+                                            int64_t R, bool own_row, uint32_t* s_cnt, const OccDev& o) {
+  const int lane = threadIdx.x & 31, cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
+  if (ct != e.run_ct || e.run_tiles == kStatsRunTiles) {
+    stream_flush(e, s_cnt, o);
+    e.run_ct = ct;
+    e.run_tiles = 0;
+  }
+  ++e.run_tiles;
+  uint32_t o4[4];
+#pragma unroll
+  for (int w = 0; w < 4; ++w) {
+    e.cnt[w] += (n[0][w] + n[1][w]) + (n[2][w] + n[3][w]);
+    o4[w] = (n[0][w] | n[1][w]) | (n[2][w] | n[3][w]);
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t b = __ballot_sync(0xffffffffu, (n[i][0] | n[i][1] | n[i][2] | n[i][3]) != 0u);
+    const int64_t r = row0 + rs + 32 * i;
+    if ((lane & 7) == 0 && r < R) {
+      const bool nzr = ((b >> lane) & 0xFFu) != 0u;
+      if (own_row) o.row_bm[r] = nzr ? 1ull : 0ull;
+      else if (nzr) atomicOr(&o.row_bm[r * o.W64 + (ct >> 6)], 1ull << (ct & 63));
+    }
+  }
+  const uint32_t m8 = (o4[0] & 1u) | ((o4[0] >> 15) & 2u) | ((o4[1] << 2) & 4u) | ((o4[1] >> 13) & 8u) |
+                      ((o4[2] << 4) & 16u) | ((o4[2] >> 11) & 32u) | ((o4[3] << 6) & 64u) |
+                      ((o4[3] >> 9) & 128u);
+  uint32_t v = m8 << ((cg & 3) * 8);
+  v |= __shfl_xor_sync(0xffffffffu, v, 1);
+  v |= __shfl_xor_sync(0xffffffffu, v, 2);
+  v |= __shfl_xor_sync(0xffffffffu, v, 8);
+  v |= __shfl_xor_sync(0xffffffffu, v, 16);
+  if ((lane & 27) == 0 && v) {  // lanes 0 and 4
+    const int w = ct * 2 + (lane >> 2);
+    if (w < o.C32) atomicOr(&o.blk_mask[(row0 >> 7) * o.C32 + w], v);
+  }
+}
+
+// Stand-alone bias / batch norm / residual / activation over [R, C] (C % 8
+// == 0), y and its occupancy.
+__global__ void __launch_bounds__(kTileThreads, 2) bn_act_kernel(const __nv_bfloat16* __restrict__ x, int64_t R,
+                                                                 int C, EpiDev ep_param,
+                                                                 __nv_bfloat16* __restrict__ y, OccDev o_param,
+                                                                 int emit) {
+  const OccDev o = o_param;
+  const EpiDev ep = ep_param;
+  __shared__ uint32_t s_cnt[8 * 64];
+  const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
+  const int ctn = (C + 63) / 64;
+  const int64_t nrb = (R + 127) / 128;
+  const int64_t P = nrb * ctn;
+  const int64_t L0 = (int64_t)blockIdx.x * P / gridDim.x, L1 = ((int64_t)blockIdx.x + 1) * P / gridDim.x;
+  const bool own_row = ctn == 1;
+  const int ct0 = L0 < L1 ? (int)(L0 / nrb) : 0;
+  const int64_t rb0 = L0 - (int64_t)ct0 * nrb;
+  const __nv_bfloat16* const res = ep.residual;
+  pdl_wait();
+  pdl_trigger();
+  int64_t Ln = L0;
+  int l_ct = ct0;
+  int64_t l_rb = rb0;
+  auto load = [&](uint4 (&u)[4]) {
+    if (Ln < L1) {
+      const int64_t r0 = l_rb * 128 + rs;
+      const int c0 = l_ct * 64 + cg * 8;
+      const int64_t off = r0 * C + c0;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const bool ok = r0 + 32 * i < R && c0 < C;
+        u[i] = ok ? __ldg(reinterpret_cast<const uint4*>(x + off + 32 * i * (int64_t)C)) : make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
+    ++Ln;
+    if (++l_rb == nrb) {
+      l_rb = 0;
+      ++l_ct;
+    }
+  };
+  StreamEmit e;
+#pragma unroll
+  for (int w = 0; w < 4; ++w) e.cnt[w] = 0u;
+  e.run_ct = ct0;
+  e.run_tiles = 0;
+  int aff_ct = -1;
+  float sc[8], sh[8];
+  int t_ct = ct0;
+  int64_t t_rb = rb0;
+  auto tile = [&](uint4 (&u)[4]) {
+    const int ct = t_ct;
+    const int64_t row0 = t_rb * 128;
+    if (++t_rb == nrb) {
+      t_rb = 0;
+      ++t_ct;
+    }
+    const int c0 = ct * 64 + cg * 8;
+    if (ct != aff_ct) {  // the column affine of this thread's 8 columns
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        sc[j] = 1.f;
+        sh[j] = 0.f;
+        if (c0 + j < C) epi_affine(ep, C, c0 + j, sc[j], sh[j]);
+      }
+      aff_ct = ct;
+    }
+    uint4 ur[4];  // the residual rows, all in flight together
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int64_t r = row0 + rs + 32 * i;
+      ur[i] = (res && r < R && c0 < C) ? *reinterpret_cast<const uint4*>(res + r * C + c0) : make_uint4(0u, 0u, 0u, 0u);
+    }
+    uint32_t n[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int64_t r = row0 + rs + 32 * i;
+      float f[8], rv[8];
+      unpack8(u[i], f);
+      unpack8(ur[i], rv);
+      float v[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v[j] = epi_act(fmaf(f[j], sc[j], sh[j]) + rv[j], ep.act);
+      const uint4 pk = pack8(v);
+      const bool ok = r < R && c0 < C;
+      if (ok) *reinterpret_cast<uint4*>(y + r * C + c0) = pk;
+      n[i][0] = ok ? nz_pairs(pk.x) : 0u;
+      n[i][1] = ok ? nz_pairs(pk.y) : 0u;
+      n[i][2] = ok ? nz_pairs(pk.z) : 0u;
+      n[i][3] = ok ? nz_pairs(pk.w) : 0u;
+    }
+    load(u);  // the tile two ahead
+    if (emit) stream_tile(e, n, ct, row0, R, own_row, s_cnt, o);
+  };
+  uint4 ua[4], ub[4];
+  load(ua);
+  load(ub);
+  for (int64_t L = L0; L < L1; ++L) {
+    tile(ua);
+    if (++L >= L1) break;
+    tile(ub);
+  }
+  if (emit) stream_flush(e, s_cnt, o);
+}
+
+// k x k max pooling (C % 8 == 0), y [N, Ho, Wo, C] and its occupancy: per
+// output row and 8 channels, the window's taps are loaded together (addresses
+// clamped into the image; taps outside it count as -inf) and reduced with
+// packed bf16 maxima.
+__global__ void __launch_bounds__(kTileThreads, 3)
+    maxpool_kernel(const __nv_bfloat16* __restrict__ x, int N, int H, int W, int C, int k,
+                   int stride, int pad, int Ho, int Wo, __nv_bfloat16* __restrict__ y, OccDev o_param,
+                   int emit) {
+  const OccDev o = o_param;
+  __shared__ uint32_t s_cnt[8 * 64];
+  const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
+  const int64_t R = (int64_t)N * Ho * Wo;
+  const int ctn = (C + 63) / 64;
+  const int64_t nrb = (R + 127) / 128;
+  const int64_t P = nrb * ctn;
+  const int64_t L0 = (int64_t)blockIdx.x * P / gridDim.x, L1 = ((int64_t)blockIdx.x + 1) * P / gridDim.x;
+  const bool own_row = ctn == 1;
+  const int hw = Ho * Wo;
+  pdl_wait();
+  pdl_trigger();
+  StreamEmit e;
+#pragma unroll
+  for (int w = 0; w < 4; ++w) e.cnt[w] = 0u;
+  e.run_ct = L0 < L1 ? (int)(L0 / nrb) : 0;
+  e.run_tiles = 0;
+  const __nv_bfloat162 ninf = __halves2bfloat162(__ushort_as_bfloat16(0xFF80u), __ushort_as_bfloat16(0xFF80u));
+  for (int64_t L = L0; L < L1; ++L) {
+    const int ct = (int)(L / nrb);
+    const int64_t row0 = (L - (int64_t)ct * nrb) * 128;
+    const int c0 = ct * 64 + cg * 8;
+    uint32_t n[4][4];
+    uint4 outv[4];
+    bool okr[4];
+    if (k == 3) {
+      // two rows at a time: their 18 taps in flight together
+#pragma unroll
+      for (int i0 = 0; i0 < 4; i0 += 2) {
+        uint4 u[2][9];
+        uint32_t inb[2];
+#pragma unroll
+        for (int ii = 0; ii < 2; ++ii) {
+          const int i = i0 + ii;
+          const int64_t mrow = row0 + rs + 32 * i;
+          okr[i] = mrow < R && c0 < C;
+          const int mr = okr[i] ? (int)mrow : 0;
+          const int img = mr / hw, rem = mr - (mr / hw) * hw;
+          const int oh = rem / Wo, ow = rem - (rem / Wo) * Wo;
+          inb[ii] = 0u;
+#pragma unroll
+          for (int r = 0; r < 3; ++r) {
+            const int ih = oh * stride - pad + r;
+            const int ihc = ih < 0 ? 0 : (ih >= H ? H - 1 : ih);
+#pragma unroll
+            for (int s2 = 0; s2 < 3; ++s2) {
+              const int iw = ow * stride - pad + s2;
+              const int iwc = iw < 0 ? 0 : (iw >= W ? W - 1 : iw);
+              if (ih == ihc && iw == iwc) inb[ii] |= 1u << (r * 3 + s2);
+              u[ii][r * 3 + s2] = okr[i] ? __ldg(reinterpret_cast<const uint4*>(x + (((int64_t)img * H + ihc) * W + iwc) * C + c0))
+                                         : make_uint4(0u, 0u, 0u, 0u);
+            }
+          }
+        }
+#pragma unroll
+        for (int ii = 0; ii < 2; ++ii) {
+          __nv_bfloat162 m[4] = {ninf, ninf, ninf, ninf};
+#pragma unroll
+          for (int t = 0; t < 9; ++t) {
+            if (!((inb[ii] >> t) & 1u)) continue;
+            const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u[ii][t]);
+#pragma unroll
+            for (int w = 0; w < 4; ++w) m[w] = __hmax2(m[w], h[w]);
+          }
+          outv[i0 + ii] = make_uint4(*reinterpret_cast<uint32_t*>(&m[0]), *reinterpret_cast<uint32_t*>(&m[1]),
+                                     *reinterpret_cast<uint32_t*>(&m[2]), *reinterpret_cast<uint32_t*>(&m[3]));
+        }
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int64_t mrow = row0 + rs + 32 * i;
+        okr[i] = mrow < R && c0 < C;
+        __nv_bfloat162 m[4] = {ninf, ninf, ninf, ninf};
+        if (okr[i]) {
+          const int mr = (int)mrow;
+          const int img = mr / hw, rem = mr - (mr / hw) * hw;
+          const int oh = rem / Wo, ow = rem - (rem / Wo) * Wo;
+          for (int r = 0; r < k; ++r) {
+            const int ih = oh * stride - pad + r;
+            if (ih < 0 || ih >= H) continue;
+            for (int s2 = 0; s2 < k; ++s2) {
+              const int iw = ow * stride - pad + s2;
+              if (iw < 0 || iw >= W) continue;
+              const uint4 v = __ldg(reinterpret_cast<const uint4*>(x + (((int64_t)img * H + ih) * W + iw) * C + c0));
+              const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+              for (int w = 0; w < 4; ++w) m[w] = __hmax2(m[w], h[w]);
+            }
+          }
+        }
+        outv[i] = make_uint4(*reinterpret_cast<uint32_t*>(&m[0]), *reinterpret_cast<uint32_t*>(&m[1]),
+                             *reinterpret_cast<uint32_t*>(&m[2]), *reinterpret_cast<uint32_t*>(&m[3]));
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int64_t mrow = row0 + rs + 32 * i;
+      if (okr[i]) *reinterpret_cast<uint4*>(y + mrow * C + c0) = outv[i];
+      n[i][0] = okr[i] ? nz_pairs(outv[i].x) : 0u;
+      n[i][1] = okr[i] ? nz_pairs(outv[i].y) : 0u;
+      n[i][2] = okr[i] ? nz_pairs(outv[i].z) : 0u;
+      n[i][3] = okr[i] ? nz_pairs(outv[i].w) : 0u;
+    }
+    if (emit) stream_tile(e, n, ct, row0, R, own_row, s_cnt, o);
+  }
+  if (emit) stream_flush(e, s_cnt, o);
+}
+
+// ---------------------------------------------------------------------------
 __global__ void pad_kernel(const __nv_bfloat16* __restrict__ x, int64_t P, int C, int Cp,
                            __nv_bfloat16* __restrict__ y) {
   pdl_wait();
@@ -863,89 +1172,6 @@ __global__ void __launch_bounds__(kTileThreads) dw3_kernel(const DwArgs a_param,
 }
 
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kTileThreads)
-    maxpool_kernel(const __nv_bfloat16* __restrict__ x, int N, int H, int W, int C, int k,
-                   int stride, int pad, int Ho, int Wo, __nv_bfloat16* __restrict__ y, OccDev o_param,
-                   int emit) {
-  const OccDev o = o_param;
-  __shared__ uint32_t s_cnt[8 * 64];
-  extern __shared__ uint32_t s_acc[];  // [C] when acc (dynamic)
-  const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
-  const int64_t R = (int64_t)N * Ho * Wo;
-  const bool acc = emit && C <= kMaxAccCols;
-  acc_init(s_acc, C, acc);
-  pdl_wait();
-  pdl_trigger();
-  TileEmit e;
-  e.init();
-  SPAROA_TILE_LOOP(R, C) {
-    const int64_t row0 = (tile / ctn) * 128;
-    const int col0 = (int)(tile % ctn) * 64;
-    const int c0 = col0 + cg * 8;
-    for (int i = 0; i < 4; ++i) {
-      const int64_t mrow = row0 + rs + 32 * i;
-      uint32_t mask = 0;
-      if (mrow < R && c0 < C) {
-        const int hw = Ho * Wo;
-        const int img = (int)(mrow / hw);
-        const int rem = (int)(mrow - (int64_t)img * hw);
-        const int oh = rem / Wo, ow = rem - (rem / Wo) * Wo;
-        float mx[8];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) mx[j] = -INFINITY;
-        if (k == 3) {
-          // 3x3: the 9 loads unconditional (addresses clamped into the image,
-          // out-of-range taps left out of the max), all in flight together
-          uint4 u[9];
-          uint32_t inb = 0u;
-#pragma unroll
-          for (int r = 0; r < 3; ++r) {
-            const int ih = oh * stride - pad + r;
-            const int ihc = ih < 0 ? 0 : (ih >= H ? H - 1 : ih);
-#pragma unroll
-            for (int s = 0; s < 3; ++s) {
-              const int iw = ow * stride - pad + s;
-              const int iwc = iw < 0 ? 0 : (iw >= W ? W - 1 : iw);
-              if (ih == ihc && iw == iwc) inb |= 1u << (r * 3 + s);
-              u[r * 3 + s] = __ldg(reinterpret_cast<const uint4*>(x + (((int64_t)img * H + ihc) * W + iwc) * C + c0));
-            }
-          }
-#pragma unroll
-          for (int t = 0; t < 9; ++t) {
-            if (!((inb >> t) & 1u)) continue;
-            float f[8];
-            unpack8(u[t], f);
-#pragma unroll
-            for (int j = 0; j < 8; ++j)
-              if (f[j] > mx[j]) mx[j] = f[j];
-          }
-        } else {
-          for (int r = 0; r < k; ++r) {
-            const int ih = oh * stride - pad + r;
-            if (ih < 0 || ih >= H) continue;
-            for (int s = 0; s < k; ++s) {
-              const int iw = ow * stride - pad + s;
-              if (iw < 0 || iw >= W) continue;
-              float f[8];
-              unpack8(__ldg(reinterpret_cast<const uint4*>(x + (((int64_t)img * H + ih) * W + iw) * C + c0)), f);
-#pragma unroll
-              for (int j = 0; j < 8; ++j)
-                if (f[j] > mx[j]) mx[j] = f[j];
-            }
-          }
-        }
-        const uint4 u = pack8(mx);
-        *reinterpret_cast<uint4*>(y + mrow * C + c0) = u;
-        mask = nz_mask8(u);
-      }
-      if (emit) e.row(mask, mrow, col0, o);
-    }
-    if (emit) e.tile_done(row0, col0, o, s_cnt, s_acc, acc);
-  }
-  if (emit) cta_done(o, s_acc, acc);
-}
-
-// ---------------------------------------------------------------------------
 // Global average pooling [N, HW, C] -> [N, C] (C % 8 == 0): one CTA per (image,
 // 64-channel slice).  Lane l of warp w sums pixels 4 w + l / 8 + 32 k of the 8
 // channels 8 (l % 8) .. + 7, so every load of the CTA is in flight at once;
@@ -1007,52 +1233,6 @@ __global__ void __launch_bounds__(kTileThreads)
       }
     }
   }
-}
-
-// ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kTileThreads)
-    bn_act_kernel(const __nv_bfloat16* __restrict__ x, int64_t R, int C, EpiDev ep_param,
-                  __nv_bfloat16* __restrict__ y, OccDev o_param, int emit) {
-  const OccDev o = o_param;
-  const EpiDev ep = ep_param;
-  __shared__ uint32_t s_cnt[8 * 64];
-  extern __shared__ uint32_t s_acc[];  // [C] when acc (dynamic)
-  const int cg = threadIdx.x & 7, rs = threadIdx.x >> 3;
-  const bool acc = emit && C <= kMaxAccCols;
-  acc_init(s_acc, C, acc);
-  pdl_wait();
-  pdl_trigger();
-  TileEmit e;
-  e.init();
-  SPAROA_TILE_LOOP(R, C) {
-    const int64_t row0 = (tile / ctn) * 128;
-    const int col0 = (int)(tile % ctn) * 64;
-    const int c0 = col0 + cg * 8;
-    float sc[8], sh[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      sc[j] = 1.f;
-      sh[j] = 0.f;
-      if (c0 < C) epi_affine(ep, C, c0 + j, sc[j], sh[j]);
-    }
-    for (int i = 0; i < 4; ++i) {
-      const int64_t r = row0 + rs + 32 * i;
-      uint32_t mask = 0;
-      if (r < R && c0 < C) {
-        float f[8], rv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        unpack8(__ldg(reinterpret_cast<const uint4*>(x + r * C + c0)), f);
-        if (ep.residual) unpack8(*reinterpret_cast<const uint4*>(ep.residual + r * C + c0), rv);
-#pragma unroll
-        for (int j = 0; j < 8; ++j) f[j] = epi_act(fmaf(f[j], sc[j], sh[j]) + rv[j], ep.act);
-        const uint4 u = pack8(f);
-        *reinterpret_cast<uint4*>(y + r * C + c0) = u;
-        mask = nz_mask8(u);
-      }
-      if (emit) e.row(mask, r, col0, o);
-    }
-    if (emit) e.tile_done(row0, col0, o, s_cnt, s_acc, acc);
-  }
-  if (emit) cta_done(o, s_acc, acc);
 }
 
 // Dynamic shared memory of a tile kernel: the per-CTA column counters.
@@ -1167,7 +1347,10 @@ cudaError_t launch_maxpool(const __nv_bfloat16* x, int N, int H, int W, int C, i
                            cudaStream_t s) {
   const int64_t R = (int64_t)N * Ho * Wo;
   if (R <= 0) return cudaSuccess;
-  return launch_kernel(maxpool_kernel, dim3(tile_grid(R, C)), dim3(kTileThreads), acc_smem(emit, C),
+  if (C % 8) return cudaErrorInvalidValue;
+  const int64_t tiles = ((R + 127) / 128) * ((C + 63) / 64);
+  const int64_t cap = 3LL * device_sm_count();  // the resident CTAs split the tiles
+  return launch_kernel(maxpool_kernel, dim3((unsigned)(tiles < cap ? tiles : cap)), dim3(kTileThreads), 0,
                        s, x, N, H, W, C, k, stride, pad, Ho, Wo, y, o, emit);
 }
 
@@ -1184,7 +1367,10 @@ cudaError_t launch_avgpool(const __nv_bfloat16* x, int N, int HW, int C, __nv_bf
 cudaError_t launch_bn_act(const __nv_bfloat16* x, int64_t R, int C, const EpiDev& ep,
                           __nv_bfloat16* y, const OccDev& o, int emit, cudaStream_t s) {
   if (R <= 0) return cudaSuccess;
-  return launch_kernel(bn_act_kernel, dim3(tile_grid(R, C)), dim3(kTileThreads), acc_smem(emit, C),
+  if (C % 8) return cudaErrorInvalidValue;
+  const int64_t tiles = ((R + 127) / 128) * ((C + 63) / 64);
+  const int64_t cap2 = 2LL * device_sm_count();  // the resident CTAs (two per SM) split the tiles
+  return launch_kernel(bn_act_kernel, dim3((unsigned)(tiles < cap2 ? tiles : cap2)), dim3(kTileThreads), 0,
                        s, x, R, C, ep, y, o, emit);
 }
 
