@@ -48,7 +48,9 @@ def parse_args():
     p.add_argument("--impl", default="sparoa", choices=["sparoa", "reference"])
     p.add_argument("--workload", default="conv",
                    choices=["conv", "fc", "resnet18", "mobilenet_v2", "vit_b16", "mlp_sweep", "ops",
-                            "calibrate", "batching", "split"])
+                            "calibrate", "batching", "split", "profile"])
+    p.add_argument("--op", default="conv_cfg2",
+                   help="profile: the operator to run (see run_profile)")
     p.add_argument("--batch", type=int, default=32)
     p.add_argument("--thresholds", default="default", choices=["default", "calibrated"],
                    help="graph workloads: the default s_thr/c_thr, or the per-operator thresholds "
@@ -1156,6 +1158,83 @@ def run_split(args, rank, local_rank, world, peaks):
             "rows": rows}
 
 
+def run_profile(args, rank, local_rank, world, peaks):
+    """One operator at a workload shape, called 4 times on the same inputs (no
+    CUDA graph): the fixed launch sequence that the committed ncu summaries
+    capture (e.g. ``-k regex:conv3 -s 3 -c 1`` takes the 4th launch).  Inputs
+    larger than L2 are the bench's shapes; the 4th call finds them partly in
+    L2 (a capture's DRAM bytes are read against that)."""
+    import torch
+
+    from paper_2511_19457_gb300 import sparoa as sp
+    from paper_2511_19457_gb300 import synth
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    ctx = sp.Context(local_rank)
+    gen = torch.Generator(device=dev).manual_seed(0)
+
+    def act(*shape, zero_p=0.5):
+        v = torch.randn(*shape, device=dev, generator=gen).abs()
+        v[torch.rand(*shape, device=dev, generator=gen) < zero_p] = 0.0
+        return v.to(torch.bfloat16)
+
+    op = args.op
+    if op == "conv_cfg2":  # the default bench step: stats + dispatch + 3x3 conv, BN + ReLU
+        d = synth.conv_layer(seed=0)
+        x = sp.bits_to_device(d["x"]).view(8, 56, 56, 64)
+        w = sp.bits_to_device(d["w"]).view(64, 3, 3, 64)
+        bn = torch.from_numpy(d["bn"]).to(dev)
+        y = torch.empty(8, 56, 56, 64, dtype=torch.bfloat16, device=dev)
+        yo = sp.OccupancyBuffer(8 * 56 * 56, 64)
+        call = lambda: sp.sparoa_conv2d(ctx, x, w, y, stride=1, pad=1, bn=bn, act=sp.ACT_RELU, y_occ=yo)
+    elif op == "fc_cfg1":
+        d = synth.fc_layer(seed=0)
+        x = sp.bits_to_device(d["x"]).view(64, 512)
+        w = sp.bits_to_device(d["w"]).view(512, 512)
+        wkn = sp.bits_to_device(d["w_kn"]).view(512, 512)
+        y = torch.empty(64, 512, dtype=torch.float32, device=dev)
+        call = lambda: sp.sparoa_gemm(ctx, x, w, y, W_kn=wkn)
+    elif op in ("gemm_dense_mlp", "gemm_skip_mlp_block32"):
+        wts = synth.mlp_weights(seed=0)
+        w2 = sp.bits_to_device(wts["w2"]).view(768, 3072)
+        h = sp.bits_to_device(synth.mlp_hidden(4096, 0.5, "block32", seed=1)).view(4096, 3072)
+        y = torch.empty(4096, 768, dtype=torch.bfloat16, device=dev)
+        force = 1 if op == "gemm_dense_mlp" else 2
+        call = lambda: sp.sparoa_gemm(ctx, h, w2, y, thr=sp.thresholds(force_path=force))
+    elif op in ("dw3_s2", "dw3_s1"):
+        N, H, W, C, s_ = (32, 112, 112, 96, 2) if op == "dw3_s2" else (32, 56, 56, 144, 1)
+        Ho, Wo = (H + 2 - 3) // s_ + 1, (W + 2 - 3) // s_ + 1
+        x = act(N, H, W, C)
+        w = (torch.randn(C, 3, 3, 1, device=dev, generator=gen) / 3).to(torch.bfloat16)
+        bnp = torch.tensor(synth.identity_bn(C), device=dev)
+        y = torch.empty(N, Ho, Wo, C, dtype=torch.bfloat16, device=dev)
+        yo = sp.OccupancyBuffer(N * Ho * Wo, C)
+        call = lambda: sp.sparoa_conv2d(ctx, x, w, y, stride=s_, pad=1, groups=C, bn=bnp, act=sp.ACT_RELU6, y_occ=yo)
+    elif op == "maxpool":
+        x = act(32, 112, 112, 64)
+        y = torch.empty(32, 56, 56, 64, dtype=torch.bfloat16, device=dev)
+        yo = sp.OccupancyBuffer(32 * 56 * 56, 64)
+        call = lambda: sp.sparoa_maxpool2d(ctx, x, y, y_occ=yo)
+    elif op == "bn_act":
+        x = act(32, 56, 56, 64, zero_p=0.0)
+        bnp = torch.tensor(synth.identity_bn(64), device=dev)
+        y = torch.empty(32, 56, 56, 64, dtype=torch.bfloat16, device=dev)
+        yo = sp.OccupancyBuffer(32 * 56 * 56, 64)
+        call = lambda: sp.sparoa_bn_act(ctx, x, y, bn=bnp, act=sp.ACT_RELU, y_occ=yo)
+    elif op == "stats_large":
+        x = act(401408, 64)
+        oc = sp.OccupancyBuffer(401408, 64)
+        call = lambda: sp.sparoa_op_stats(ctx, x, (401408, 64), occ=oc, host=False)
+    else:
+        raise SystemExit(f"profile: unknown op {op}")
+    t0 = time.perf_counter()
+    for _ in range(4):
+        call()
+    torch.cuda.synchronize()
+    ctx.close()
+    return {"workload": "profile", "op": op, "calls": 4, "seconds": time.perf_counter() - t0}
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -1198,6 +1277,8 @@ def main():
         line = run_batching(args, rank, local_rank, world, peaks)
     elif args.workload == "split":
         line = run_split(args, rank, local_rank, world, peaks)
+    elif args.workload == "profile":
+        line = run_profile(args, rank, local_rank, world, peaks)
     else:
         raise SystemExit(f"workload {args.workload} is not wired into bench.py")
     if rank == 0:
