@@ -37,6 +37,9 @@ if ROOT not in sys.path:
 
 METRIC = "effective TFLOP/s & % roofline per op; synthetic CNN images/s at batch 1/32"
 NBUF = 40   # rotating input/output sets per step, 40 x 6.6 MB > 129 MB L2
+# one sparoa_conv2d call measuring its own input: a small clear (the input's
+# counters and block masks), the stats kernel (which also zeroes the output's
+# occupancy block) and the conv kernel
 LAUNCHES_PER_CONV_STEP = 3
 
 
@@ -330,9 +333,8 @@ def run_conv(args, rank, local_rank, world, peaks):
                          x_occ=xo[j], y_occ=yo[j])
 
     def step(j):
-        # one call: the input's Eq. 1 statistics measured inside it (one clear
-        # launch for the input's and the output's occupancy, the stats kernel),
-        # then the dispatched conv kernel
+        # one call: the input's Eq. 1 statistics measured inside it (a small
+        # clear, the stats kernel), then the dispatched conv kernel
         sp.sparoa_conv2d(ctx, xs[j], w, ys[j], stride=1, pad=1, bn=bn, act=sp.ACT_RELU, thr=thr,
                          y_occ=yo[j])
 

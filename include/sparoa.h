@@ -214,13 +214,22 @@ sparoa_status sparoa_set_stream(sparoa_ctx *ctx, void *stream);
 /* Launch overlap (default on): each kernel of a call is launched with CUDA's
  * programmatic stream serialization, so that its on-chip prologue (barrier
  * initialisation, tensor-memory allocation) runs while the kernel before it
- * on the stream finishes.  No kernel reads or writes global memory before the
- * previous grid has completed, so results do not depend on this setting.
- * enable = 0 launches plainly.  Errors: INVALID_ARG (ctx == NULL). */
+ * on the stream finishes.  Before the previous grid has completed a kernel
+ * writes no global memory and reads only inputs that an earlier kernel of the
+ * same call has already waited for (so they are complete), so results do not
+ * depend on this setting.  enable = 0 launches plainly.
+ * Errors: INVALID_ARG (ctx == NULL). */
 sparoa_status sparoa_set_overlap(sparoa_ctx *ctx, int32_t enable);
 
 /* Wait for the stream; report (and clear) a device-side timeout. */
 sparoa_status sparoa_sync(sparoa_ctx *ctx);
+
+/* Wait for the stream and write to *path the path that the last sparoa_gemm
+ * or sparoa_conv2d call on this context took (SPAROA_PATH_DENSE_TC /
+ * SPAROA_PATH_ZERO_SKIP / SPAROA_PATH_DEPTHWISE, as its kernel recorded it on
+ * the device: Sec. 3's rule), without the call's full statistics record.
+ * Errors: INVALID_ARG (ctx or path NULL), CUDA, TIMEOUT as sparoa_sync. */
+sparoa_status sparoa_last_path(sparoa_ctx *ctx, int32_t *path);
 
 /* Testing hooks for the failure paths (the paper has no counterpart).
  *

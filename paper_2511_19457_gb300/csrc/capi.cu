@@ -317,7 +317,7 @@ sparoa_status offer_splitk(sparoa_ctx* ctx, IgemmArgs* a, int slot = -1) {
 sparoa_status run_stats(sparoa_ctx* ctx, const void* x, int64_t R, int64_t C,
                         const sparoa_occupancy& o) {
   SP_TRY(occ_clear(ctx, o, stats_writes_rows_whole(R, (int)C)));
-  SP_CUDA(launch_stats(static_cast<const __nv_bfloat16*>(x), R, (int)C, to_dev(o), ctx->stream));
+  SP_CUDA(launch_stats(static_cast<const __nv_bfloat16*>(x), R, (int)C, to_dev(o), ctx->stream, true));
   return SPAROA_OK;
 }
 
@@ -544,6 +544,9 @@ struct ConvPlan {
   sparoa_occupancy xo;
   const sparoa_occupancy* yo;
   DispatchDev disp;
+  // a kernel of this library was launched between the producers of x, w and
+  // the epilogue's parameters and the conv (IgemmArgs::early)
+  int early = 0;
 };
 
 sparoa_status run_conv(sparoa_ctx* ctx, const ConvPlan& c) {
@@ -579,6 +582,7 @@ sparoa_status run_conv(sparoa_ctx* ctx, const ConvPlan& c) {
   a.err = ctx->d_err();
   a.wait_limit = ctx->wait_limit;
   a.fault = ctx->fault == 1 ? kFaultSkipFirstAccCommit : 0;
+  a.early = c.early;
   if (!pointwise && conv3_supported(a)) {
     SP_CUDA(launch_conv3(a, ctx->stream));
     return SPAROA_OK;
@@ -692,6 +696,16 @@ sparoa_status sparoa_set_overlap(sparoa_ctx* ctx, int32_t enable) {
 sparoa_status sparoa_set_stream(sparoa_ctx* ctx, void* stream) {
   if (!ctx) return SPAROA_ERR_INVALID_ARG;
   ctx->stream = static_cast<cudaStream_t>(stream);
+  return SPAROA_OK;
+}
+
+sparoa_status sparoa_last_path(sparoa_ctx* ctx, int32_t* path) {
+  if (!ctx || !path) return SPAROA_ERR_INVALID_ARG;
+  DeviceGuard g(ctx->device, ctx->overlap);
+  int32_t p = 0;
+  SP_CUDA(cudaMemcpyAsync(&p, ctx->d_path(), 4, cudaMemcpyDeviceToHost, ctx->stream));
+  SP_TRY(read_device_error(ctx));
+  *path = p;
   return SPAROA_OK;
 }
 
@@ -967,20 +981,39 @@ sparoa_status sparoa_conv2d(sparoa_ctx* ctx, const void* x, int64_t N, int64_t H
   const Work wk = conv_work(N, H, W, C_in, C_out, kh, kw, Ho, Wo, groups);
   sparoa_occupancy xo;
   const bool need_x_occ = !depthwise || host_out;
+  bool launched = false;  // a kernel of this call runs before the operator's
   if (need_x_occ && !x_occ && N > 0) {
-    // the input's occupancy is measured into context scratch: one clear
-    // launch for it and the output's block, then the statistics
+    // The input's occupancy is measured into context scratch: one small
+    // clear launch (the counters and block masks; the stats kernel writes the
+    // row bitmaps whole when C_in <= 64), then the stats kernel, which also
+    // zeroes the output's occupancy block.  The clear comes between x's
+    // producer and the stats kernel, so that kernel may read x before its
+    // griddepcontrol.wait.
     const int64_t R = N * H * W;
     SP_TRY(ensure(ctx, ctx->occ, occ_layout(R, C_in).total));
     occ_carve(ctx->occ.p, R, C_in, &xo);
-    std::vector<std::pair<uint32_t*, int64_t>> rg;
-    occ_ranges(xo, stats_writes_rows_whole(R, (int)C_in), &rg);
-    if (y_occ) occ_ranges(*y_occ, false, &rg);
-    SP_TRY(clear_ranges(ctx, rg));
-    SP_CUDA(launch_stats(static_cast<const __nv_bfloat16*>(x), R, (int)C_in, to_dev(xo), ctx->stream));
+    std::vector<std::pair<uint32_t*, int64_t>> pre, yr;
+    occ_ranges(xo, stats_writes_rows_whole(R, (int)C_in), &pre);
+    if (y_occ) occ_ranges(*y_occ, false, &yr);
+    if (yr.size() > 5) {  // a caller block in separate fields: cleared with the input's
+      pre.insert(pre.end(), yr.begin(), yr.end());
+      yr.clear();
+    }
+    ClearArgs z = {};
+    for (size_t k = 0; k < yr.size(); ++k) {
+      z.p[k] = yr[k].first;
+      z.words[k] = yr[k].second;
+    }
+    SP_TRY(clear_ranges(ctx, pre));
+    SP_CUDA(launch_stats(static_cast<const __nv_bfloat16*>(x), R, (int)C_in, to_dev(xo), ctx->stream, true,
+                         &z));
+    launched = true;
   } else {
     if (need_x_occ && x_occ) xo = *x_occ;
-    if (y_occ) SP_TRY(occ_clear(ctx, *y_occ));
+    if (y_occ) {
+      SP_TRY(occ_clear(ctx, *y_occ));
+      launched = true;
+    }
   }
   if (N > 0) {
     if (depthwise) {
@@ -1040,6 +1073,7 @@ sparoa_status sparoa_conv2d(sparoa_ctx* ctx, const void* x, int64_t N, int64_t H
       c.disp.fpb_ok = intensity_ok(t, wk);
       c.disp.force = t.force_path;
       c.disp.path_out = ctx->d_path();
+      c.early = launched && c.Cp == C_in ? 1 : 0;  // (padding launches write x and w)
       SP_TRY(run_conv(ctx, c));
     }
   }

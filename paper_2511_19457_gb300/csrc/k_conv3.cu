@@ -25,9 +25,19 @@
 // occupancy (column counts kept in registers across tiles, row flags of the
 // two column halves combined at one 64-thread barrier per lane quarter).
 //
-// Warp roles (416 threads, persistent CTAs): warp 0 lane 0 issues the slab
-// TMA loads, warp 1 computes the skip masks, warps 4-11 epilogue (two per TMEM
-// lane quarter, 32 columns each), warp 12 MMA.
+// Warp roles (352 threads, persistent CTAs): warp 0 lane 0 issues the slab
+// TMA loads, warp 1 computes the skip masks, warp 2 lane 0 issues the MMAs,
+// warps 3-10 epilogue (two per TMEM lane quarter -- warp w reads lanes
+// 32 (w % 4).. -- 32 columns each).
+//
+// Overlap with the statistics kernel launched before it: at most 128
+// registers a thread (45,056 a CTA) leave room on an SM for one CTA of that
+// kernel, so these CTAs become resident while it runs; when the host
+// launched a kernel of this library between the producers of x / w and this
+// grid (IgemmArgs::early), the weights, the first slab and the epilogue's
+// column affine are loaded before griddepcontrol.wait.  After the wait one
+// thread reads the input's count for the rule and warp 1 reads the first
+// tile's block masks, side by side.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -51,8 +61,9 @@ int conv3_smem(int C, int Co, int W) {
 
 constexpr int kEpiWarps = 8;                      // two per TMEM lane quarter, 32 columns each
 constexpr int kEpiThreads = 32 * kEpiWarps;
-constexpr int kMmaWarp = 4 + kEpiWarps;
-constexpr int kThreads = 32 * (kMmaWarp + 1);     // 4 producer warps, epilogue warps, MMA warp
+constexpr int kMmaWarp = 2;
+constexpr int kFirstEpiWarp = 3;
+constexpr int kThreads = 32 * (kFirstEpiWarp + kEpiWarps);  // slab loads, masks, MMA, epilogue
 constexpr int kBM = 128;
 constexpr int kMaxPos = 1024;  // slab positions (bounds the slab size)
 
@@ -176,7 +187,7 @@ __device__ __forceinline__ void conv3_issue(uint32_t d, uint64_t adesc0, uint64_
 }
 
 template <int CO>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __maxnreg__(128)
     conv3_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
                  const IgemmArgs P, const Conv3Geo G) {
   extern __shared__ uint8_t smem_raw[];
@@ -200,6 +211,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(ctl + 156);
   uint32_t* s_tapm = reinterpret_cast<uint32_t*>(ctl + 160);          // [2] 9-bit occupied-tap masks
   int* s_slabs = reinterpret_cast<int*>(ctl + 176);                    // slabs issued (drain after an abort)
+  volatile int* s_path = reinterpret_cast<volatile int*>(ctl + 180);   // the rule's decision
   uint8_t* s_rowf = ctl + 256;                                         // [3][2][128] row has a non-zero
   float* s_scale = reinterpret_cast<float*>(ctl + 1024);              // [CO]
   float* s_shift = s_scale + CO;                                       // [CO]
@@ -229,15 +241,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tmap(&tmW);
   }
   if (warp == kMmaWarp) tmem_alloc(smem_u32(s_tmem), (uint32_t)(2 * CO));
-  if (warp >= 4 && warp < kMmaWarp)
-    for (int c = threadIdx.x - 128; c < CO; c += kEpiThreads) s_acc[c] = 0u;
+  if (warp >= kFirstEpiWarp)
+    for (int c = threadIdx.x - 32 * kFirstEpiWarp; c < CO; c += kEpiThreads) s_acc[c] = 0u;
   // the first tile's slab origin (arithmetic on the parameters only)
   const int t_first = blockIdx.x;
   const int img_first = t_first / G.tiles_per_img;
   const int oh0_first = (t_first - img_first * G.tiles_per_img) * kBM / Wp;
-  pdl_wait();
-  pdl_trigger();
-  if (threadIdx.x == 0 && t_first < tiles) {
+  auto issue_first = [&]() {
     // The weights (the same 72 KB for every CTA, from L2) go out first, then
     // the first tile's slab.
     mbar_arrive_expect_tx(bar_w, (uint32_t)(9 * (C / 64) * CO * 128));
@@ -248,13 +258,36 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int cb = 0; cb < C / 64; ++cb)
       tma_load_4d(sSlab + (uint32_t)(cb * G.chunk_stride), &tmX, bar_full, cb * 64, -1, oh0_first - 1,
                   img_first);
+  };
+  auto load_affine = [&]() {  // epilogue threads: the column affine into shared memory
+    for (int c = threadIdx.x - 32 * kFirstEpiWarp; c < CO; c += kEpiThreads) {
+      float sc = 1.f, sh = 0.f;
+      if (c < G.Co) epi_affine(P.ep, G.Co, c, sc, sh);
+      s_scale[c] = sc;
+      s_shift[c] = sh;
+    }
+  };
+  if (P.early) {
+    if (threadIdx.x == 0 && t_first < tiles) issue_first();
+    if (warp >= kFirstEpiWarp) load_affine();
   }
-  const int path = decide_path(P.disp);
-  record_path(P.disp, path);
-  const bool skip = path == 2;
+  pdl_wait();
+  pdl_trigger();
+  if (!P.early && threadIdx.x == 0 && t_first < tiles) issue_first();
+  // the rule (one read of the input's count per CTA) and, side by side, the
+  // first tile's occupied taps (used on the zero-skip path only)
+  uint32_t first_mask = 0x1FFu;
+  if (threadIdx.x == 0) {
+    const int pth = decide_path(P.disp);
+    record_path(P.disp, pth);
+    *s_path = pth;
+  } else if (warp == 1 && t_first < tiles && P.disp.force != 1 && P.in_blk) {
+    first_mask = conv3_tap_mask(G, P.in_blk, P.in_C32, t_first, lane);
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  const bool skip = *s_path == 2;
   const uint32_t tmem = *s_tmem;
 
   if (warp == 0) {
@@ -287,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0 && j >= 2)
           ok = mbar_wait(bar_empty + 8 * b, (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutEmpty, wlim);
         if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) break;
-        const uint32_t m = conv3_tap_mask(G, P.in_blk, P.in_C32, t, lane);
+        const uint32_t m = j == 0 ? first_mask : conv3_tap_mask(G, P.in_blk, P.in_C32, t, lane);
         if (lane == 0) {
           s_tapm[b] = m;
           mbar_arrive(bar_mask + 8 * b);
@@ -331,26 +364,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int k = 0; k < 2 && ok; ++k, ++j)
         ok = mbar_wait(bar_acce + 8 * (j & 1), (uint32_t)(((j >> 1) & 1) ^ 1), err, s_abort, kErrTimeoutAcc, wlim);
     }
-  } else if (warp >= 4) {
+  } else if (warp >= kFirstEpiWarp) {
     // -------------------------------------------------------------- epilogue
     // warp w reads TMEM lanes 32 (w % 4).. (its quarter of the tile's rows) and
-    // the 32 accumulator columns 32 ((w - 4) / 4)..; the two warps of a lane
+    // the 32 accumulator columns 32 ((w - 3) / 4)..; the two warps of a lane
     // quarter meet at one 64-thread named barrier per tile (id 3 + quarter)
-    const int q = warp & 3, r = q * 32 + lane, et = threadIdx.x - 128;
-    const int hf = (warp - 4) >> 2;
+    const int q = warp & 3, r = q * 32 + lane, et = threadIdx.x - 32 * kFirstEpiWarp;
+    const int hf = (warp - kFirstEpiWarp) >> 2;
     const int c0 = hf * 32;
     const int pair_bar = 3 + q;
     const OccDev o = P.out_occ;
     const int act = P.ep.act;
     const __nv_bfloat16* const residual = P.ep.residual;
-    // the column affine, read here rather than before the CTA barrier so that
-    // its global loads do not hold up the first MMAs
-    for (int c = et; c < CO; c += kEpiThreads) {
-      float sc = 1.f, sh = 0.f;
-      if (c < G.Co) epi_affine(P.ep, G.Co, c, sc, sh);
-      s_scale[c] = sc;
-      s_shift[c] = sh;
-    }
+    // without the early loads the column affine is read here, after the CTA
+    // barrier, so that its global loads do not hold up the first MMAs
+    if (!P.early) load_affine();
     named_bar_sync(2, kEpiThreads);
     // this warp's 32 columns of the affine stay in registers for every tile
     float sc[32], sh[32];

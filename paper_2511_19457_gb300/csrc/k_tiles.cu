@@ -290,8 +290,20 @@ __device__ __forceinline__ uint32_t nz_pairs(uint32_t w) {
   return (((w & 0x7FFF7FFFu) + 0x7FFF7FFFu) >> 15) & 0x00010001u;
 }
 
+// Grid-stride zeroing of up to five word ranges.
+__device__ __forceinline__ void zero_ranges(const ClearArgs& a) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+#pragma unroll
+  for (int k = 0; k < 5; ++k) {
+    uint32_t* p = a.p[k];
+    const int64_t n = a.words[k];
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) p[i] = 0u;
+  }
+}
+
 __global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloat16* __restrict__ x,
-                                                                int64_t R, int C, OccDev o_param) {
+                                                                int64_t R, int C, OccDev o_param,
+                                                                int early, const ClearArgs zero) {
   const OccDev o = o_param;  // registers, not parameter-space loads
   __shared__ uint32_t s_cnt[8 * 64];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -305,8 +317,6 @@ __global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloa
   // 64-bit division per tile)
   const int ct0 = L0 < L1 ? (int)(L0 / nrb) : 0;
   const int64_t rb0 = L0 - (int64_t)ct0 * nrb;
-  pdl_wait();
-  pdl_trigger();
   int64_t Ln = L0;  // next tile to load, at (l_ct, l_rb)
   int l_ct = ct0;
   int64_t l_rb = rb0;
@@ -419,9 +429,21 @@ __global__ void __launch_bounds__(kTileThreads, 3) stats_kernel(const __nv_bfloa
       if (w < o.C32) atomicOr(&o.blk_mask[(row0 >> 7) * o.C32 + w], v);
     }
   };
+  // with `early` (x complete when the grid starts) the first two tiles are in
+  // flight while griddepcontrol.wait waits for the clear of the counters
   uint4 ua[4], ub[4];
-  load(ua);
-  load(ub);
+  if (early) {
+    load(ua);
+    load(ub);
+    pdl_wait();
+    pdl_trigger();
+  } else {
+    pdl_wait();
+    pdl_trigger();
+    load(ua);
+    load(ub);
+  }
+  zero_ranges(zero);  // another block's counters and masks (the loads are in flight)
   for (int64_t L = L0; L < L1; ++L) {
     tile(ua);
     if (++L >= L1) break;
@@ -1244,13 +1266,7 @@ size_t acc_smem(int emit, int C) {
 __global__ void __launch_bounds__(256) clear_kernel(const ClearArgs a) {
   pdl_wait();
   pdl_trigger();
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-#pragma unroll
-  for (int k = 0; k < 5; ++k) {
-    uint32_t* p = a.p[k];
-    const int64_t n = a.words[k];
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) p[i] = 0u;
-  }
+  zero_ranges(a);
 }
 
 // Grid-stride over 128 x 64 tiles with at most 4 CTAs per SM.
@@ -1274,18 +1290,39 @@ bool stats_writes_rows_whole(int64_t R, int C) {
   return C <= 64;  // one column tile: both kernels store each row's word whole
 }
 
-cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev& o, cudaStream_t s) {
+// CTAs of the stats kernel for an [R, C] tensor.
+unsigned stats_grid(int64_t R, int C) {
+  const int64_t tiles = ((R + 127) / 128) * ((C + 63) / 64);
+  if (C % 8 != 0) {
+    const int chunk = stats_chunk(R, C);
+    const int64_t items = ((R + 127) / 128) * ((((C + 63) / 64) + chunk - 1) / chunk);
+    const int64_t cap = 3LL * device_sm_count();
+    return (unsigned)(items < cap ? items : cap);
+  }
+  const int64_t sms = device_sm_count();
+  // the resident CTAs (3 per SM) split the tiles; up to two tiles per SM,
+  // one CTA per SM takes one or two (its loads of both are in flight
+  // together), which leaves each SM room for a CTA of the consumer kernel
+  // launched after it
+  const int64_t cap = tiles <= 2 * sms ? sms : 3 * sms;
+  return (unsigned)(tiles < cap ? tiles : cap);
+}
+
+cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev& o, cudaStream_t s,
+                         bool early, const ClearArgs* zero) {
   if (R <= 0 || C <= 0) return cudaSuccess;
+  ClearArgs z = {};
+  if (zero) z = *zero;
   if (C % 8 == 0) {
-    const int64_t tiles = ((R + 127) / 128) * ((C + 63) / 64);
-    const int64_t cap = 3LL * device_sm_count();  // the resident CTAs (3 per SM) split the tiles
-    const unsigned grid = (unsigned)(tiles < cap ? tiles : cap);
-    return launch_kernel(stats_kernel, dim3(grid), dim3(kTileThreads), 0, s, x, R, C, o);
+    const unsigned grid = stats_grid(R, C);
+    return launch_kernel(stats_kernel, dim3(grid), dim3(kTileThreads), 0, s, x, R, C, o, early ? 1 : 0, z);
+  }
+  if (zero) {  // the scalar kernel zeroes nothing: a clear launch first
+    const cudaError_t e = launch_clear(z, s);
+    if (e != cudaSuccess) return e;
   }
   const int chunk = stats_chunk(R, C);
-  const int64_t items = ((R + 127) / 128) * ((((C + 63) / 64) + chunk - 1) / chunk);
-  const int64_t cap = 3LL * device_sm_count();  // the resident CTAs (3 per SM) loop over the items
-  const unsigned grid = (unsigned)(items < cap ? items : cap);
+  const unsigned grid = stats_grid(R, C);  // the resident CTAs (3 per SM) loop over the items
   const size_t smem = C <= kMaxAccCols ? sizeof(uint32_t) * (size_t)C : 0;
   return launch_kernel(stats_scalar_kernel, dim3(grid), dim3(kTileThreads), smem, s, x, R, C, o, chunk);
 }

@@ -50,15 +50,21 @@ struct DispatchDev {
   int32_t* path_out;  // nullable; written once by CTA (0,0,0) thread 0
 };
 
-// The threshold rule, in IEEE double (path 1 = dense, 2 = zero-skip).
-__device__ __forceinline__ int decide_path(const DispatchDev& d) {
+// The threshold rule, in IEEE double (path 1 = dense, 2 = zero-skip), for an
+// input with `nnz` non-zeros.
+__device__ __forceinline__ int decide_path_count(const DispatchDev& d, unsigned long long nnz) {
   if (d.force == 1) return 1;
   if (d.force == 2) return 2;
-  const unsigned long long nnz = *d.in_nnz;
   const double zeros = (double)(d.numel - nnz);
   const double bound = __dmul_rn(d.s_thr, (double)d.numel);
   if (zeros >= bound) return 2;
   return d.fpb_ok ? 1 : 2;
+}
+
+__device__ __forceinline__ int decide_path(const DispatchDev& d) {
+  if (d.force == 1) return 1;
+  if (d.force == 2) return 2;
+  return decide_path_count(d, *d.in_nnz);
 }
 
 __device__ __forceinline__ void record_path(const DispatchDev& d, int path) {

@@ -74,6 +74,11 @@ struct IgemmArgs {
   uint32_t* err = nullptr;
   long long wait_limit = 0;          // cycles before a bounded wait gives up (0: the default)
   int fault = 0;                     // error-path tests: kFaultSkipFirstAccCommit or 0
+  // 1: the host launched a kernel of this library between the producers of
+  // x, w and the epilogue's parameters and this grid, so they are complete
+  // when this grid starts and may be read before griddepcontrol.wait (every
+  // kernel here triggers its dependents only after its own wait)
+  int early = 0;
   // split K (set by launch_igemm from the scratch offered here): fp32 partial
   // tiles [tiles][ksplit][128][BN] in `ws` (ws_bytes), one zeroed arrival
   // counter per output tile in `ws_cnt` (ws_cnt_len), left zero again
@@ -159,7 +164,13 @@ cudaError_t launch_select(const __nv_bfloat16* x, int N, int T, int D, int index
 // bitmaps, are accumulated and must be zero on entry.
 constexpr int kStatsWholeRowCols = 512;
 bool stats_writes_rows_whole(int64_t R, int C);
-cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev& o, cudaStream_t s);
+// early: x is complete when the kernel starts (a kernel of this library was
+// launched between its producer and this one), so its first tiles are loaded
+// before griddepcontrol.wait.  zero: word ranges the kernel zeroes after its
+// wait, besides its own work (blocks that a later kernel accumulates into;
+// not `o`).
+cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev& o, cudaStream_t s,
+                         bool early = false, const ClearArgs* zero = nullptr);
 
 // Copy [P, C] to [P, Cp] with zero channels C..Cp-1.
 cudaError_t launch_pad_channels(const __nv_bfloat16* x, int64_t P, int C, int Cp,

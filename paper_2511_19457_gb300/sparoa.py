@@ -85,6 +85,7 @@ _sig("sparoa_set_overlap", [_P, _I32])
 _sig("sparoa_graph_workspace", [_P, _P, _I32, _I64, _I64, _I64, _I64, ctypes.POINTER(ctypes.c_uint64)])
 _sig("sparoa_gemm_split", [_P, _P, _I64, _I64, _P, _P, _I64, _P, ctypes.c_double, _P, _I32, _P, _P])
 _sig("sparoa_sync", [_P])
+_sig("sparoa_last_path", [_P, ctypes.POINTER(_I32)])
 _sig("sparoa_set_wait_limit", [_P, ctypes.c_int64])
 _sig("sparoa_set_fault", [_P, ctypes.c_int32])
 _lib.sparoa_status_str.restype = ctypes.c_char_p
@@ -114,6 +115,7 @@ _sig("sparoa_gemm_noalloc", [_P, _P, _I64, _I64, _P, _P, _I64, ctypes.POINTER(Ep
                              ctypes.POINTER(Thresholds), _P, _I32, ctypes.POINTER(Stats)])
 
 EXPORTED = ["sparoa_create", "sparoa_destroy", "sparoa_set_stream", "sparoa_set_overlap", "sparoa_sync",
+            "sparoa_last_path",
             "sparoa_set_wait_limit", "sparoa_set_fault",
             "sparoa_status_str", "sparoa_last_error", "sparoa_occupancy_bytes",
             "sparoa_occupancy_init", "sparoa_op_stats", "sparoa_gemm", "sparoa_conv2d",
@@ -173,6 +175,12 @@ class Context:
 
     def sync(self):
         self._check(_lib.sparoa_sync(self.h))
+
+    def last_path(self) -> int:
+        """The path the last sparoa_gemm / sparoa_conv2d call took (synchronises)."""
+        p = _I32(0)
+        self._check(_lib.sparoa_last_path(self.h, ctypes.byref(p)))
+        return int(p.value)
 
     def set_overlap(self, enable: bool):
         """Programmatic dependent launch between consecutive kernels (default on)."""
