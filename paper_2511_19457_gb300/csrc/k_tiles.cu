@@ -1299,12 +1299,7 @@ unsigned stats_grid(int64_t R, int C) {
     const int64_t cap = 3LL * device_sm_count();
     return (unsigned)(items < cap ? items : cap);
   }
-  const int64_t sms = device_sm_count();
-  // the resident CTAs (3 per SM) split the tiles; up to two tiles per SM,
-  // one CTA per SM takes one or two (its loads of both are in flight
-  // together), which leaves each SM room for a CTA of the consumer kernel
-  // launched after it
-  const int64_t cap = tiles <= 2 * sms ? sms : 3 * sms;
+  const int64_t cap = 3LL * device_sm_count();  // the resident CTAs (3 per SM) split the tiles
   return (unsigned)(tiles < cap ? tiles : cap);
 }
 
