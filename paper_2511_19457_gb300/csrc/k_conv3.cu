@@ -248,16 +248,16 @@ __global__ void __maxnreg__(128)
   const int img_first = t_first / G.tiles_per_img;
   const int oh0_first = (t_first - img_first * G.tiles_per_img) * kBM / Wp;
   auto issue_first = [&]() {
-    // The weights (the same 72 KB for every CTA, from L2) go out first, then
-    // the first tile's slab.
-    mbar_arrive_expect_tx(bar_w, (uint32_t)(9 * (C / 64) * CO * 128));
-    for (int tap = 0; tap < 9; ++tap)
-      for (int cb = 0; cb < C / 64; ++cb)
-        tma_load_3d(sW + (uint32_t)((tap * (C / 64) + cb) * CO * 128), &tmW, bar_w, cb * 64, tap, 0);
+    // The first tile's slab goes out first, then the weights (the same 72 KB
+    // for every CTA, from L2; the larger and slower of the two).
     mbar_arrive_expect_tx(bar_full, (uint32_t)(C / 64 * 128 * Wp * G.R));
     for (int cb = 0; cb < C / 64; ++cb)
       tma_load_4d(sSlab + (uint32_t)(cb * G.chunk_stride), &tmX, bar_full, cb * 64, -1, oh0_first - 1,
                   img_first);
+    mbar_arrive_expect_tx(bar_w, (uint32_t)(9 * (C / 64) * CO * 128));
+    for (int tap = 0; tap < 9; ++tap)
+      for (int cb = 0; cb < C / 64; ++cb)
+        tma_load_3d(sW + (uint32_t)((tap * (C / 64) + cb) * CO * 128), &tmW, bar_w, cb * 64, tap, 0);
   };
   auto load_affine = [&]() {  // epilogue threads: the column affine into shared memory
     for (int c = threadIdx.x - 32 * kFirstEpiWarp; c < CO; c += kEpiThreads) {
