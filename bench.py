@@ -963,9 +963,8 @@ def run_ops(args, rank, local_rank, world, peaks):
     kocc = int((x0.float().abs().sum(0) != 0).sum().item())
     b = kocc * N * 2 + M * K * 2 + M * N * 4
     measure(f"fc zero-skip [{M},{K}]x[{K},{N}] (occupied K {kocc})",
-            lambda: (x0.clone(), torch.empty(M, N, dtype=torch.float32, device=dev), sp.OccupancyBuffer(M, K)),
-            lambda st: (sp.sparoa_op_stats(ctx, st[0], (M, K), occ=st[2], host=False),
-                        sp.sparoa_gemm(ctx, st[0], wfc, st[1], W_kn=wkn, x_occ=st[2])),
+            lambda: (x0.clone(), torch.empty(M, N, dtype=torch.float32, device=dev)),
+            lambda st: sp.sparoa_gemm(ctx, st[0], wfc, st[1], W_kn=wkn),
             M * K * 2 + M * N * 4, alg_bytes=b)
     # a5 dense GEMMs (MLP block) and the 3x3 conv
     for (M, K, N) in [(4096, 768, 3072), (4096, 3072, 768)]:

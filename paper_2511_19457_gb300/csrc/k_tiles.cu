@@ -540,8 +540,31 @@ __device__ __forceinline__ void stream_tile(StreamEmit& e, const uint32_t (&n)[4
   }
 }
 
+// Two fp32 values through the activation to a bf16 pair (round to nearest
+// even), `lo` in the low half; ReLU is applied by the conversion itself.
+template <int ACT>
+__device__ __forceinline__ uint32_t act_pack2(float lo, float hi) {
+  if (ACT == 2) {
+    lo = fminf(fmaxf(lo, 0.f), 6.f);
+    hi = fminf(fmaxf(hi, 0.f), 6.f);
+  } else if (ACT == 3) {
+    lo = gelu_f(lo);
+    hi = gelu_f(hi);
+  }
+  uint32_t d;
+  if (ACT == 1)
+    asm("cvt.rn.relu.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  else
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  return d;
+}
+
 // Stand-alone bias / batch norm / residual / activation over [R, C] (C % 8
-// == 0), y and its occupancy.
+// == 0), y and its occupancy.  The activation and the presence of a residual
+// are compile-time parameters, so that a tile's 32 values per thread go
+// through straight-line code (bf16 halves widened by shifts, one FMA each,
+// the activation fused into the packing conversion).
+template <int ACT, bool RES>
 __global__ void __launch_bounds__(kTileThreads, 2) bn_act_kernel(const __nv_bfloat16* __restrict__ x, int64_t R,
                                                                  int C, EpiDev ep_param,
                                                                  __nv_bfloat16* __restrict__ y, OccDev o_param,
@@ -607,22 +630,31 @@ __global__ void __launch_bounds__(kTileThreads, 2) bn_act_kernel(const __nv_bflo
       aff_ct = ct;
     }
     uint4 ur[4];  // the residual rows, all in flight together
+    if (RES) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int64_t r = row0 + rs + 32 * i;
-      ur[i] = (res && r < R && c0 < C) ? *reinterpret_cast<const uint4*>(res + r * C + c0) : make_uint4(0u, 0u, 0u, 0u);
+      for (int i = 0; i < 4; ++i) {
+        const int64_t r = row0 + rs + 32 * i;
+        ur[i] = (r < R && c0 < C) ? *reinterpret_cast<const uint4*>(res + r * C + c0) : make_uint4(0u, 0u, 0u, 0u);
+      }
     }
     uint32_t n[4][4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const int64_t r = row0 + rs + 32 * i;
-      float f[8], rv[8];
-      unpack8(u[i], f);
-      unpack8(ur[i], rv);
-      float v[8];
+      const uint32_t* xw = reinterpret_cast<const uint32_t*>(&u[i]);
+      const uint32_t* rw = reinterpret_cast<const uint32_t*>(&ur[i]);
+      uint4 pk;
+      uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) v[j] = epi_act(fmaf(f[j], sc[j], sh[j]) + rv[j], ep.act);
-      const uint4 pk = pack8(v);
+      for (int w = 0; w < 4; ++w) {
+        float lo = fmaf(__uint_as_float(xw[w] << 16), sc[2 * w], sh[2 * w]);
+        float hi = fmaf(__uint_as_float(xw[w] & 0xFFFF0000u), sc[2 * w + 1], sh[2 * w + 1]);
+        if (RES) {
+          lo += __uint_as_float(rw[w] << 16);
+          hi += __uint_as_float(rw[w] & 0xFFFF0000u);
+        }
+        pw[w] = act_pack2<ACT>(lo, hi);
+      }
       const bool ok = r < R && c0 < C;
       if (ok) *reinterpret_cast<uint4*>(y + r * C + c0) = pk;
       n[i][0] = ok ? nz_pairs(pk.x) : 0u;
@@ -678,7 +710,21 @@ __global__ void __launch_bounds__(kTileThreads, 3)
     uint4 outv[4];
     bool okr[4];
     if (k == 3) {
-      // two rows at a time: their 18 taps in flight together
+      // This thread's output rows row0 + rs + 32 i: (image, oh, ow) by one
+      // division for the first and stepping for the others; an output whose
+      // 3 x 3 window lies inside the image loads its taps at fixed offsets
+      // from one address, a border output clamps each tap and leaves the
+      // outside ones out.  Two outputs at a time: 18 loads in flight.
+      const int64_t m0 = row0 + rs;
+      int img = 0, oh = 0, ow = 0;
+      if (m0 < R) {
+        const int mr = (int)m0;
+        img = mr / hw;
+        const int rem = mr - img * hw;
+        oh = rem / Wo;
+        ow = rem - oh * Wo;
+      }
+      const int64_t rowC = (int64_t)W * C;
 #pragma unroll
       for (int i0 = 0; i0 < 4; i0 += 2) {
         uint4 u[2][9];
@@ -686,23 +732,44 @@ __global__ void __launch_bounds__(kTileThreads, 3)
 #pragma unroll
         for (int ii = 0; ii < 2; ++ii) {
           const int i = i0 + ii;
-          const int64_t mrow = row0 + rs + 32 * i;
-          okr[i] = mrow < R && c0 < C;
-          const int mr = okr[i] ? (int)mrow : 0;
-          const int img = mr / hw, rem = mr - (mr / hw) * hw;
-          const int oh = rem / Wo, ow = rem - (rem / Wo) * Wo;
-          inb[ii] = 0u;
+          if (i > 0) {  // the next output row of this thread: 32 positions on
+            ow += 32;
+            while (ow >= Wo) {
+              ow -= Wo;
+              if (++oh == Ho) {
+                oh = 0;
+                ++img;
+              }
+            }
+          }
+          okr[i] = m0 + 32 * i < R && c0 < C;
+          const int ih0 = oh * stride - pad, iw0 = ow * stride - pad;
+          const bool inner = ih0 >= 0 && ih0 + 2 < H && iw0 >= 0 && iw0 + 2 < W;
+          inb[ii] = 0x1FFu;
+          if (!okr[i]) {
 #pragma unroll
-          for (int r = 0; r < 3; ++r) {
-            const int ih = oh * stride - pad + r;
-            const int ihc = ih < 0 ? 0 : (ih >= H ? H - 1 : ih);
+            for (int t = 0; t < 9; ++t) u[ii][t] = make_uint4(0u, 0u, 0u, 0u);
+          } else if (inner) {
+            const __nv_bfloat16* p = x + (((int64_t)img * H + ih0) * W + iw0) * C + c0;
 #pragma unroll
-            for (int s2 = 0; s2 < 3; ++s2) {
-              const int iw = ow * stride - pad + s2;
-              const int iwc = iw < 0 ? 0 : (iw >= W ? W - 1 : iw);
-              if (ih == ihc && iw == iwc) inb[ii] |= 1u << (r * 3 + s2);
-              u[ii][r * 3 + s2] = okr[i] ? __ldg(reinterpret_cast<const uint4*>(x + (((int64_t)img * H + ihc) * W + iwc) * C + c0))
-                                         : make_uint4(0u, 0u, 0u, 0u);
+            for (int r = 0; r < 3; ++r)
+#pragma unroll
+              for (int s2 = 0; s2 < 3; ++s2)
+                u[ii][r * 3 + s2] = __ldg(reinterpret_cast<const uint4*>(p + r * rowC + s2 * C));
+          } else {
+            inb[ii] = 0u;
+#pragma unroll
+            for (int r = 0; r < 3; ++r) {
+              const int ih = ih0 + r;
+              const int ihc = ih < 0 ? 0 : (ih >= H ? H - 1 : ih);
+#pragma unroll
+              for (int s2 = 0; s2 < 3; ++s2) {
+                const int iw = iw0 + s2;
+                const int iwc = iw < 0 ? 0 : (iw >= W ? W - 1 : iw);
+                if (ih == ihc && iw == iwc) inb[ii] |= 1u << (r * 3 + s2);
+                u[ii][r * 3 + s2] =
+                    __ldg(reinterpret_cast<const uint4*>(x + (((int64_t)img * H + ihc) * W + iwc) * C + c0));
+              }
             }
           }
         }
@@ -1402,8 +1469,19 @@ cudaError_t launch_bn_act(const __nv_bfloat16* x, int64_t R, int C, const EpiDev
   if (C % 8) return cudaErrorInvalidValue;
   const int64_t tiles = ((R + 127) / 128) * ((C + 63) / 64);
   const int64_t cap2 = 2LL * device_sm_count();  // the resident CTAs (two per SM) split the tiles
-  return launch_kernel(bn_act_kernel, dim3((unsigned)(tiles < cap2 ? tiles : cap2)), dim3(kTileThreads), 0,
-                       s, x, R, C, ep, y, o, emit);
+  const dim3 grid((unsigned)(tiles < cap2 ? tiles : cap2));
+  const bool res = ep.residual != nullptr;
+  switch (ep.act * 2 + (res ? 1 : 0)) {
+    case 0: return launch_kernel(bn_act_kernel<0, false>, grid, dim3(kTileThreads), 0, s, x, R, C, ep, y, o, emit);
+    case 1: return launch_kernel(bn_act_kernel<0, true>, grid, dim3(kTileThreads), 0, s, x, R, C, ep, y, o, emit);
+    case 2: return launch_kernel(bn_act_kernel<1, false>, grid, dim3(kTileThreads), 0, s, x, R, C, ep, y, o, emit);
+    case 3: return launch_kernel(bn_act_kernel<1, true>, grid, dim3(kTileThreads), 0, s, x, R, C, ep, y, o, emit);
+    case 4: return launch_kernel(bn_act_kernel<2, false>, grid, dim3(kTileThreads), 0, s, x, R, C, ep, y, o, emit);
+    case 5: return launch_kernel(bn_act_kernel<2, true>, grid, dim3(kTileThreads), 0, s, x, R, C, ep, y, o, emit);
+    case 6: return launch_kernel(bn_act_kernel<3, false>, grid, dim3(kTileThreads), 0, s, x, R, C, ep, y, o, emit);
+    case 7: return launch_kernel(bn_act_kernel<3, true>, grid, dim3(kTileThreads), 0, s, x, R, C, ep, y, o, emit);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 }  // namespace sparoa

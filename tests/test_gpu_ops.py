@@ -293,8 +293,12 @@ def test_depthwise(sp, ctx, N, H, W, C, s):
     assert_occ_equal(yo.to_host(), orc.stats(sp.device_to_bits(y), N * Ho * Wo, C), "dw y_occ")
 
 
-def test_maxpool_bit_exact(sp, ctx):
-    N, H, W, C = 2, 33, 31, 64
+@pytest.mark.parametrize("shape", [(2, 33, 31, 64), (3, 9, 11, 128), (4, 112, 112, 64), (1, 2, 3, 8)])
+def test_maxpool_bit_exact(sp, ctx, shape):
+    """Interior windows (fixed tap offsets) and border windows (clamped taps),
+    output rows that wrap several image rows per 32-row step (Wo = 5, 6),
+    two column tiles, many tiles, and a window larger than the image."""
+    N, H, W, C = shape
     xb = _bits((N, H, W, C), 9, zero_p=0.4)
     Ho, Wo = (H + 2 - 3) // 2 + 1, (W + 2 - 3) // 2 + 1
     y = torch.empty(N, Ho, Wo, C, dtype=torch.bfloat16, device="cuda")
@@ -316,17 +320,22 @@ def test_avgpool(sp, ctx):
     assert_occ_equal(yo.to_host(), orc.stats(sp.device_to_bits(y), N, C), "avgpool y_occ")
 
 
-def test_bn_act(sp, ctx):
-    R, C = 300, 72
+@pytest.mark.parametrize("R,C", [(300, 72), (1000, 64)])
+@pytest.mark.parametrize("with_res", [False, True])
+@pytest.mark.parametrize("act", [0, 1, 2, 3])
+def test_bn_act(sp, ctx, R, C, with_res, act):
+    """Every activation, with and without a residual (the kernel's
+    compile-time variants), on one and on two column tiles."""
     g = torch.Generator().manual_seed(2)
     xb = _bits((R, C), 11, zero_p=0.3)
     rb = _bits((R, C), 12, zero_p=0.3)
     bn = synth.random_bn(C, g)
     y = torch.empty(R, C, dtype=torch.bfloat16, device="cuda")
     yo = sp.OccupancyBuffer(R, C)
-    sp.sparoa_bn_act(ctx, _dev(sp, xb, (R, C)), y, bn=torch.from_numpy(bn).cuda(), act=sp.ACT_RELU6,
-                     residual=_dev(sp, rb, (R, C)), y_occ=yo)
-    assert_close(_f64(y), orc.bn_act(xb, R, C, bn=bn, residual_bits=rb, act=2), what="bn_act")
+    sp.sparoa_bn_act(ctx, _dev(sp, xb, (R, C)), y, bn=torch.from_numpy(bn).cuda(), act=act,
+                     residual=_dev(sp, rb, (R, C)) if with_res else None, y_occ=yo)
+    ref = orc.bn_act(xb, R, C, bn=bn, residual_bits=rb if with_res else None, act=act)
+    assert_close(_f64(y), ref, what=f"bn_act act {act} residual {with_res}")
     assert_occ_equal(yo.to_host(), orc.stats(sp.device_to_bits(y), R, C), "bn_act y_occ")
 
 
