@@ -17,7 +17,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libsparoa.so")
-SOURCES = ["capi.cu", "k_igemm.cu", "k_conv3.cu", "k_tiles.cu", "k_fcskip.cu", "k_vit.cu", "noalloc.cu"]
+SOURCES = ["capi.cu", "k_igemm.cu", "k_conv3.cu", "k_dw3.cu", "k_tiles.cu", "k_fcskip.cu", "k_vit.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

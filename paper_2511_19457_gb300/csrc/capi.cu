@@ -1035,6 +1035,8 @@ sparoa_status sparoa_conv2d(sparoa_ctx* ctx, const void* x, int64_t N, int64_t H
       if (y_occ) a.out_occ = to_dev(*y_occ);
       a.emit = y_occ ? 1 : 0;
       a.path_out = ctx->d_path();
+      a.err = ctx->d_err();
+      a.wait_limit = ctx->wait_limit;
       SP_CUDA(launch_dwconv(a, ctx->stream));
     } else {
       ConvPlan c;
@@ -1430,6 +1432,8 @@ sparoa_status sparoa_run_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_
           a.out_occ = to_dev(*yo);
           a.emit = 1;
           a.path_out = d_paths + i;
+          a.err = ctx->d_err();
+          a.wait_limit = ctx->wait_limit;
           SP_CUDA(launch_dwconv(a, ctx->stream));
           break;
         }

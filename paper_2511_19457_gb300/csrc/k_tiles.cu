@@ -7,8 +7,8 @@
 // over HBM.
 //   stats_kernel    Eq. 1 count and bitmaps of an existing tensor (C % 8 == 0;
 //                   stats_scalar_kernel for other widths)
-//   dw3_kernel      depthwise 3x3, stride 1 or 2, on 2-D output tiles (MobileNetV2
-//                   layers); dwconv_kernel for other depthwise shapes
+//   dwconv_kernel   depthwise convolutions other than the 3x3 shapes of
+//                   k_dw3.cu
 //   maxpool_kernel  k x k max pooling
 //   avgpool_kernel  global average pooling
 //   bn_act_kernel   stand-alone bias / batch norm / residual / activation
@@ -947,320 +947,6 @@ __global__ void __launch_bounds__(kTileThreads) dwconv_kernel(const DwArgs a_par
 }
 
 // ---------------------------------------------------------------------------
-// Depthwise 3x3, pad 1, stride S in {1, 2} (every MobileNetV2 depthwise layer)
-// on 2-D output tiles: a CTA computes kDwTH x kDwTW output pixels of one image
-// and one 64-channel slice.  The input tile with its halo is staged in shared
-// memory once (cp.async, zero-filled outside the image = the padding); each
-// thread then computes 4 horizontally adjacent pixels x 8 channels, reading
-// every input column it needs once per kernel row.  Tiles run channel-slice
-// major so a CTA's consecutive tiles keep their weights and affine.
-constexpr int kDwTH = 8, kDwTW = 16;
-// input tiles a stride-S CTA keeps in shared memory: two (the next step's tile
-// loads while this one is computed) when they fit next to two CTAs per SM
-constexpr int dw3_buffers(int S) { return S == 1 ? 2 : 1; }
-
-constexpr int kDwMaxBlk = 16;  // 128-row blocks one output tile can touch (Wo up to ~280)
-
-template <int S>
-__global__ void __launch_bounds__(kTileThreads) dw3_kernel(const DwArgs a_param, int inner) {
-  const DwArgs a = a_param;  // registers, not parameter-space loads
-  constexpr int IH = (kDwTH - 1) * S + 3, IW = (kDwTW - 1) * S + 3;
-  constexpr int NCOL = 3 * S + 3;  // input columns a 4-pixel strip reads: (4 - 1) S + 3
-  constexpr int NB = dw3_buffers(S);  // input tiles in flight: 2 = the next one loads during this one
-  extern __shared__ __align__(16) uint8_t dsm[];
-  const int Cp = ((a.C + 63) / 64) * 64;  // channels rounded up to whole slices
-  __nv_bfloat16* s_in0 = reinterpret_cast<__nv_bfloat16*>(dsm);  // [NB][IH][IW][64]
-  float* s_wf = reinterpret_cast<float*>(dsm + NB * IH * IW * 128);  // [9][Cp] weights
-  float* s_sc = s_wf + 9 * Cp;                                   // [Cp] affine scale
-  float* s_sh = s_sc + Cp;                                       // [Cp] affine shift
-  uint32_t* s_acc = reinterpret_cast<uint32_t*>(s_sh + Cp);      // [C] when acc
-  uint32_t* s_blk = s_acc + (a.emit && a.C <= kMaxAccCols ? ((a.C + 3) & ~3) : 0);  // [kDwMaxBlk][C32]
-  __shared__ unsigned long long s_rowbm[kDwTH * kDwTW];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int cg = lane & 7, st = lane >> 3;  // channel group, 4-pixel strip of the warp's row
-  const bool acc = a.emit && a.C <= kMaxAccCols;
-  const OccDev o = a.out_occ;
-  // inner: a CTA runs every channel slice of its pixel tile, so it owns the
-  // tile's row-bitmap words (one plain store each) and gathers its block-mask
-  // words in shared memory; otherwise slices are separate work items
-  const bool own = inner != 0;
-  if (acc)
-    for (int c = threadIdx.x; c < a.C; c += kTileThreads) s_acc[c] = 0u;
-  if (own && a.emit) {
-    for (int i = threadIdx.x; i < kDwMaxBlk * o.C32; i += kTileThreads) s_blk[i] = 0u;
-    if (threadIdx.x < kDwTH * kDwTW) s_rowbm[threadIdx.x] = 0ull;
-  }
-  pdl_wait();
-  pdl_trigger();
-  if (a.path_out && blockIdx.x == 0 && threadIdx.x == 0) *a.path_out = 3;
-  const int ctn = (a.C + 63) / 64;
-  const int tiles_h = (a.Ho + kDwTH - 1) / kDwTH, tiles_w = (a.Wo + kDwTW - 1) / kDwTW;
-  const int nsp = a.N * tiles_h * tiles_w;
-  const int64_t items = own ? (int64_t)nsp : (int64_t)nsp * ctn;
-  // A step is one (item, channel slice): owned items run all their slices,
-  // otherwise an item is one slice.  Steps of this CTA in order: items
-  // blockIdx.x, + gridDim.x, ...; slices ct_begin .. ct_end - 1 of each.
-  struct Step {
-    int64_t item;
-    int n, ty, tx, ct, ct_end;
-  };
-  auto make_step = [&](int64_t item, int ct) {
-    Step q;
-    q.item = item;
-    const int ct_begin = own ? 0 : (int)(item / nsp);
-    q.ct_end = own ? ctn : ct_begin + 1;
-    q.ct = ct < 0 ? ct_begin : ct;
-    int rest = (int)(own ? item : item - (int64_t)ct_begin * nsp);
-    q.n = rest / (tiles_h * tiles_w);
-    rest -= q.n * tiles_h * tiles_w;
-    q.ty = rest / tiles_w;
-    q.tx = rest - q.ty * tiles_w;
-    return q;
-  };
-  auto next_step = [&](const Step& q) {
-    if (q.ct + 1 < q.ct_end) {
-      Step r = q;
-      r.ct = q.ct + 1;
-      return r;
-    }
-    return make_step(q.item + gridDim.x, -1);
-  };
-  // stage a step's input tile: 16-byte chunks (8 channels) of IH x IW pixels
-  auto stage = [&](const Step& q, int buf) {
-    const uint32_t dst = smem_u32(s_in0) + (uint32_t)(buf * IH * IW * 128);
-    const int col0 = q.ct * 64;
-    const int gy0 = q.ty * kDwTH * S - 1, gx0 = q.tx * kDwTW * S - 1;
-    const __nv_bfloat16* ximg = a.x + (int64_t)q.n * a.H * a.W * a.C;
-    for (int idx = threadIdx.x; idx < IH * IW * 8; idx += kTileThreads) {
-      const int p = idx >> 3, ch = idx & 7;
-      const int iy = p / IW, ix = p - (p / IW) * IW;
-      const int gy = gy0 + iy, gx = gx0 + ix;
-      const int cc = col0 + ch * 8;
-      const bool ok = gy >= 0 && gy < a.H && gx >= 0 && gx < a.W && cc < a.C;
-      const __nv_bfloat16* src = ok ? ximg + ((uint32_t)(gy * a.W + gx) * (uint32_t)a.C + cc) : a.x;
-      cp_async_16(dst + (uint32_t)(p * 128 + ch * 16), src, ok ? 16u : 0u);
-    }
-    cp_async_commit();
-  };
-  Step cur = make_step(blockIdx.x, -1);
-  if (cur.item < items) stage(cur, 0);
-  // weights and affine of channels [cb, ce) into shared memory: 8 independent
-  // weight loads per thread before their stores, the affine 4 channels at a time
-  auto stage_weights = [&](int cb, int ce) {
-    const int nw = 9 * (ce - cb);
-    for (int base = threadIdx.x; base < nw; base += 8 * kTileThreads) {
-      float v[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int idx = base + u * kTileThreads;
-        const int gi = cb * 9 + idx;
-        v[u] = (idx < nw && gi / 9 < a.C) ? __bfloat162float(a.w[gi]) : 0.f;
-      }
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int idx = base + u * kTileThreads;
-        if (idx < nw) {
-          const int gi = cb * 9 + idx;
-          const int c = gi / 9, t = gi - (gi / 9) * 9;
-          s_wf[t * Cp + c] = v[u];
-        }
-      }
-    }
-    for (int c0 = cb + (int)threadIdx.x; c0 < ce; c0 += 4 * kTileThreads) {
-      float scv[4], shv[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int c = c0 + u * kTileThreads;
-        scv[u] = 1.f;
-        shv[u] = 0.f;
-        if (c < a.C) epi_affine(a.ep, a.C, c, scv[u], shv[u]);
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int c = c0 + u * kTileThreads;
-        if (c < ce) {
-          s_sc[c] = scv[u];
-          s_sh[c] = shv[u];
-        }
-      }
-    }
-  };
-  // while the first input tile is in flight: every channel when the CTA runs
-  // all slices of its pixel tiles or more than one item, else its one item's
-  // slice
-  int w_ct = -1;  // slice whose weights are staged (-1: all)
-  if (own || items > (int64_t)gridDim.x) {
-    stage_weights(0, Cp);
-  } else if (cur.item < items) {
-    stage_weights(cur.ct * 64, cur.ct * 64 + 64);
-    w_ct = cur.ct;
-  }
-  __syncthreads();
-  for (int sj = 0; cur.item < items; ++sj) {
-    const Step nxt = next_step(cur);
-    const int buf = NB == 2 ? (sj & 1) : 0;
-    __syncthreads();  // the step before is done with its buffer (and, owned, with the tile flush)
-    if (NB == 2) {
-      if (nxt.item < items) {
-        stage(nxt, buf ^ 1);
-        cp_async_wait<1>();
-      } else {
-        cp_async_wait<0>();
-      }
-    } else {
-      if (sj > 0) stage(cur, 0);  // the first step's tile was issued before the weights
-      cp_async_wait<0>();
-    }
-    if (w_ct >= 0 && cur.ct != w_ct) {  // one slice staged, another needed (the same for every thread)
-      stage_weights(cur.ct * 64, cur.ct * 64 + 64);
-      w_ct = cur.ct;
-    }
-    __syncthreads();
-    const __nv_bfloat16* s_in = s_in0 + buf * IH * IW * 64;
-    const int n = cur.n, ty = cur.ty, tx = cur.tx, ct = cur.ct;
-    // first 128-row block the tile touches (block-mask words gathered relative to it)
-    const int b0 = (int)((((uint32_t)n * a.Ho + ty * kDwTH) * a.Wo + tx * kDwTW) >> 7);
-    {
-      const int col0 = ct * 64;
-      const int c0 = col0 + cg * 8;
-      const bool cvalid = c0 < a.C;
-      // compute: warp = output row of the tile, strip st = pixels 4 st .. 4 st + 3
-      const int oy = warp, ox0 = st * 4;
-      float accv[4][8];
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-#pragma unroll
-        for (int k = 0; k < 8; ++k) accv[j][k] = 0.f;
-#pragma unroll
-      for (int r = 0; r < 3; ++r) {
-        float wr[3][8];
-#pragma unroll
-        for (int c = 0; c < 3; ++c) {
-          const float4 w0 = *reinterpret_cast<const float4*>(&s_wf[(r * 3 + c) * Cp + c0]);
-          const float4 w1 = *reinterpret_cast<const float4*>(&s_wf[(r * 3 + c) * Cp + c0 + 4]);
-          wr[c][0] = w0.x; wr[c][1] = w0.y; wr[c][2] = w0.z; wr[c][3] = w0.w;
-          wr[c][4] = w1.x; wr[c][5] = w1.y; wr[c][6] = w1.z; wr[c][7] = w1.w;
-        }
-        const int iy = oy * S + r;
-#pragma unroll
-        for (int q = 0; q < NCOL; ++q) {  // input column ox0 * S + q
-          float f[8];
-          unpack8(*reinterpret_cast<const uint4*>(&s_in[((iy * IW) + ox0 * S + q) * 64 + cg * 8]), f);
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const int c = q - j * S;  // kernel column that pixel j applies to this input column
-            if (c >= 0 && c < 3) {
-#pragma unroll
-              for (int k = 0; k < 8; ++k) accv[j][k] = fmaf(f[k], wr[c][k], accv[j][k]);
-            }
-          }
-        }
-      }
-      // epilogue: affine, residual, activation, store, occupancy
-      const int oh = ty * kDwTH + oy;
-      float sc[8], sh[8];
-      {
-        const float4 a0 = *reinterpret_cast<const float4*>(&s_sc[c0]);
-        const float4 a1 = *reinterpret_cast<const float4*>(&s_sc[c0 + 4]);
-        const float4 b0v = *reinterpret_cast<const float4*>(&s_sh[c0]);
-        const float4 b1v = *reinterpret_cast<const float4*>(&s_sh[c0 + 4]);
-        sc[0] = a0.x; sc[1] = a0.y; sc[2] = a0.z; sc[3] = a0.w; sc[4] = a1.x; sc[5] = a1.y; sc[6] = a1.z; sc[7] = a1.w;
-        sh[0] = b0v.x; sh[1] = b0v.y; sh[2] = b0v.z; sh[3] = b0v.w; sh[4] = b1v.x; sh[5] = b1v.y; sh[6] = b1v.z; sh[7] = b1v.w;
-      }
-      uint32_t cnt[8];
-#pragma unroll
-      for (int k = 0; k < 8; ++k) cnt[k] = 0u;
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int ow = tx * kDwTW + ox0 + j;
-        const bool live = cvalid && oh < a.Ho && ow < a.Wo;
-        const uint32_t mrow = ((uint32_t)n * a.Ho + (oh < a.Ho ? oh : 0)) * a.Wo + (ow < a.Wo ? ow : 0);
-        float rv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        if (a.ep.residual && live) unpack8(*reinterpret_cast<const uint4*>(a.ep.residual + (int64_t)mrow * a.C + c0), rv);
-        float ov[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) ov[k] = epi_act(fmaf(accv[j][k], sc[k], sh[k]) + rv[k], a.ep.act);
-        const uint4 uo = pack8(ov);
-        uint32_t mask = 0u;
-        if (live) {
-          *reinterpret_cast<uint4*>(a.y + (int64_t)mrow * a.C + c0) = uo;
-          mask = nz_mask8(uo);
-        }
-        if (a.emit) {
-          // row bitmap: the strip's 8 lanes hold this pixel's 64 channels
-          const uint32_t b = __ballot_sync(0xffffffffu, mask != 0u);
-          if (cg == 0 && ((b >> (8 * st)) & 0xFFu)) {
-            const unsigned long long bit = 1ull << ((col0 >> 6) & 63);
-            if (own) atomicOr(&s_rowbm[oy * kDwTW + ox0 + j], bit);
-            else atomicOr(&o.row_bm[(int64_t)mrow * o.W64 + (col0 >> 12)], bit);
-          }
-          // block mask: OR over the 4 lanes of one 32-column word, then one add
-          uint32_t bits = mask << ((cg & 3) * 8);
-          bits |= __shfl_xor_sync(0xffffffffu, bits, 1);
-          bits |= __shfl_xor_sync(0xffffffffu, bits, 2);
-          const int word = (col0 >> 5) + (cg >> 2);
-          if ((cg & 3) == 0 && bits && word < o.C32) {
-            const int lb = (int)(mrow >> 7) - b0;
-            if (own && lb >= 0 && lb < kDwMaxBlk) atomicOr(&s_blk[lb * o.C32 + word], bits);
-            else atomicOr(&o.blk_mask[(int64_t)(mrow >> 7) * o.C32 + word], bits);
-          }
-#pragma unroll
-          for (int k = 0; k < 8; ++k) cnt[k] += (mask >> k) & 1u;
-        }
-      }
-      if (a.emit) {
-        // column counts: lanes cg, cg + 8, cg + 16, cg + 24 hold one channel
-        // group; its first lane adds them (shared-memory atomics, no barrier)
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          cnt[k] += __shfl_xor_sync(0xffffffffu, cnt[k], 8);
-          cnt[k] += __shfl_xor_sync(0xffffffffu, cnt[k], 16);
-        }
-        if (lane < 8 && cvalid) {
-          if (acc) {
-#pragma unroll
-            for (int k = 0; k < 8; ++k)
-              if (cnt[k]) atomicAdd(&s_acc[c0 + k], cnt[k]);
-          } else {
-            uint32_t sum = 0u;
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              if (cnt[k]) atomicAdd(&o.col_nnz[c0 + k], cnt[k]);
-              sum += cnt[k];
-            }
-            if (sum) {
-              atomicAdd(&o.tile_nnz[col0 >> 6], sum);
-              atomicAdd(o.nnz, (unsigned long long)sum);
-            }
-          }
-        }
-      }
-    }
-    if (own && a.emit && cur.ct + 1 == cur.ct_end) {
-      // the tile's row words (owned: plain stores) and its block-mask words
-      __syncthreads();
-      if (threadIdx.x < kDwTH * kDwTW) {
-        const int oy = threadIdx.x / kDwTW, ox = threadIdx.x - (threadIdx.x / kDwTW) * kDwTW;
-        const int oh = ty * kDwTH + oy, ow = tx * kDwTW + ox;
-        if (oh < a.Ho && ow < a.Wo)
-          o.row_bm[(int64_t)(((uint32_t)n * a.Ho + oh) * a.Wo + ow) * o.W64] = s_rowbm[threadIdx.x];
-        s_rowbm[threadIdx.x] = 0ull;
-      }
-      for (int i = threadIdx.x; i < kDwMaxBlk * o.C32; i += kTileThreads) {
-        const uint32_t v = s_blk[i];
-        if (v) {
-          const int lb = i / o.C32, w = i - (i / o.C32) * o.C32;
-          atomicOr(&o.blk_mask[(int64_t)(b0 + lb) * o.C32 + w], v);
-          s_blk[i] = 0u;
-        }
-      }
-    }
-    cur = nxt;
-  }
-  if (a.emit) cta_done(o, s_acc, acc);
-}
-
-// ---------------------------------------------------------------------------
 // Global average pooling [N, HW, C] -> [N, C] (C % 8 == 0): one CTA per (image,
 // 64-channel slice).  Lane l of warp w sums pixels 4 w + l / 8 + 32 k of the 8
 // channels 8 (l % 8) .. + 7, so every load of the CTA is in flight at once;
@@ -1410,33 +1096,7 @@ cudaError_t launch_dwconv(const DwArgs& a, cudaStream_t s) {
   if (R <= 0) return cudaSuccess;
   // the kernels' 32-bit index math: output rows and one image's elements
   if (R >= ((int64_t)1 << 31) || (int64_t)a.H * a.W * a.C >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;
-  const bool shape3 = a.kh == 3 && a.kw == 3 && a.pad == 1 && (a.stride == 1 || a.stride == 2) && (a.C % 8) == 0;
-  const int tiles = ((a.Ho + kDwTH - 1) / kDwTH) * ((a.Wo + kDwTW - 1) / kDwTW);
-  const int64_t nsp = (int64_t)a.N * tiles;
-  const int64_t ntiles = nsp * ((a.C + 63) / 64);
-  const int ih = (kDwTH - 1) * a.stride + 3, iw = (kDwTW - 1) * a.stride + 3;
-  const int C32 = (a.C + 31) / 32;
-  const int Cp = ((a.C + 63) / 64) * 64;
-  const size_t acc_b = a.emit && a.C <= kMaxAccCols ? sizeof(uint32_t) * (size_t)((a.C + 3) & ~3) : 0;
-  const size_t smem = (size_t)dw3_buffers(a.stride) * ih * iw * 128 + sizeof(float) * 11 * (size_t)Cp + acc_b +
-                      sizeof(uint32_t) * (size_t)kDwMaxBlk * C32;
-  if (shape3 && ntiles < ((int64_t)1 << 31) && smem <= 200 * 1024) {
-    // 2-D tiles with the input staged in shared memory; one CTA runs every
-    // channel slice of its pixel tile when that still fills the GPU
-    // pipelined (two input tiles) CTAs stay resident two per SM and loop over
-    // their steps; the single-buffered ones get a third CTA per SM to hide loads
-    const int64_t cap = (dw3_buffers(a.stride) == 2 ? 2LL : 3LL) * device_sm_count();
-    const int inner = (nsp >= 2LL * device_sm_count() && a.C <= 4096) ? 1 : 0;
-    const int64_t items = inner ? nsp : ntiles;
-    const unsigned grid = (unsigned)(items < cap ? items : cap);
-    auto kern = a.stride == 1 ? dw3_kernel<1> : dw3_kernel<2>;
-    // opt in above the 48 KB default, which also counts the static shared memory
-    if (smem > 40 * 1024) {
-      cudaError_t e = smem_optin(reinterpret_cast<const void*>(kern), smem);
-      if (e != cudaSuccess) return e;
-    }
-    return launch_kernel(kern, dim3(grid), dim3(kTileThreads), smem, s, a, inner);
-  }
+  if (dw3_supported(a)) return launch_dw3(a, s);
   return launch_kernel(dwconv_kernel, dim3(tile_grid(R, a.C)), dim3(kTileThreads),
                        acc_smem(a.emit, a.C), s, a);
 }

@@ -185,8 +185,15 @@ struct DwArgs {
   OccDev out_occ{};
   int emit = 0;
   int32_t* path_out = nullptr;
+  uint32_t* err = nullptr;           // bounded waits: error bits (k_dw3.cu)
+  long long wait_limit = 0;          // cycles before a bounded wait gives up (0: the default)
 };
 cudaError_t launch_dwconv(const DwArgs& a, cudaStream_t s);
+// The TMA-staged 3x3 depthwise kernel (k_dw3.cu): stride 1 or 2, pad 1,
+// C % 8 == 0, a 16-byte aligned input and the weights of every channel in
+// shared memory.
+bool dw3_supported(const DwArgs& a);
+cudaError_t launch_dw3(const DwArgs& a, cudaStream_t s);
 
 cudaError_t launch_maxpool(const __nv_bfloat16* x, int N, int H, int W, int C, int k, int stride,
                            int pad, int Ho, int Wo, __nv_bfloat16* y, const OccDev& o, int emit,

@@ -273,22 +273,29 @@ def test_conv_structured_zeros_skip_equals_dense(sp, ctx):
 # ---------------------------------------------------------------------------
 # depthwise, pooling, batch norm
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("N,H,W,C,s", [(2, 17, 15, 96, 1), (2, 17, 15, 96, 2), (1, 8, 8, 8, 1),
-                                       (3, 14, 14, 960, 1)])
-def test_depthwise(sp, ctx, N, H, W, C, s):
+@pytest.mark.parametrize("N,H,W,C,s,act,res", [
+    (2, 17, 15, 96, 1, 2, False), (2, 17, 15, 96, 2, 2, False), (1, 8, 8, 8, 1, 2, False),
+    (3, 14, 14, 960, 1, 2, False),
+    # every activation and a residual; C = 32 and 144 leave a partial 64-channel slice
+    (4, 29, 31, 32, 2, 0, False), (2, 11, 9, 144, 1, 1, True), (2, 12, 20, 48, 2, 3, False),
+    (1, 7, 7, 576, 2, 2, True),
+    # enough pixel tiles that every CTA runs all slices of its tiles (owned row words)
+    (32, 56, 56, 144, 1, 2, False), (32, 112, 112, 96, 2, 2, False)])
+def test_depthwise(sp, ctx, N, H, W, C, s, act, res):
     g = torch.Generator().manual_seed(C + s)
     xb = _bits((N, H, W, C), C * s, zero_p=0.5, dist="abs")
     wb = synth.to_bf16_bits(synth.he_normal((C, 3, 3, 1), 9, g))
     bn = synth.random_bn(C, g)
     Ho, Wo = (H + 2 - 3) // s + 1, (W + 2 - 3) // s + 1
+    rb = _bits((N, Ho, Wo, C), C + 7, zero_p=0.3) if res else None
     y = torch.empty(N, Ho, Wo, C, dtype=torch.bfloat16, device="cuda")
     yo = sp.OccupancyBuffer(N * Ho * Wo, C)
     st = sp.sparoa_conv2d(ctx, _dev(sp, xb, (N, H, W, C)), _dev(sp, wb, (C, 3, 3, 1)), y, stride=s,
-                          pad=1, groups=C, bn=torch.from_numpy(bn).cuda(), act=sp.ACT_RELU6,
-                          y_occ=yo, host=True)
+                          pad=1, groups=C, bn=torch.from_numpy(bn).cuda(), act=act,
+                          residual=_dev(sp, rb, (N, Ho, Wo, C)) if res else None, y_occ=yo, host=True)
     assert st.path == sp.PATH_DEPTHWISE
     assert st.nnz == orc.stats(xb, N * H * W, C).nnz
-    ref = orc.conv2d(xb, N, H, W, C, wb, C, 3, 3, s, 1, groups=C, bn=bn, act=2)
+    ref = orc.conv2d(xb, N, H, W, C, wb, C, 3, 3, s, 1, groups=C, bn=bn, residual_bits=rb, act=act)
     assert_close(_f64(y), ref, what="depthwise")
     assert_occ_equal(yo.to_host(), orc.stats(sp.device_to_bits(y), N * Ho * Wo, C), "dw y_occ")
 
