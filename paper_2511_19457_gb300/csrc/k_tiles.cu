@@ -829,6 +829,161 @@ __global__ void __launch_bounds__(kTileThreads, 3)
 }
 
 // ---------------------------------------------------------------------------
+// ---------------------------------------------------------------------------
+// Narrow tensors (C < 8 channels, the RGB input): a thread takes groups of 8
+// consecutive rows = C 16-byte words (the group starts on a 16-byte boundary
+// when x does), so every load is a full vector.  Element e of a group is row
+// e / C, channel e % C; its non-zero bit goes to bit e of a 64-bit mask, and
+// the channel counts are population counts of the mask under a constant
+// per-channel pattern.
+template <int C>
+struct NarrowMasks {
+  static constexpr unsigned long long chan(int c) {
+    unsigned long long m = 0ull;
+    for (int p = 0; p < 8; ++p) m |= 1ull << (p * C + c);
+    return m;
+  }
+};
+
+template <int C>
+__device__ __forceinline__ bool narrow_load(const __nv_bfloat16* __restrict__ x, int64_t R, int64_t g,
+                                            uint32_t (&w)[4 * C]) {
+  const int64_t r0 = g * 8;
+  if (r0 + 8 <= R) {
+    const uint4* p = reinterpret_cast<const uint4*>(x + r0 * C);
+#pragma unroll
+    for (int k = 0; k < C; ++k) {
+      const uint4 v = __ldg(p + k);
+      w[4 * k] = v.x;
+      w[4 * k + 1] = v.y;
+      w[4 * k + 2] = v.z;
+      w[4 * k + 3] = v.w;
+    }
+    return true;
+  }
+  // the last, partial group: element by element, zero past the tensor
+  const uint16_t* q = reinterpret_cast<const uint16_t*>(x);
+  const int64_t n = (R - r0) * C;
+#pragma unroll
+  for (int k = 0; k < 4 * C; ++k) {
+    const uint32_t lo = 2 * k < n ? q[r0 * C + 2 * k] : 0u;
+    const uint32_t hi = 2 * k + 1 < n ? q[r0 * C + 2 * k + 1] : 0u;
+    w[k] = lo | (hi << 16);
+  }
+  return false;
+}
+
+// Eq. 1 count and occupancy of an [R, C] tensor with C < 8.  Rows are whole
+// words of the row bitmap (one column tile) and a half warp's 16 groups are
+// one 128-row block, so row words and block masks are plain stores; the
+// counts meet in shared memory and reach global memory once per CTA.
+template <int C>
+__global__ void __launch_bounds__(256) stats_narrow_kernel(const __nv_bfloat16* __restrict__ x, int64_t R,
+                                                           OccDev o, int early) {
+  __shared__ uint32_t s_cnt[C];
+  const int lane = threadIdx.x & 31;
+  if (threadIdx.x < C) s_cnt[threadIdx.x] = 0u;
+  __syncthreads();
+  if (!early) {
+    pdl_wait();
+    pdl_trigger();
+  }
+  const int64_t groups = (R + 7) / 8;
+  const int64_t RB = (R + 127) / 128;
+  uint32_t cnt[C];
+#pragma unroll
+  for (int c = 0; c < C; ++c) cnt[c] = 0u;
+  bool waited = !early;
+  // whole warps step together (32 groups = two 128-row blocks per step)
+  const int64_t wstride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t g0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); g0 < groups; g0 += wstride) {
+    const int64_t g = g0 + lane;
+    uint32_t w[4 * C];
+    if (g < groups) narrow_load<C>(x, R, g, w);
+    else
+#pragma unroll
+      for (int k = 0; k < 4 * C; ++k) w[k] = 0u;
+    if (!waited) {  // the loads of the first step were issued before the wait
+      pdl_wait();
+      pdl_trigger();
+      waited = true;
+    }
+    unsigned long long m = 0ull;
+#pragma unroll
+    for (int k = 0; k < 4 * C; ++k) {
+      const uint32_t t = ((w[k] & 0x7FFF7FFFu) + 0x7FFF7FFFu) >> 15;
+      m |= (unsigned long long)(t & 1u) << (2 * k);
+      m |= (unsigned long long)((t >> 16) & 1u) << (2 * k + 1);
+    }
+    uint32_t chbits = 0u;
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      const unsigned long long mc = m & NarrowMasks<C>::chan(c);
+      cnt[c] += (uint32_t)__popcll(mc);
+      chbits |= (mc != 0ull ? 1u : 0u) << c;
+    }
+    if (g < groups) {
+      const int64_t r0 = g * 8;
+#pragma unroll
+      for (int p = 0; p < 8; ++p)
+        if (r0 + p < R) o.row_bm[r0 + p] = ((m >> (p * C)) & ((1ull << C) - 1ull)) ? 1ull : 0ull;
+    }
+    // block masks: lanes 0-15 and 16-31 are the blocks g0 / 16 and g0 / 16 + 1
+    const uint32_t blo = __reduce_or_sync(0xffffffffu, lane < 16 ? chbits : 0u);
+    const uint32_t bhi = __reduce_or_sync(0xffffffffu, lane >= 16 ? chbits : 0u);
+    const int64_t b = g0 / 16;
+    if (lane == 0 && b < RB) o.blk_mask[b] = blo;
+    if (lane == 16 && b + 1 < RB) o.blk_mask[b + 1] = bhi;
+  }
+  if (!waited) {
+    pdl_wait();
+    pdl_trigger();
+  }
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    const uint32_t v = __reduce_add_sync(0xffffffffu, cnt[c]);
+    if (lane == 0 && v) atomicAdd(&s_cnt[c], v);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t tot = 0u;
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      const uint32_t v = s_cnt[c];
+      if (v) atomicAdd(&o.col_nnz[c], v);
+      tot += v;
+    }
+    if (tot) {
+      atomicAdd(&o.tile_nnz[0], tot);
+      atomicAdd(o.nnz, (unsigned long long)tot);
+    }
+  }
+}
+
+// [P, C] -> [P, 8] (C < 8, zero channels appended): C 16-byte loads and 8
+// 16-byte stores per group of 8 rows.
+template <int C>
+__global__ void __launch_bounds__(256) pad8_kernel(const __nv_bfloat16* __restrict__ x, int64_t P,
+                                                   __nv_bfloat16* __restrict__ y) {
+  pdl_wait();
+  pdl_trigger();
+  const int64_t groups = (P + 7) / 8;
+  for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < groups;
+       g += (int64_t)gridDim.x * blockDim.x) {
+    uint32_t w[4 * C];
+    narrow_load<C>(x, P, g, w);
+    const uint16_t* h = reinterpret_cast<const uint16_t*>(w);
+#pragma unroll
+    for (int p = 0; p < 8; ++p) {
+      if (g * 8 + p >= P) break;
+      uint32_t o4[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+      for (int c = 0; c < C; ++c) o4[c >> 1] |= (uint32_t)h[p * C + c] << (16 * (c & 1));
+      reinterpret_cast<uint4*>(y)[g * 8 + p] = make_uint4(o4[0], o4[1], o4[2], o4[3]);
+    }
+  }
+}
+
 __global__ void pad_kernel(const __nv_bfloat16* __restrict__ x, int64_t P, int C, int Cp,
                            __nv_bfloat16* __restrict__ y) {
   pdl_wait();
@@ -1065,9 +1220,25 @@ cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev&
     const unsigned grid = stats_grid(R, C);
     return launch_kernel(stats_kernel, dim3(grid), dim3(kTileThreads), 0, s, x, R, C, o, early ? 1 : 0, z);
   }
-  if (zero) {  // the scalar kernel zeroes nothing: a clear launch first
+  if (zero) {  // the kernels below zero nothing: a clear launch first
     const cudaError_t e = launch_clear(z, s);
     if (e != cudaSuccess) return e;
+  }
+  if (C < 8 && (reinterpret_cast<uintptr_t>(x) & 15u) == 0) {
+    const int64_t groups = (R + 7) / 8;
+    const int64_t cap = 4LL * device_sm_count();
+    int64_t blocks = (groups + 255) / 256;
+    blocks = blocks < cap ? blocks : cap;
+    const int e1 = early ? 1 : 0;
+    switch (C) {
+      case 1: return launch_kernel(stats_narrow_kernel<1>, dim3((unsigned)blocks), dim3(256), 0, s, x, R, o, e1);
+      case 2: return launch_kernel(stats_narrow_kernel<2>, dim3((unsigned)blocks), dim3(256), 0, s, x, R, o, e1);
+      case 3: return launch_kernel(stats_narrow_kernel<3>, dim3((unsigned)blocks), dim3(256), 0, s, x, R, o, e1);
+      case 4: return launch_kernel(stats_narrow_kernel<4>, dim3((unsigned)blocks), dim3(256), 0, s, x, R, o, e1);
+      case 5: return launch_kernel(stats_narrow_kernel<5>, dim3((unsigned)blocks), dim3(256), 0, s, x, R, o, e1);
+      case 6: return launch_kernel(stats_narrow_kernel<6>, dim3((unsigned)blocks), dim3(256), 0, s, x, R, o, e1);
+      default: return launch_kernel(stats_narrow_kernel<7>, dim3((unsigned)blocks), dim3(256), 0, s, x, R, o, e1);
+    }
   }
   const int chunk = stats_chunk(R, C);
   const unsigned grid = stats_grid(R, C);  // the resident CTAs (3 per SM) loop over the items
@@ -1088,6 +1259,21 @@ cudaError_t launch_pad_channels(const __nv_bfloat16* x, int64_t P, int C, int Cp
                                 __nv_bfloat16* y, cudaStream_t s) {
   const int64_t n = P * Cp;
   if (n <= 0) return cudaSuccess;
+  if (Cp == 8 && C < 8 && (reinterpret_cast<uintptr_t>(x) & 15u) == 0 && (reinterpret_cast<uintptr_t>(y) & 15u) == 0) {
+    const int64_t groups = (P + 7) / 8;
+    const int64_t cap = 4LL * device_sm_count();
+    int64_t blocks = (groups + 255) / 256;
+    const dim3 grid((unsigned)(blocks < cap ? blocks : cap));
+    switch (C) {
+      case 1: return launch_kernel(pad8_kernel<1>, grid, dim3(256), 0, s, x, P, y);
+      case 2: return launch_kernel(pad8_kernel<2>, grid, dim3(256), 0, s, x, P, y);
+      case 3: return launch_kernel(pad8_kernel<3>, grid, dim3(256), 0, s, x, P, y);
+      case 4: return launch_kernel(pad8_kernel<4>, grid, dim3(256), 0, s, x, P, y);
+      case 5: return launch_kernel(pad8_kernel<5>, grid, dim3(256), 0, s, x, P, y);
+      case 6: return launch_kernel(pad8_kernel<6>, grid, dim3(256), 0, s, x, P, y);
+      default: return launch_kernel(pad8_kernel<7>, grid, dim3(256), 0, s, x, P, y);
+    }
+  }
   return launch_kernel(pad_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, x, P, C, Cp, y);
 }
 

@@ -53,7 +53,12 @@ def _f64(t):
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("R,C,zp", [(1, 8, 0.5), (64, 512, 0.7), (130, 72, 0.5), (257, 40, 0.9),
                                     (129, 70, 0.5), (50176, 3, 0.1), (25088, 64, 0.5),
-                                    (300, 4104, 0.3), (200, 64, 0.0), (200, 64, 1.0)])
+                                    (300, 4104, 0.3), (200, 64, 0.0), (200, 64, 1.0),
+                                    # narrow tensors (C < 8): whole and partial 8-row groups,
+                                    # blocks split between half warps, many blocks
+                                    (1, 3, 0.5), (7, 3, 0.5), (1001, 1, 0.5), (999, 2, 0.3),
+                                    (50177, 3, 0.5), (4097, 5, 0.7), (131, 6, 0.2), (12345, 7, 0.9),
+                                    (1605632, 3, 0.0)])
 def test_stats_bit_exact(sp, ctx, R, C, zp):
     bits = _bits((R, C), R + C, zero_p=zp)
     if R * C > 16:
@@ -216,6 +221,8 @@ CONV_CASES = [
     (2, 14, 14, 96, 24, 1, 1, 0, 0, True),     # pointwise (TMA GEMM mode), linear + residual
     (2, 14, 14, 64, 128, 1, 2, 0, 0, False),   # strided 1x1 downsample
     (1, 32, 30, 3, 64, 7, 2, 3, 1, False),     # stem, C_in padded to 8
+    (3, 21, 19, 3, 32, 3, 2, 1, 2, False),     # 3x3 stem; 1197 pixels: a partial 8-pixel group
+    (2, 9, 13, 5, 16, 3, 1, 1, 0, False),      # C_in 5
     (2, 9, 11, 144, 32, 1, 1, 0, 2, False),    # K = 144 (ragged 32-block)
     (2, 10, 10, 24, 144, 3, 1, 1, 2, False),   # C_in 24: blocks straddle taps
     (1, 7, 7, 512, 512, 3, 1, 1, 1, True),
