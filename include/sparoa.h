@@ -420,18 +420,18 @@ sparoa_status sparoa_graph_workspace(sparoa_ctx *ctx, const sparoa_op *ops, int3
 
 /*
  * sparoa_gemm without any device allocation.  The paper has no counterpart:
- * this exists for callers that cannot call cudaMalloc -- work recorded into a
- * CUDA graph by stream capture (an allocation cannot be captured), plugins
- * inside a framework whose allocator owns the device memory, and loops with a
- * memory budget fixed at start-up.  It computes exactly what sparoa_gemm
+ * this exists for callers that cannot call cudaMalloc -- plugins inside a
+ * framework whose allocator owns the device memory, and loops with a memory
+ * budget fixed at start-up.  It computes exactly what sparoa_gemm
  * computes with x_occ = y_occ = NULL, but needs no context: work goes to
  * `stream` (a cudaStream_t; NULL = legacy default stream) on the current
  * device, and the input's occupancy (the only scratch) lives in a static
  * device array of SPAROA_NOALLOC_SCRATCH_BYTES bytes, 256 of which hold
  * control words.
  *   - The first call on a device looks the array's address up with
- *     cudaGetSymbolAddress while that device is current; make that first call
- *     before any stream capture starts.
+ *     cudaGetSymbolAddress while that device is current and keeps it for the
+ *     process: a device reset (cudaDeviceReset) after that first call is not
+ *     supported.
  *   - Calls share the array and each clears the part it uses before writing;
  *     calls whose work overlaps on the GPU (other streams or host threads)
  *     race on it and must be serialised by the caller.

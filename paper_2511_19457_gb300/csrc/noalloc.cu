@@ -1,20 +1,19 @@
 // sparoa_gemm_noalloc: the fully connected operator with threshold dispatch,
 // for callers that must not allocate device memory.
 //
-// Who needs this: code that records its work into a CUDA graph by stream
-// capture (cudaMalloc cannot be captured and would break the capture), plugins
-// that run inside another framework whose caching allocator owns all device
-// memory, and latency-critical loops whose memory budget is fixed at start-up
-// and where an allocation (slow, implicitly synchronising, or able to fail in
-// the middle of a run) is not acceptable.  sparoa_gemm needs a context, whose
+// Who needs this: plugins that run inside another framework whose caching
+// allocator owns all device memory, and latency-critical loops whose memory
+// budget is fixed at start-up and where an allocation (slow, implicitly
+// synchronising, or able to fail in the middle of a run) is not acceptable.  sparoa_gemm needs a context, whose
 // creation allocates, and it measures the input's occupancy into context
 // scratch that grows on demand.  This entry point instead keeps that scratch
 // in one statically sized __device__ array that every GPU loading the library
 // holds until the process exits.
 //
 // Use: the first call on a device resolves the array's device address with
-// cudaGetSymbolAddress (the device must be current); make that first call
-// before any stream capture begins.  Every call shares the one array, and the
+// cudaGetSymbolAddress (the device must be current) and keeps it for the
+// process, so a device reset after that call is not supported.  Every call
+// shares the one array, and the
 // array keeps the previous call's contents: each call clears the part it uses
 // before writing.  Calls whose work overlaps on the GPU (several streams, or
 // several host threads) race on the array; serialise them.

@@ -1,8 +1,7 @@
 """sparoa_gemm_noalloc: the FC operator for callers that cannot allocate (GPU).
 
-Some callers cannot call cudaMalloc: work being recorded into a CUDA graph by
-stream capture, plugins living inside another framework's allocator, or loops
-with a memory budget fixed at start-up.  sparoa_gemm_noalloc gives them the
+Some callers cannot call cudaMalloc: plugins living inside another framework's
+allocator, or loops with a memory budget fixed at start-up.  sparoa_gemm_noalloc gives them the
 same operator with its only scratch (the input's occupancy) in a static
 device array.  Here its output, Eq. 1 count and path are checked against
 sparoa_gemm and against the oracle on several calls in a row -- a sparse input
