@@ -542,17 +542,28 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_2d(sB + slot * C::kBStage, &tmB, bar_full + 8 * slot, kb * BK, g.n0);
           }
           const uint32_t dst = sA + slot * C::kAStage;
+          // (tap, channel) of the block's first 8-channel chunk by division,
+          // the block's other chunks by stepping (C % 8 == 0)
+          const int flat0 = kb * BK;
+          const int tp0 = flat0 / p.Cp;
+          int c = flat0 - tp0 * p.Cp;
+          int rr = tp0 / p.kw;
+          int ss = tp0 - rr * p.kw;
 #pragma unroll
           for (int j = 0; j < BK / 8; ++j) {
-            const int flat = kb * BK + 8 * j;
-            const int tp = flat / p.Cp;
-            const int c = flat - tp * p.Cp;
-            const int rr = tp / p.kw;
-            const int ss = tp - rr * p.kw;
+            const int flat = flat0 + 8 * j;
             const int ih = ih0 + rr, iw = iw0 + ss;
             const bool val = rvalid && flat < p.Ktot && ih >= 0 && ih < p.H && iw >= 0 && iw < p.W;
             const __nv_bfloat16* src = val ? ximg + ((int64_t)ih * p.W + iw) * p.Cp + c : xin;
             cp_async_16(dst + swz_offset<BK>(r, j), src, val ? 16u : 0u);
+            c += 8;
+            if (c == p.Cp) {
+              c = 0;
+              if (++ss == p.kw) {
+                ss = 0;
+                ++rr;
+              }
+            }
           }
           cp_async_commit();
           ++it;
