@@ -30,9 +30,14 @@ def _rand_bits(shape, seed, scale=1.0, shift=0.0):
 
 @pytest.mark.parametrize("R,C,affine", [(300, 768, True), (197, 64, False), (1, 8, True), (4099, 192, True),
                                          (7, 1024, True),    # longest row held in registers
-                                         (5, 1032, True)])   # re-read path
+                                         (5, 1032, True),    # re-read path
+                                         (6304, 768, True),  # ViT-B/16 at batch 32
+                                         (100000, 64, False)])  # several 128-row blocks per CTA
 def test_layernorm(sp, ctx, R, C, affine):
+    """Constant rows (every fourth) normalise to exact zeros without an affine,
+    so the output's row bitmaps, block masks and counts see zero rows too."""
     xb = _rand_bits((R, C), R + C, 2.0, 1.0)
+    xb.reshape(R, C)[::4] = xb.reshape(R, C)[::4, :1]
     gb = None
     if affine:
         g = torch.Generator().manual_seed(7)
