@@ -382,7 +382,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const int ih = oh * p.stride - p.pad + tp / p.kw;
               const int iw = ow * p.stride - p.pad + tp % p.kw;
               wv[u] = 0ull;
-              if (tp < taps && rvalid && ih >= 0 && ih < p.H && iw >= 0 && iw < p.W)
+              if (in_rowbm && tp < taps && rvalid && ih >= 0 && ih < p.H && iw >= 0 && iw < p.W)
                 wv[u] = in_rowbm[(((int64_t)img * p.H + ih) * p.W + iw) * in_W64];
             }
 #pragma unroll
@@ -394,7 +394,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
           named_bar_sync(1, 128);
-          const bool many = p.kh * p.kw > kMaxTaps || in_W64 > 1;  // no per-tap masks: keep all
+          // no per-tap masks (too many taps, wide rows, or an input without row
+          // bitmaps such as the window rows of a narrow stem): keep every block
+          const bool many = p.kh * p.kw > kMaxTaps || in_W64 > 1 || in_rowbm == nullptr;
           for (int w0 = 0; w0 < kblocks && w0 < kMaxKWords * 32; w0 += 128) {
             const int kb = w0 + r;
             bool occ = false;

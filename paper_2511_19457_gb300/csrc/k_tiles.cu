@@ -984,6 +984,65 @@ __global__ void __launch_bounds__(256) pad8_kernel(const __nv_bfloat16* __restri
   }
 }
 
+// Rows of kernel windows for a convolution with few input channels (the RGB
+// stems): x [N, H, W, C] -> xr [N, H + 2P, Wx, 32], Wx = W + 2P - kw + 1,
+// xr[n][h][w][s C + c] = x[n][h - P][w - P + s][c] for s < kw (zero outside
+// the image), channels kw C .. 31 zero.  A kh x kw convolution of x with
+// stride S and padding P is then a kh x 1 convolution of xr with stride S and
+// no padding over 32 channels (weights [Cout][kh][kw C], padded to 32), whose
+// operands the implicit GEMM loads with 4-D TMA boxes.  One CTA per output
+// row: the zero-padded input row is staged in shared memory, where a
+// window's kw C values are contiguous.
+__global__ void __launch_bounds__(256) im2row_kernel(const __nv_bfloat16* __restrict__ x, int N, int H, int W,
+                                                     int C, int kw, int P, __nv_bfloat16* __restrict__ xr) {
+  // the zero-padded row twice, as 32-bit words: s_even[i] = elements 2i, 2i + 1
+  // and s_odd[i] = elements 2i + 1, 2i + 2, so a window starting at element e
+  // is whole words of one of them (e even: s_even from e / 2, odd: s_odd)
+  extern __shared__ uint32_t s_w32[];
+  pdl_wait();
+  pdl_trigger();
+  const int Hx = H + 2 * P, Wx = W + 2 * P - kw + 1, Wp = W + 2 * P;
+  const int KC = kw * C;
+  const int nel = Wp * C + 32;  // elements of the padded row (+ slack read past the last window)
+  const int nw = (nel + 1) / 2;
+  uint32_t* s_even = s_w32;
+  uint32_t* s_odd = s_w32 + nw;
+  const uint16_t* xs = reinterpret_cast<const uint16_t*>(x);
+  const int KW32 = (KC + 1) / 2;  // words holding the window (the last may hold one element too many)
+  const uint32_t last_mask = (KC & 1) ? 0x0000FFFFu : 0xFFFFFFFFu;
+  for (int64_t row = blockIdx.x; row < (int64_t)N * Hx; row += gridDim.x) {
+    const int n = (int)(row / Hx), hp = (int)(row - (int64_t)n * Hx), h = hp - P;
+    const bool hin = h >= 0 && h < H;
+    const uint16_t* src = xs + ((int64_t)n * H + (hin ? h : 0)) * W * C;
+    auto elem = [&](int e) -> uint32_t {  // element e of the padded row
+      if (!hin || e >= Wp * C) return 0u;
+      const int wq = e / C - P;
+      return (wq >= 0 && wq < W) ? (uint32_t)src[wq * C + (e - (e / C) * C)] : 0u;
+    };
+    for (int i = threadIdx.x; i < nw; i += blockDim.x) {
+      const uint32_t e0 = elem(2 * i), e1 = elem(2 * i + 1), e2 = elem(2 * i + 2);
+      s_even[i] = e0 | (e1 << 16);
+      s_odd[i] = e1 | (e2 << 16);
+    }
+    __syncthreads();
+    // consecutive threads write consecutive 16-byte quarters of the output row
+    uint4* dst = reinterpret_cast<uint4*>(xr + row * Wx * 32);
+    for (int j = threadIdx.x; j < Wx * 4; j += blockDim.x) {
+      const int e = (j >> 2) * C, k0 = (j & 3) * 4;
+      const uint32_t* srcw = ((e & 1) ? s_odd : s_even) + (e >> 1);
+      uint32_t o[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int kk = k0 + k;
+        o[k] = kk < KW32 ? srcw[kk] : 0u;
+        if (kk == KW32 - 1) o[k] &= last_mask;
+      }
+      dst[j] = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+    __syncthreads();
+  }
+}
+
 __global__ void pad_kernel(const __nv_bfloat16* __restrict__ x, int64_t P, int C, int Cp,
                            __nv_bfloat16* __restrict__ y) {
   pdl_wait();
@@ -1253,6 +1312,21 @@ cudaError_t launch_clear(const ClearArgs& a, cudaStream_t s) {
   const int64_t blocks = (mx + 255) / 256;
   const int64_t cap = 2LL * device_sm_count();
   return launch_kernel(clear_kernel, dim3((unsigned)(blocks < cap ? blocks : cap)), dim3(256), 0, s, a);
+}
+
+bool im2row_applies(int C, int kw, int groups) { return groups == 1 && C < 8 && kw > 1 && kw * C <= 32; }
+
+cudaError_t launch_im2row(const __nv_bfloat16* x, int N, int H, int W, int C, int kw, int P, __nv_bfloat16* xr,
+                          cudaStream_t s) {
+  const int64_t rows = (int64_t)N * (H + 2 * P);
+  if (rows <= 0 || W + 2 * P - kw + 1 <= 0) return cudaSuccess;
+  if ((reinterpret_cast<uintptr_t>(xr) & 15u) != 0) return cudaErrorInvalidValue;
+  const size_t nw = ((size_t)(W + 2 * P) * C + 32 + 1) / 2;
+  const size_t smem = 2 * sizeof(uint32_t) * nw;
+  if (smem > 48 * 1024) return cudaErrorInvalidValue;
+  const int64_t cap = 16LL * device_sm_count();
+  return launch_kernel(im2row_kernel, dim3((unsigned)(rows < cap ? rows : cap)), dim3(256), smem, s, x, N, H,
+                       W, C, kw, P, xr);
 }
 
 cudaError_t launch_pad_channels(const __nv_bfloat16* x, int64_t P, int C, int Cp,

@@ -173,6 +173,12 @@ cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev&
                          bool early = false, const ClearArgs* zero = nullptr);
 
 // Copy [P, C] to [P, Cp] with zero channels C..Cp-1.
+// Window rows for a convolution with few input channels (k_tiles.cu):
+// x [N, H, W, C] -> xr [N, H + 2P, W + 2P - kw + 1, 32] (see im2row_kernel),
+// for groups == 1, C < 8, kw > 1 and kw C <= 32 (im2row_applies).
+bool im2row_applies(int C, int kw, int groups);
+cudaError_t launch_im2row(const __nv_bfloat16* x, int N, int H, int W, int C, int kw, int P, __nv_bfloat16* xr,
+                          cudaStream_t s);
 cudaError_t launch_pad_channels(const __nv_bfloat16* x, int64_t P, int C, int Cp,
                                 __nv_bfloat16* y, cudaStream_t s);
 
