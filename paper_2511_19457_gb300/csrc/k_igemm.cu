@@ -35,6 +35,13 @@
 // issues TMA; all 128 gather in mode 1), warps 4-11 epilogue (two per TMEM
 // lane quarter, each taking 32 of every 64 accumulator columns), warp 12 TMEM
 // allocation and MMA issue (lane 0).
+//
+// Each tile shape is compiled twice: the general kernel, and a lean one for
+// modes 0 and 2 without a K split, residual or fp32 output.  With small K the
+// epilogue is the whole cost of a tile and runs at a fraction of an
+// instruction per cycle (few warps, long dependency chains); the lean kernel's
+// smaller, branch-free epilogue issues fewer instructions per tile and misses
+// the instruction cache less.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -132,7 +139,7 @@ struct TileGeo {
 
 __device__ __forceinline__ TileGeo tile_geo(const Geo& p, int t, int nt, int BN) {
   TileGeo g;
-  const int mi = t / nt;
+  const int mi = nt == 1 ? t : t / nt;
   g.n0 = (t - mi * nt) * BN;
   g.m0 = 0;
   g.tn0 = g.th0 = g.tw0 = 0;
@@ -206,17 +213,20 @@ __device__ __forceinline__ UnitGeo unit_geo(const Geo& p, int u, int KS, int kbl
   return q;
 }
 
-template <int BN, int BK>
+template <int BN, int BK, bool LEAN>
 __global__ void __launch_bounds__(kThreads, 1)
     igemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                  const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmA32,
                  const __grid_constant__ CUtensorMap tmB32, const IgemmArgs P) {
   using C = Cfg<BN, BK>;
   const Geo p = make_geo(P);
+  // lean kernel: TMA producers only (mode 0 or 2), no K split, bf16 output
+  // without residual (the host launches it only then)
+  if (LEAN) __builtin_assume(p.conv != 1);
   const EpiDev ep = P.ep;
   const int act = P.ep.act;
-  const __nv_bfloat16* const residual = P.ep.residual;
-  const int y_f32 = P.y_f32;
+  const __nv_bfloat16* const residual = LEAN ? nullptr : P.ep.residual;
+  const int y_f32 = LEAN ? 0 : P.y_f32;
   const int emit = P.emit;
   const long long wlim = P.wait_limit > 0 ? P.wait_limit : kWaitLimitCycles;
   const __nv_bfloat16* const xin = P.x;
@@ -268,10 +278,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int tiles = mtiles * nt;
   // split K: work unit u = (tile u / KS, K range u % KS); KS consecutive units
   // (run by neighbouring CTAs at the same time) share one output tile
-  const int KS = P.ksplit > 1 ? P.ksplit : 1;
+  const int KS = (!LEAN && P.ksplit > 1) ? P.ksplit : 1;
   const int units = tiles * KS;
 
-  if (P.dense_only) {
+  if (!LEAN && P.dense_only) {
     // launched next to the fused small-FC kernel, which handles the zero-skip
     // path: decide first, and leave before any set-up when it is not ours
     pdl_wait();
@@ -282,7 +292,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      mbar_init(bar_full + 8 * s, p.conv == 1 ? 129u : 1u);
+      mbar_init(bar_full + 8 * s, (!LEAN && p.conv == 1) ? 129u : 1u);
       mbar_init(bar_empty + 8 * s, 1u);
     }
     for (int b = 0; b < 2; ++b) {
@@ -320,7 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_trigger();
   const int path = decide_path(P.disp);
   // with dense_only the zero-skip kernel of this launch runs instead
-  const bool run = !(P.dense_only && path == 2);
+  const bool run = !(!LEAN && P.dense_only && path == 2);
   if (run) record_path(P.disp, path);
   const bool skip = (path == 2);
   // zero-skip GEMM with 64-wide K blocks: stages hold two occupied 32-column
@@ -482,7 +492,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (ok && pend >= 0) ok = issue(pend, -1);
           }
         }
-      } else if (p.conv != 1) {
+      } else if (LEAN || p.conv != 1) {
         if (r == 0) {
           // The issuing lane is slow at anything but issuing: ring slot, phase
           // and the (tap, channel block) of each K block advance incrementally,
@@ -580,7 +590,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     if (r == 0) *s_issued = it;  // stages this CTA filled (TMA copies issued)
-    if (p.conv == 1) {
+    if (!LEAN && p.conv == 1) {
       cp_async_wait<0>();
       fence_proxy_async_smem();
       for (int q = pending; q > 0; --q) mbar_arrive(bar_full + 8 * ((it - q) % S));
@@ -686,6 +696,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       sn_ = rho / (p.bw * p.bh);
     }
     const uint32_t stg_base = sStg + (uint32_t)(ew * 2 * kWarpStgBytes);
+    // Tile t covers columns (t % nt) BN..; when every tile of this CTA has the
+    // same columns (one column tile, or a grid that is a multiple of the column
+    // tiles) the column affine is computed once, into buffer 0, instead of per
+    // tile (its global loads would otherwise sit on every tile's critical path)
+    const bool fixed_cols = KS == 1 && (nt == 1 || (int)gridDim.x % nt == 0 || units <= (int)gridDim.x);
+    if (fixed_cols && (int)blockIdx.x < units) {
+      const int n0 = ((int)blockIdx.x % nt) * BN;
+      for (int c = et; c < BN; c += kEpiThreads) {
+        float sc = 1.f, sh = 0.f;
+        if (n0 + c < p.N) epi_affine(ep, p.N, n0 + c, sc, sh);
+        s_scale[c] = sc;
+        s_shift[c] = sh;
+      }
+    }
     int j = 0;
     int stg_count = 0;  // blocks this warp handed to TMA so far
     for (int u = blockIdx.x; u < units; u += gridDim.x, ++j) {
@@ -695,15 +719,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool mvalid;
       int img, oh, ow;
       const int64_t m = tile_row(p, g, r, mvalid, img, oh, ow);
-      float* const scb = s_scale + b * BN;
-      float* const shb = s_shift + b * BN;
+      float* const scb = s_scale + (fixed_cols ? 0 : b * BN);
+      float* const shb = s_shift + (fixed_cols ? 0 : b * BN);
       // column affine of this tile into buffer b (its readers of tile j - 2
       // passed tile j - 1's barrier before any thread gets here)
-      for (int c = et; c < BN; c += kEpiThreads) {
-        float sc = 1.f, sh = 0.f;
-        if (g.n0 + c < p.N) epi_affine(ep, p.N, g.n0 + c, sc, sh);
-        scb[c] = sc;
-        shb[c] = sh;
+      if (!fixed_cols) {
+        for (int c = et; c < BN; c += kEpiThreads) {
+          float sc = 1.f, sh = 0.f;
+          if (g.n0 + c < p.N) epi_affine(ep, p.N, g.n0 + c, sc, sh);
+          scb[c] = sc;
+          shb[c] = sh;
+        }
       }
       const bool ok = mbar_wait(bar_accf + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutAcc, wlim);
       // publishes the affine, and makes the abort decision the same for every
@@ -1067,18 +1093,39 @@ bool make_tmap_nhwc(CUtensorMap* m, const void* base, int n, int h, int w, int c
   return r == CUDA_SUCCESS;
 }
 
-template <int BN, int BK>
+template <int BN, int BK, bool LEAN>
 cudaError_t launch_cfg(const IgemmArgs& a, const CUtensorMap& tA, const CUtensorMap& tB,
                        const CUtensorMap& tY, const CUtensorMap& tA32, const CUtensorMap& tB32,
                        int64_t tiles, cudaStream_t s) {
-  cudaError_t e0 = smem_optin(reinterpret_cast<const void*>(igemm_kernel<BN, BK>), (size_t)Cfg<BN, BK>::kSmem);
+  cudaError_t e0 =
+      smem_optin(reinterpret_cast<const void*>(igemm_kernel<BN, BK, LEAN>), (size_t)Cfg<BN, BK>::kSmem);
   if (e0 != cudaSuccess) return e0;
   const int64_t units = tiles * (a.ksplit > 1 ? a.ksplit : 1);
   const int64_t grid = units < device_sm_count() ? units : device_sm_count();
-  cudaError_t e = launch_kernel(igemm_kernel<BN, BK>, dim3((unsigned)grid), dim3(kThreads),
+  cudaError_t e = launch_kernel(igemm_kernel<BN, BK, LEAN>, dim3((unsigned)grid), dim3(kThreads),
                                 (size_t)Cfg<BN, BK>::kSmem, s, tA, tB, tY, tA32, tB32, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+
+template <bool LEAN>
+cudaError_t launch_bn(const IgemmArgs& a, int bn, int bk, const CUtensorMap& tA, const CUtensorMap& tB,
+                      const CUtensorMap& tY, const CUtensorMap& tA32, const CUtensorMap& tB32, int64_t tiles,
+                      cudaStream_t s) {
+  if (bk == 64) {
+    switch (bn) {
+      case 64: return launch_cfg<64, 64, LEAN>(a, tA, tB, tY, tA32, tB32, tiles, s);
+      case 128: return launch_cfg<128, 64, LEAN>(a, tA, tB, tY, tA32, tB32, tiles, s);
+      case 192: return launch_cfg<192, 64, LEAN>(a, tA, tB, tY, tA32, tB32, tiles, s);
+      default: return launch_cfg<256, 64, LEAN>(a, tA, tB, tY, tA32, tB32, tiles, s);
+    }
+  }
+  switch (bn) {
+    case 64: return launch_cfg<64, 32, LEAN>(a, tA, tB, tY, tA32, tB32, tiles, s);
+    case 128: return launch_cfg<128, 32, LEAN>(a, tA, tB, tY, tA32, tB32, tiles, s);
+    case 192: return launch_cfg<192, 32, LEAN>(a, tA, tB, tY, tA32, tB32, tiles, s);
+    default: return launch_cfg<256, 32, LEAN>(a, tA, tB, tY, tA32, tB32, tiles, s);
+  }
 }
 
 }  // namespace
@@ -1197,20 +1244,9 @@ cudaError_t launch_igemm(const IgemmArgs& a_in, cudaStream_t s) {
       return cudaErrorInvalidValue;
   }
   const int64_t tiles = mtiles * ((a.N + bn - 1) / bn);
-  if (bk == 64) {
-    switch (bn) {
-      case 64: return launch_cfg<64, 64>(a, tA, tB, tY, tA32, tB32, tiles, s);
-      case 128: return launch_cfg<128, 64>(a, tA, tB, tY, tA32, tB32, tiles, s);
-      case 192: return launch_cfg<192, 64>(a, tA, tB, tY, tA32, tB32, tiles, s);
-      default: return launch_cfg<256, 64>(a, tA, tB, tY, tA32, tB32, tiles, s);
-    }
-  }
-  switch (bn) {
-    case 64: return launch_cfg<64, 32>(a, tA, tB, tY, tA32, tB32, tiles, s);
-    case 128: return launch_cfg<128, 32>(a, tA, tB, tY, tA32, tB32, tiles, s);
-    case 192: return launch_cfg<192, 32>(a, tA, tB, tY, tA32, tB32, tiles, s);
-    default: return launch_cfg<256, 32>(a, tA, tB, tY, tA32, tB32, tiles, s);
-  }
+  const bool lean = a.conv != 1 && ks == 1 && !a.y_f32 && a.ep.residual == nullptr && !a.dense_only;
+  return lean ? launch_bn<true>(a, bn, bk, tA, tB, tY, tA32, tB32, tiles, s)
+              : launch_bn<false>(a, bn, bk, tA, tB, tY, tA32, tB32, tiles, s);
 }
 
 }  // namespace sparoa
