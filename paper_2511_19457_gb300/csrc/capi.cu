@@ -1048,25 +1048,25 @@ sparoa_status sparoa_conv2d(sparoa_ctx* ctx, const void* x, int64_t N, int64_t H
       c.x = x;
       c.w = w;
       int ckh = kh, ckw = kw, cstride = stride, cpad = pad;
-      bool rows = false;
-      if (im2row_applies((int)C_in, kw, groups)) {
-        // a narrow stem as a kh x 1 convolution of window rows over 32 channels
-        const int64_t Hx = H + 2 * pad, Wx = W + 2 * pad - kw + 1;
-        SP_TRY(ensure(ctx, ctx->pad_x, (size_t)(N * Hx * Wx * 32 * 2)));
-        SP_TRY(ensure(ctx, ctx->pad_w, (size_t)(C_out * kh * 32 * 2)));
-        SP_CUDA(launch_im2row(static_cast<const __nv_bfloat16*>(x), (int)N, (int)H, (int)W, (int)C_in, kw, pad,
-                              static_cast<__nv_bfloat16*>(ctx->pad_x.p), ctx->stream));
-        SP_CUDA(launch_pad_channels(static_cast<const __nv_bfloat16*>(w), C_out * kh, kw * (int)C_in, 32,
+      bool cols = false;
+      if (im2col_applies((int)C_in, kh, kw, groups, (int)W, pad)) {
+        // a narrow stem as a GEMM of its im2col rows (a 1 x 1 conv over Kp channels)
+        const int Kp = im2col_width((int)C_in, kh, kw);
+        SP_TRY(ensure(ctx, ctx->pad_x, (size_t)(N * Ho * Wo * Kp * 2)));
+        SP_TRY(ensure(ctx, ctx->pad_w, (size_t)(C_out * Kp * 2)));
+        SP_CUDA(launch_im2col(static_cast<const __nv_bfloat16*>(x), (int)N, (int)H, (int)W, (int)C_in, kh, kw,
+                              stride, pad, static_cast<__nv_bfloat16*>(ctx->pad_x.p), ctx->stream));
+        SP_CUDA(launch_pad_channels(static_cast<const __nv_bfloat16*>(w), C_out, kh * kw * (int)C_in, Kp,
                                     static_cast<__nv_bfloat16*>(ctx->pad_w.p), ctx->stream));
         c.x = ctx->pad_x.p;
         c.w = ctx->pad_w.p;
-        c.H = Hx;
-        c.W = Wx;
-        c.Cin = 32;
-        c.Cp = 32;
-        ckw = 1;
+        c.H = Ho;
+        c.W = Wo;
+        c.Cin = Kp;
+        c.Cp = Kp;
+        ckh = ckw = cstride = 1;
         cpad = 0;
-        rows = true;
+        cols = true;
       } else if (c.Cp != C_in) {
         const int64_t P = N * H * W, Q = C_out * kh * kw;
         SP_TRY(ensure(ctx, ctx->pad_x, (size_t)(P * c.Cp * 2)));
@@ -1088,7 +1088,7 @@ sparoa_status sparoa_conv2d(sparoa_ctx* ctx, const void* x, int64_t N, int64_t H
       c.ep = to_dev(ep);
       c.y = y;
       c.xo = xo;
-      if (rows) {  // the window rows have no occupancy: every K block is kept
+      if (cols) {  // the im2col rows have no occupancy: every K block is kept
         c.xo.blk_mask = nullptr;
         c.xo.row_bm = nullptr;
       }
@@ -1227,7 +1227,7 @@ struct Val {
 struct Aux {
   size_t padx = 0, padw = 0, fcocc = 0;
   int64_t cp = 0;
-  bool rows = false;  // narrow stem as window rows (im2row_applies)
+  bool cols = false;  // narrow stem as a GEMM of its im2col rows (im2col_applies)
   bool fc_view = false;
 };
 struct GraphPlan {
@@ -1266,9 +1266,9 @@ sparoa_status plan_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_ops, i
                op.c_out};
         if (out.h <= 0 || out.w <= 0)
           return fail(ctx, SPAROA_ERR_INVALID_ARG, "run_graph: op %d empty output", i);
-        if (!dw && im2row_applies(op.c_in, op.kw, op.groups)) {
-          aux[(size_t)i].rows = true;
-          aux[(size_t)i].cp = 32;
+        if (!dw && im2col_applies(op.c_in, op.kh, op.kw, op.groups, (int)in.w, op.pad)) {
+          aux[(size_t)i].cols = true;
+          aux[(size_t)i].cp = im2col_width(op.c_in, op.kh, op.kw);
         } else if (!dw && op.c_in % 8) {
           aux[(size_t)i].cp = (op.c_in + 7) / 8 * 8;
         }
@@ -1358,13 +1358,12 @@ sparoa_status plan_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_ops, i
     off += align_up((size_t)(vals[v].n * vals[v].h * vals[v].w * vals[v].c) * 2);
   }
   for (int i = 0; i < n_ops; ++i) {
-    if (aux[(size_t)i].rows) {
-      const Val& in = vals[(size_t)ops[i].input];
-      const int64_t Hx = in.h + 2 * ops[i].pad, Wx = in.w + 2 * ops[i].pad - ops[i].kw + 1;
+    if (aux[(size_t)i].cols) {
+      const Val& out = vals[(size_t)i + 1];
       aux[(size_t)i].padx = off;
-      off += align_up((size_t)(in.n * Hx * Wx * 32) * 2);
+      off += align_up((size_t)(out.n * out.h * out.w * aux[(size_t)i].cp) * 2);
       aux[(size_t)i].padw = off;
-      off += align_up((size_t)(ops[i].c_out * ops[i].kh * 32) * 2);
+      off += align_up((size_t)(ops[i].c_out * aux[(size_t)i].cp) * 2);
     } else if (aux[(size_t)i].cp) {
       const Val& in = vals[(size_t)ops[i].input];
       aux[(size_t)i].padx = off;
@@ -1483,19 +1482,20 @@ sparoa_status sparoa_run_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_
         c.Cp = aux[(size_t)i].cp ? aux[(size_t)i].cp : in.c;
         c.x = act(op.input);
         c.w = op.weight;
-        const bool rows = aux[(size_t)i].rows;
-        if (rows) {  // a narrow stem as a kh x 1 convolution of window rows over 32 channels
+        const bool cols = aux[(size_t)i].cols;
+        if (cols) {  // a narrow stem as a GEMM of its im2col rows (a 1 x 1 conv over Kp channels)
           void* px = base + aux[(size_t)i].padx;
           void* pw = base + aux[(size_t)i].padw;
-          SP_CUDA(launch_im2row(static_cast<const __nv_bfloat16*>(c.x), (int)in.n, (int)in.h, (int)in.w, (int)in.c,
-                                op.kw, op.pad, static_cast<__nv_bfloat16*>(px), ctx->stream));
-          SP_CUDA(launch_pad_channels(static_cast<const __nv_bfloat16*>(op.weight), (int64_t)op.c_out * op.kh,
-                                      op.kw * (int)in.c, 32, static_cast<__nv_bfloat16*>(pw), ctx->stream));
+          SP_CUDA(launch_im2col(static_cast<const __nv_bfloat16*>(c.x), (int)in.n, (int)in.h, (int)in.w, (int)in.c,
+                                op.kh, op.kw, op.stride, op.pad, static_cast<__nv_bfloat16*>(px), ctx->stream));
+          SP_CUDA(launch_pad_channels(static_cast<const __nv_bfloat16*>(op.weight), (int64_t)op.c_out,
+                                      op.kh * op.kw * (int)in.c, (int)c.Cp, static_cast<__nv_bfloat16*>(pw),
+                                      ctx->stream));
           c.x = px;
           c.w = pw;
-          c.H = in.h + 2 * op.pad;
-          c.W = in.w + 2 * op.pad - op.kw + 1;
-          c.Cin = 32;
+          c.H = out.h;
+          c.W = out.w;
+          c.Cin = c.Cp;
         } else if (aux[(size_t)i].cp) {
           const int64_t P = in.n * in.h * in.w, Q = (int64_t)op.c_out * op.kh * op.kw;
           void* px = base + aux[(size_t)i].padx;
@@ -1508,16 +1508,16 @@ sparoa_status sparoa_run_graph(sparoa_ctx* ctx, const sparoa_op* ops, int32_t n_
           c.w = pw;
         }
         c.Cout = op.c_out;
-        c.kh = op.kh;
-        c.kw = rows ? 1 : op.kw;
-        c.stride = op.stride;
-        c.pad = rows ? 0 : op.pad;
+        c.kh = cols ? 1 : op.kh;
+        c.kw = cols ? 1 : op.kw;
+        c.stride = cols ? 1 : op.stride;
+        c.pad = cols ? 0 : op.pad;
         c.Ho = out.h;
         c.Wo = out.w;
         c.ep = ep;
         c.y = act(i + 1);
         c.xo = xo;
-        if (rows) {  // the window rows have no occupancy: every K block is kept
+        if (cols) {  // the im2col rows have no occupancy: every K block is kept
           c.xo.blk_mask = nullptr;
           c.xo.row_bm = nullptr;
         }

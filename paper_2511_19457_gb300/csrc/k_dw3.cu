@@ -69,49 +69,12 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const void* tmap, uint
       : "memory");
 }
 
-typedef unsigned long long f2_t;  // two fp32 values (low: even channel)
-
-__device__ __forceinline__ f2_t f2(float lo, float hi) {
-  f2_t r;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
-  return r;
-}
-__device__ __forceinline__ void f2_split(f2_t v, float& lo, float& hi) {
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
-}
-__device__ __forceinline__ f2_t ffma2(f2_t a, f2_t b, f2_t c) {
-  f2_t d;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
-  return d;
-}
 // a bf16 pair widened to fp32 (exact)
 __device__ __forceinline__ f2_t widen(uint32_t w) {
   return f2(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
 }
 
-// bit 0 / bit 16: the low / high bf16 of w is non-zero (any bit but the sign)
-__device__ __forceinline__ uint32_t nz_pairs(uint32_t w) {
-  return (((w & 0x7FFF7FFFu) + 0x7FFF7FFFu) >> 15) & 0x00010001u;
-}
 
-// Two fp32 values through the activation to a bf16 pair (round to nearest
-// even); ReLU is applied by the conversion.
-template <int ACT>
-__device__ __forceinline__ uint32_t act_pack2(float lo, float hi) {
-  if (ACT == 2) {
-    lo = fminf(fmaxf(lo, 0.f), 6.f);
-    hi = fminf(fmaxf(hi, 0.f), 6.f);
-  } else if (ACT == 3) {
-    lo = gelu_f(lo);
-    hi = gelu_f(hi);
-  }
-  uint32_t d;
-  if (ACT == 1)
-    asm("cvt.rn.relu.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
-  else
-    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
-  return d;
-}
 
 struct Step {
   long long item;

@@ -36,8 +36,9 @@
 // lane quarter, each taking 32 of every 64 accumulator columns), warp 12 TMEM
 // allocation and MMA issue (lane 0).
 //
-// Each tile shape is compiled twice: the general kernel, and a lean one for
-// modes 0 and 2 without a K split, residual or fp32 output.  With small K the
+// Each tile shape is compiled three times: the general kernel, and lean ones
+// for modes 0 and 2 without a K split or fp32 output, without a residual and
+// with one (N % 32 == 0).  With small K the
 // epilogue is the whole cost of a tile and runs at a fraction of an
 // instruction per cycle (few warps, long dependency chains); the lean kernel's
 // smaller, branch-free epilogue issues fewer instructions per tile and misses
@@ -63,7 +64,7 @@ constexpr int kMaxKWords = 128;  // K-block occupancy bits: up to 4096 blocks
 constexpr int kMaxTaps = 64;
 constexpr int kStgBytes = 128 * 128;  // output staging: per epilogue warp 2 blocks of 32 rows x 64 bytes
 constexpr int kWarpStgBytes = 32 * 64;
-constexpr int kMaxAccCols = 2048;     // per-CTA column counters (output occupancy)
+constexpr int kMaxAccCols = 4096;     // per-CTA column counters (output occupancy)
 
 template <int BN, int BK>
 struct Cfg {
@@ -77,8 +78,8 @@ struct Cfg {
   // but the ring (barriers and flags of at most 12 stages) plus the 1024 bytes
   // of alignment slack.
   static constexpr int kFixed = 2 * kStgBytes + (2 * 12 + 5) * 8 + (12 + 8) * 4 + 16 + kMaxKWords * 4 +
-                                kMaxTaps * 8 + 4 * BN * 4 + 4 * BN * 4 + kMaxAccCols * 4 + kBM * 8 +
-                                (BN / 32) * 4 + 16 + 1024;
+                                kMaxTaps * 8 + 4 * BN * 4 + 4 * BN * 4 + kMaxAccCols * 4 + 2 * kBM * 8 +
+                                2 * (BN / 32) * 4 + 16 + 1024;
   static constexpr int kBudget =
       BN == 192 ? 227 * 1024 - kFixed : 200 * 1024 - 2 * kStgBytes - 6 * 1024 - kMaxAccCols * 4;
   static constexpr int kStagesRaw = kBudget / kStageBytes;
@@ -96,9 +97,9 @@ struct Cfg {
   static constexpr int kShiftOff = kScaleOff + 2 * BN * 4;  // scale / shift: [2 accumulators][BN]
   static constexpr int kCntOff = kShiftOff + 2 * BN * 4;
   static constexpr int kAccOff = kCntOff + 4 * BN * 4;
-  static constexpr int kRowOff = kAccOff + kMaxAccCols * 4;   // [128] row bits of the tile
-  static constexpr int kBlkOff = kRowOff + kBM * 8;           // [BN / 32] block-mask words
-  static constexpr int kBytes = kBlkOff + (BN / 32) * 4 + 16;
+  static constexpr int kRowOff = kAccOff + kMaxAccCols * 4;   // [2][128] row bits of the tile
+  static constexpr int kBlkOff = kRowOff + 2 * kBM * 8;       // [2][BN / 32] block-mask words
+  static constexpr int kBytes = kBlkOff + 2 * (BN / 32) * 4 + 16;
   static constexpr int kSmem = kBytes + 1024;  // slack for 1024-byte alignment
   // TMEM: accumulator b starts at column b * kAccCols (BN rounded up to a
   // power of two, so each starts on a power-of-two column); the allocation
@@ -180,6 +181,75 @@ __device__ __forceinline__ int64_t tile_row(const Geo& p, const TileGeo& g, int 
   return m;
 }
 
+// One row's 32 accumulator values (fp32 bits) through the column affine
+// (scale and shift from shared memory; none when sc is null), the residual
+// (32 bf16 at rp, none when rp is null) and the activation, packed to 16 bf16
+// pairs: fp32x2 FMAs, ReLU folded into the conversion.  The same operations
+// in the same order as the general epilogue (fmaf, then + residual, then the
+// activation, then round to bf16).
+template <int ACT, bool RES>
+__device__ __forceinline__ void affine_act_pack32(const uint32_t (&raw)[32], const float* sc, const float* sh,
+                                                  const uint4* rp, uint32_t (&pk)[16]) {
+  uint4 rv = make_uint4(0u, 0u, 0u, 0u);  // residual values 8 (i / 2) .. + 7
+  if (!RES) rp = nullptr;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    if (RES && rp && (i & 1) == 0) rv = rp[i >> 1];
+    if (sc == nullptr && rp == nullptr) {  // the accumulators as they are
+      pk[2 * i] = act_pack2<ACT>(__uint_as_float(raw[4 * i]), __uint_as_float(raw[4 * i + 1]));
+      pk[2 * i + 1] = act_pack2<ACT>(__uint_as_float(raw[4 * i + 2]), __uint_as_float(raw[4 * i + 3]));
+      continue;
+    }
+    if (sc == nullptr) {
+      float a = __uint_as_float(raw[4 * i]), b = __uint_as_float(raw[4 * i + 1]);
+      float c = __uint_as_float(raw[4 * i + 2]), d = __uint_as_float(raw[4 * i + 3]);
+      const uint32_t w0 = (i & 1) ? rv.z : rv.x, w1 = (i & 1) ? rv.w : rv.y;
+      a += __uint_as_float(w0 << 16);
+      b += __uint_as_float(w0 & 0xFFFF0000u);
+      c += __uint_as_float(w1 << 16);
+      d += __uint_as_float(w1 & 0xFFFF0000u);
+      pk[2 * i] = act_pack2<ACT>(a, b);
+      pk[2 * i + 1] = act_pack2<ACT>(c, d);
+      continue;
+    }
+    const float4 s4 = reinterpret_cast<const float4*>(sc)[i];
+    const float4 h4 = reinterpret_cast<const float4*>(sh)[i];
+    float a, b, c, d;
+    f2_split(ffma2(f2(__uint_as_float(raw[4 * i]), __uint_as_float(raw[4 * i + 1])), f2(s4.x, s4.y),
+                   f2(h4.x, h4.y)),
+             a, b);
+    f2_split(ffma2(f2(__uint_as_float(raw[4 * i + 2]), __uint_as_float(raw[4 * i + 3])), f2(s4.z, s4.w),
+                   f2(h4.z, h4.w)),
+             c, d);
+    if (RES && rp) {
+      const uint32_t w0 = (i & 1) ? rv.z : rv.x, w1 = (i & 1) ? rv.w : rv.y;
+      a += __uint_as_float(w0 << 16);
+      b += __uint_as_float(w0 & 0xFFFF0000u);
+      c += __uint_as_float(w1 << 16);
+      d += __uint_as_float(w1 & 0xFFFF0000u);
+    }
+    pk[2 * i] = act_pack2<ACT>(a, b);
+    pk[2 * i + 1] = act_pack2<ACT>(c, d);
+  }
+}
+
+// Bit c of the result: bf16 value c of the 16 packed pairs is non-zero.  Per
+// two words: the non-zero flags of their four halves (bits 15 and 31 after
+// nz_pairs' carry trick) are gathered into one word's byte tops (bits 7, 15,
+// 23, 31) by a byte permute, and the multiply by 1 + 2^7 + 2^14 + 2^21 moves
+// them, without carries, to bits 28..31.
+__device__ __forceinline__ uint32_t nz_mask32(const uint32_t (&pk)[16]) {
+  uint32_t m = 0u;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const uint32_t ta = (pk[2 * i] & 0x7FFF7FFFu) + 0x7FFF7FFFu;
+    const uint32_t tb = (pk[2 * i + 1] & 0x7FFF7FFFu) + 0x7FFF7FFFu;
+    const uint32_t x = __byte_perm(ta, tb, 0x7531) & 0x80808080u;
+    m |= ((x * 0x00204081u) >> 28) << (4 * i);
+  }
+  return m;
+}
+
 // Everything a producer thread needs to know about work unit u (tile u / ks,
 // K range u % ks): pure arithmetic on the parameters, 32-bit throughout.
 struct UnitGeo {
@@ -213,19 +283,20 @@ __device__ __forceinline__ UnitGeo unit_geo(const Geo& p, int u, int KS, int kbl
   return q;
 }
 
-template <int BN, int BK, bool LEAN>
+template <int BN, int BK, int LEAN>
 __global__ void __launch_bounds__(kThreads, 1)
     igemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                  const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmA32,
                  const __grid_constant__ CUtensorMap tmB32, const IgemmArgs P) {
   using C = Cfg<BN, BK>;
   const Geo p = make_geo(P);
-  // lean kernel: TMA producers only (mode 0 or 2), no K split, bf16 output
-  // without residual (the host launches it only then)
+  // lean kernels (LEAN 1: no residual, 2: a residual and N % 32 == 0): TMA
+  // producers only (mode 0 or 2), no K split, bf16 output (the host launches
+  // them only then)
   if (LEAN) __builtin_assume(p.conv != 1);
   const EpiDev ep = P.ep;
   const int act = P.ep.act;
-  const __nv_bfloat16* const residual = LEAN ? nullptr : P.ep.residual;
+  const __nv_bfloat16* const residual = LEAN == 1 ? nullptr : P.ep.residual;
   const int y_f32 = LEAN ? 0 : P.y_f32;
   const int emit = P.emit;
   const long long wlim = P.wait_limit > 0 ? P.wait_limit : kWaitLimitCycles;
@@ -314,8 +385,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (acc_smem && warp >= 4 && warp < kMmaWarp)
     for (int c = threadIdx.x - 128; c < p.N; c += kEpiThreads) s_acc[c] = 0u;
   if (warp >= 4 && warp < kMmaWarp) {
-    for (int i = threadIdx.x - 128; i < kBM; i += kEpiThreads) s_rowbm[i] = 0ull;
-    for (int i = threadIdx.x - 128; i < BN / 32; i += kEpiThreads) s_blk[i] = 0u;
+    for (int i = threadIdx.x - 128; i < 2 * kBM; i += kEpiThreads) s_rowbm[i] = 0ull;
+    for (int i = threadIdx.x - 128; i < 2 * (BN / 32); i += kEpiThreads) s_blk[i] = 0u;
   }
   // The producers' first work unit is laid out before the grid dependency
   // wait: no memory is read, and under programmatic dependent launch this
@@ -335,7 +406,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const bool skip = (path == 2);
   // zero-skip GEMM with 64-wide K blocks: stages hold two occupied 32-column
   // groups each (compacted), loaded as 32-column boxes with the 64-byte swizzle
-  const bool compact = skip && p.conv == 0 && BK == 64 && kgroups <= kMaxKWords * 32;
+  const bool compact = skip && p.conv == 0 && BK == 64 && kgroups <= kMaxKWords * 32 && in_blk != nullptr;
 
   if (!run) {
     // nothing to do; fall through to the common exit (TMEM is freed there)
@@ -346,7 +417,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     int it = 0;        // stages filled so far (ring position)
     int pending = 0;   // mode 1: filled stages whose A arrivals are still owed
     bool ok = true;
-    for (int u = blockIdx.x; u < units; u += gridDim.x) {
+    // dense TMA modes: thread 0 issues everything, the other producer threads
+    // have no part in the loop (their tile geometry would only take issue
+    // slots from the epilogue warps on the same schedulers)
+    const bool lone = !skip && (LEAN || p.conv != 1);
+    for (int u = (lone && r != 0) ? units : (int)blockIdx.x; u < units; u += gridDim.x) {
       if (u != (int)blockIdx.x) ug = unit_geo(p, u, KS, kblocks, nt, BN, BK, r);
       const int kb0 = ug.kb0, kb1 = ug.kb1;
       const TileGeo g = ug.g;
@@ -371,8 +446,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int w0 = 0; w0 < kblocks && w0 < kMaxKWords * 32; w0 += 128) {
             const int kb = w0 + r;
             // a K block covers BK / 32 words of the 128-row block-column mask
+            // (an input without block masks, such as the im2col rows of a
+            // narrow stem, keeps every block)
             bool occ = false;
-            if (kb < kblocks) {
+            if (kb < kblocks && in_blk == nullptr) {
+              occ = true;
+            } else if (kb < kblocks) {
               const uint32_t* words = in_blk + (int64_t)(g.m0 >> 7) * in_C32;
               occ = words[kb * (BK / 32)] != 0u;
               if (BK == 64 && kb * 2 + 1 < in_C32) occ |= words[kb * 2 + 1] != 0u;
@@ -671,6 +750,195 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (ok && !(P.fault == kFaultSkipFirstAccCommit && j == 0)) tc_commit(bar_accf + 8 * b);
       }
     }
+  } else if constexpr (LEAN) {
+    // ------------------------------------------------------------- lean epilogue
+    // The general epilogue's blocks (32 rows of one TMEM lane quarter x 32
+    // columns, staged with the 64-byte swizzle, one TMA store each) without
+    // K split or fp32 output, and with one barrier per tile: the
+    // output occupancy a tile leaves in shared memory (row bitmaps and block-
+    // column words, buffer j & 1) is written out after the next tile's
+    // barrier, and column counts go straight into the CTA's column sums.
+    const int q = warp & 3;
+    const int hf = (warp - 4) >> 2;
+    const int ew = warp - 4;
+    const int r = q * 32 + lane;
+    const int et = threadIdx.x - 128;
+    int sw_ = 0, sh_ = 0, sn_ = 0;
+    if (p.conv == 2) {
+      const int rho = q * 32;
+      sw_ = rho % p.bw;
+      sh_ = (rho / p.bw) % p.bh;
+      sn_ = rho / (p.bw * p.bh);
+    }
+    const uint32_t stg_base = sStg + (uint32_t)(ew * 2 * kWarpStgBytes);
+    const bool fixed_cols = nt == 1 || (int)gridDim.x % nt == 0 || units <= (int)gridDim.x;
+    if (fixed_cols && (int)blockIdx.x < units) {
+      const int n0 = ((int)blockIdx.x % nt) * BN;
+      for (int c = et; c < BN; c += kEpiThreads) {
+        float sc = 1.f, sh = 0.f;
+        if (n0 + c < p.N) epi_affine(ep, p.N, n0 + c, sc, sh);
+        s_scale[c] = sc;
+        s_shift[c] = sh;
+      }
+    }
+    const bool affine = ep.bias != nullptr || ep.bn != nullptr;  // else the column affine is 1, 0
+    const OccDev o = P.out_occ;
+    // Writes out the occupancy that tile (m0, n0) left in buffer pb: the row
+    // bitmap word of row r (its half-0 thread) and the block-column words of
+    // its 128-row block (mode 0: the tile is that block).
+    auto flush_tile = [&](int pb, int64_t m_t, bool v_t, int m0_t, int n0_t) {
+      if (hf == 0) {
+        unsigned long long* const srow = s_rowbm + pb * kBM + r;
+        const unsigned long long v = *srow;
+        *srow = 0ull;
+        if (v_t) {
+          unsigned long long* dst = &o.row_bm[m_t * o.W64 + (n0_t >> 12)];
+          if (nt == 1) *dst = v;  // the tile spans the row's whole bitmap word
+          else if (v) atomicOr(dst, v);
+        }
+      }
+      if (p.conv != 2 && et < BN / 32) {
+        uint32_t* const sb = s_blk + pb * (BN / 32) + et;
+        const uint32_t v = *sb;
+        *sb = 0u;
+        const int word = (n0_t >> 5) + et;
+        if (word < o.C32) o.blk_mask[(m0_t >> 7) * o.C32 + word] = v;
+      }
+    };
+    int j = 0;
+    int stg_count = 0;
+    int64_t m_prev = 0;
+    bool v_prev = false;
+    int m0_prev = 0, n0_prev = 0;
+    for (int u = blockIdx.x; u < units; u += gridDim.x, ++j) {
+      const int b = j & 1;
+      const TileGeo g = tile_geo(p, u, nt, BN);
+      bool mvalid;
+      int img, oh, ow;
+      const int64_t m = tile_row(p, g, r, mvalid, img, oh, ow);
+      float* const scb = s_scale + (fixed_cols ? 0 : b * BN);
+      float* const shb = s_shift + (fixed_cols ? 0 : b * BN);
+      if (!fixed_cols) {
+        for (int c = et; c < BN; c += kEpiThreads) {
+          float sc = 1.f, sh = 0.f;
+          if (g.n0 + c < p.N) epi_affine(ep, p.N, g.n0 + c, sc, sh);
+          scb[c] = sc;
+          shb[c] = sh;
+        }
+      }
+      const bool ok = mbar_wait(bar_accf + 8 * b, (uint32_t)((j >> 1) & 1), err, s_abort, kErrTimeoutAcc, wlim);
+      if (named_bar_or(2, kEpiThreads, !ok)) break;
+      if (emit && j > 0) flush_tile(b ^ 1, m_prev, v_prev, m0_prev, n0_prev);
+      tc_fence_after();
+      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)b * C::kAccCols;
+      const int blk = mvalid ? (int)(m >> 7) : -1;
+      const uint32_t grp = p.conv == 2 ? __match_any_sync(0xffffffffu, blk) : 0xffffffffu;
+      const bool leader = (__ffs(grp) - 1) == lane;
+      unsigned long long tl = 0ull;
+      // One block: columns ncol0..+31 of 64-column group gcol, accumulator
+      // values in raw, staged in buffer stg; the TMA store and this block's
+      // share of the output occupancy.
+      auto block = [&](const uint32_t (&raw)[32], int gcol, uint32_t stg) {
+        const int nbase = g.n0 + gcol * 64;
+        const int ncol0 = nbase + hf * 32;
+        const float* scg = affine ? scb + gcol * 64 + hf * 32 : nullptr;
+        const float* shg = shb + gcol * 64 + hf * 32;
+        const uint4* rp =
+            residual && mvalid ? reinterpret_cast<const uint4*>(residual + m * p.N + ncol0) : nullptr;
+        uint32_t pk[16];
+        constexpr bool kRes = LEAN == 2;
+        if (act == 1) affine_act_pack32<1, kRes>(raw, scg, shg, rp, pk);
+        else if (act == 2) affine_act_pack32<2, kRes>(raw, scg, shg, rp, pk);
+        else if (act == 0) affine_act_pack32<0, kRes>(raw, scg, shg, rp, pk);
+        else affine_act_pack32<3, kRes>(raw, scg, shg, rp, pk);
+        const uint32_t row_addr = stg + (uint32_t)lane * 64u;
+        const int sx = (lane >> 1) & 3;
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          sts_u4(row_addr + (uint32_t)((k ^ sx) << 4), make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]));
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          if (p.conv == 2)
+            tma_store_4d(&tmY, stg, ncol0, g.tw0 + sw_, g.th0 + sh_, g.tn0 + sn_);
+          else
+            tma_store_2d(&tmY, stg, ncol0, g.m0 + q * 32);
+          bulk_commit();
+        }
+        if (emit) {
+          uint32_t rw = nz_mask32(pk);  // bit c: column ncol0 + c of row r is non-zero
+          const int nvalid = p.N - ncol0;
+          if (!mvalid) rw = 0u;
+          else if (nvalid < 32) rw &= nvalid > 0 ? ((1u << nvalid) - 1u) : 0u;
+          if (rw) tl |= 1ull << ((nbase >> 6) & 63);
+          const uint32_t bits = __reduce_or_sync(grp, rw);
+          const int word = ncol0 >> 5;
+          if (leader && blk >= 0 && bits && word < o.C32) {
+            if (p.conv == 2) atomicOr(&o.blk_mask[blk * o.C32 + word], bits);
+            else atomicOr(&s_blk[b * (BN / 32) + gcol * 2 + hf], bits);  // the tile is the whole block
+          }
+          // lane c: non-zeros of column ncol0 + c in the warp's 32 rows
+          const uint32_t cnt = __popc(warp_transpose32(rw));
+          const int col = ncol0 + lane;
+          if (acc_smem) {
+            if (cnt) atomicAdd(&s_acc[col], cnt);
+          } else if (col < o.C) {
+            if (cnt) atomicAdd(&o.col_nnz[col], cnt);
+            const uint32_t sum = __reduce_add_sync(0xffffffffu, cnt);
+            if (lane == 0 && sum) {
+              atomicAdd(&o.tile_nnz[ncol0 >> 6], sum);
+              atomicAdd(o.nnz, (unsigned long long)sum);
+            }
+          }
+        }
+      };
+      // This warp's blocks of the tile (32-column halves past N have none).
+      // (Two blocks per step, both accumulator loads in flight first, made
+      // the kernel spill and was slower.)
+      int nblk = 0;
+      for (int gc = 0; gc < BN / 64; ++gc) nblk += (g.n0 + gc * 64 + hf * 32 < p.N) ? 1 : 0;
+#pragma unroll 1
+      for (int gcol = 0; gcol < nblk; ++gcol) {
+        const uint32_t stg = stg_base + (uint32_t)((stg_count & 1) * kWarpStgBytes);
+        if (lane == 0) bulk_wait_read<1>();  // the store that used this buffer has read it
+        __syncwarp();
+        uint32_t raw[32];
+        tmem_ld32_nowait(tbase + (uint32_t)(gcol * 64 + hf * 32), raw);
+        tmem_wait_ld32(raw);
+        block(raw, gcol, stg);
+        ++stg_count;
+      }
+      // accumulator b is free for the MMA of tile j + 2
+      tc_fence_before();
+      mbar_arrive(bar_acce + 8 * b);
+      if (emit) {
+        if (tl) atomicOr(&s_rowbm[b * kBM + r], tl);
+        m_prev = m;
+        v_prev = mvalid;
+        m0_prev = g.m0;
+        n0_prev = g.n0;
+      }
+    }
+    if (emit) {
+      named_bar_sync(2, kEpiThreads);  // the last tile's shared-memory occupancy is complete
+      if (j > 0) flush_tile((j - 1) & 1, m_prev, v_prev, m0_prev, n0_prev);
+    }
+    if (acc_smem) {
+      named_bar_sync(2, kEpiThreads);
+      unsigned long long total = 0ull;
+      for (int c0 = 0; c0 < p.N; c0 += kEpiThreads) {
+        const int c = c0 + et;
+        const uint32_t cnt = c < p.N ? s_acc[c] : 0u;
+        if (cnt) atomicAdd(&o.col_nnz[c], cnt);
+        uint32_t sum = cnt;
+#pragma unroll
+        for (int s = 16; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
+        total += sum;
+        if (lane == 0 && sum) atomicAdd(&o.tile_nnz[c >> 6], sum);
+      }
+      if (lane == 0 && total) atomicAdd(o.nnz, total);
+    }
+    if (lane == 0) bulk_wait_all();
   } else {
     // ------------------------------------------------------------------ epilogue
     // Each epilogue warp owns a 32-row x 32-column block of every 64-column
@@ -1093,7 +1361,7 @@ bool make_tmap_nhwc(CUtensorMap* m, const void* base, int n, int h, int w, int c
   return r == CUDA_SUCCESS;
 }
 
-template <int BN, int BK, bool LEAN>
+template <int BN, int BK, int LEAN>
 cudaError_t launch_cfg(const IgemmArgs& a, const CUtensorMap& tA, const CUtensorMap& tB,
                        const CUtensorMap& tY, const CUtensorMap& tA32, const CUtensorMap& tB32,
                        int64_t tiles, cudaStream_t s) {
@@ -1108,7 +1376,7 @@ cudaError_t launch_cfg(const IgemmArgs& a, const CUtensorMap& tA, const CUtensor
   return cudaGetLastError();
 }
 
-template <bool LEAN>
+template <int LEAN>
 cudaError_t launch_bn(const IgemmArgs& a, int bn, int bk, const CUtensorMap& tA, const CUtensorMap& tB,
                       const CUtensorMap& tY, const CUtensorMap& tA32, const CUtensorMap& tB32, int64_t tiles,
                       cudaStream_t s) {
@@ -1244,9 +1512,12 @@ cudaError_t launch_igemm(const IgemmArgs& a_in, cudaStream_t s) {
       return cudaErrorInvalidValue;
   }
   const int64_t tiles = mtiles * ((a.N + bn - 1) / bn);
-  const bool lean = a.conv != 1 && ks == 1 && !a.y_f32 && a.ep.residual == nullptr && !a.dense_only;
-  return lean ? launch_bn<true>(a, bn, bk, tA, tB, tY, tA32, tB32, tiles, s)
-              : launch_bn<false>(a, bn, bk, tA, tB, tY, tA32, tB32, tiles, s);
+  const bool lean = a.conv != 1 && ks == 1 && !a.y_f32 && !a.dense_only &&
+                    (a.ep.residual == nullptr ||
+                     (a.N % 32 == 0 && (reinterpret_cast<uintptr_t>(a.ep.residual) & 15u) == 0));
+  if (!lean) return launch_bn<0>(a, bn, bk, tA, tB, tY, tA32, tB32, tiles, s);
+  return a.ep.residual ? launch_bn<2>(a, bn, bk, tA, tB, tY, tA32, tB32, tiles, s)
+                       : launch_bn<1>(a, bn, bk, tA, tB, tY, tA32, tB32, tiles, s);
 }
 
 }  // namespace sparoa

@@ -283,12 +283,6 @@ __global__ void __launch_bounds__(kTileThreads, 3) stats_scalar_kernel(const __n
 // flight while a tile is reduced.
 constexpr int kStatsRunTiles = 8192;  // tiles per run: 4 rows each, under the 16-bit counters' 65535
 
-// bit 0 / bit 16 set where the low / high bf16 of w is non-zero (any bit but
-// the sign): adding 0x7FFF to a 15-bit magnitude carries into bit 15 exactly
-// when the magnitude is not zero, and never out of its 16-bit half
-__device__ __forceinline__ uint32_t nz_pairs(uint32_t w) {
-  return (((w & 0x7FFF7FFFu) + 0x7FFF7FFFu) >> 15) & 0x00010001u;
-}
 
 // Grid-stride zeroing of up to five word ranges.
 __device__ __forceinline__ void zero_ranges(const ClearArgs& a) {
@@ -540,24 +534,6 @@ __device__ __forceinline__ void stream_tile(StreamEmit& e, const uint32_t (&n)[4
   }
 }
 
-// Two fp32 values through the activation to a bf16 pair (round to nearest
-// even), `lo` in the low half; ReLU is applied by the conversion itself.
-template <int ACT>
-__device__ __forceinline__ uint32_t act_pack2(float lo, float hi) {
-  if (ACT == 2) {
-    lo = fminf(fmaxf(lo, 0.f), 6.f);
-    hi = fminf(fmaxf(hi, 0.f), 6.f);
-  } else if (ACT == 3) {
-    lo = gelu_f(lo);
-    hi = gelu_f(hi);
-  }
-  uint32_t d;
-  if (ACT == 1)
-    asm("cvt.rn.relu.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
-  else
-    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
-  return d;
-}
 
 // Stand-alone bias / batch norm / residual / activation over [R, C] (C % 8
 // == 0), y and its occupancy.  The activation and the presence of a residual
@@ -984,62 +960,78 @@ __global__ void __launch_bounds__(256) pad8_kernel(const __nv_bfloat16* __restri
   }
 }
 
-// Rows of kernel windows for a convolution with few input channels (the RGB
-// stems): x [N, H, W, C] -> xr [N, H + 2P, Wx, 32], Wx = W + 2P - kw + 1,
-// xr[n][h][w][s C + c] = x[n][h - P][w - P + s][c] for s < kw (zero outside
-// the image), channels kw C .. 31 zero.  A kh x kw convolution of x with
-// stride S and padding P is then a kh x 1 convolution of xr with stride S and
-// no padding over 32 channels (weights [Cout][kh][kw C], padded to 32), whose
-// operands the implicit GEMM loads with 4-D TMA boxes.  One CTA per output
-// row: the zero-padded input row is staged in shared memory, where a
-// window's kw C values are contiguous.
-__global__ void __launch_bounds__(256) im2row_kernel(const __nv_bfloat16* __restrict__ x, int N, int H, int W,
-                                                     int C, int kw, int P, __nv_bfloat16* __restrict__ xr) {
-  // the zero-padded row twice, as 32-bit words: s_even[i] = elements 2i, 2i + 1
-  // and s_odd[i] = elements 2i + 1, 2i + 2, so a window starting at element e
-  // is whole words of one of them (e even: s_even from e / 2, odd: s_odd)
-  extern __shared__ uint32_t s_w32[];
+// im2col for a convolution with few input channels (the RGB stems):
+// x [N, H, W, C] -> xc [N Ho Wo, Kp], row (n, oh, ow) = the kh x kw x C window
+// of output pixel (n, oh, ow) in [kh][kw][C] order (zero outside the image),
+// columns Kc = kh kw C .. Kp - 1 zero (Kp = Kc rounded up to 32).  The
+// convolution is then a plain GEMM of xc with the weights [C_out][Kc] padded to
+// Kp, whose A rows the implicit GEMM loads with 2-D TMA boxes of 128-byte rows.
+// One CTA per output row (n, oh): the kh zero-padded input rows it needs are
+// staged in shared memory (row r at r RLp + pre, `pre` placing the image part
+// of each row on a 16-byte boundary so that aligned rows are copied in 16-byte
+// pieces), where window element k of pixel ow sits at off[k] + ow S C.  Each
+// thread owns one 16-byte chunk position q of the output rows (its eight
+// offsets in registers) and writes that chunk for every (256 / Q)-th pixel.
+__global__ void __launch_bounds__(256) im2col_kernel(const __nv_bfloat16* __restrict__ x, int N, int H, int W,
+                                                     int C, int kh, int kw, int S, int P, int Ho, int Wo, int Kp,
+                                                     __nv_bfloat16* __restrict__ xc) {
+  extern __shared__ uint4 s_v4[];
+  const int RL = (W + 2 * P) * C;               // elements of one padded input row
+  const int pre = (8 - (P * C) % 8) % 8;        // leading slack: image part 16-byte aligned
+  const int RLp = (pre + RL + 7) / 8 * 8;       // row pitch (elements)
+  const int Kc = kh * kw * C, Q = Kp / 8;
+  uint16_t* s_rows = reinterpret_cast<uint16_t*>(s_v4);
+  const int ppc = (int)blockDim.x / Q;          // pixels per pass
+  const int q = (int)threadIdx.x % Q, p0 = (int)threadIdx.x / Q;
+  int off[8];
+#pragma unroll
+  for (int t = 0; t < 8; ++t) {
+    const int k = 8 * q + t;
+    off[t] = -1;
+    if (k < Kc) {
+      const int c = k % C, tap = k / C;
+      off[t] = (tap / kw) * RLp + pre + (tap % kw) * C + c;
+    }
+  }
   pdl_wait();
   pdl_trigger();
-  const int Hx = H + 2 * P, Wx = W + 2 * P - kw + 1, Wp = W + 2 * P;
-  const int KC = kw * C;
-  const int nel = Wp * C + 32;  // elements of the padded row (+ slack read past the last window)
-  const int nw = (nel + 1) / 2;
-  uint32_t* s_even = s_w32;
-  uint32_t* s_odd = s_w32 + nw;
   const uint16_t* xs = reinterpret_cast<const uint16_t*>(x);
-  const int KW32 = (KC + 1) / 2;  // words holding the window (the last may hold one element too many)
-  const uint32_t last_mask = (KC & 1) ? 0x0000FFFFu : 0xFFFFFFFFu;
-  for (int64_t row = blockIdx.x; row < (int64_t)N * Hx; row += gridDim.x) {
-    const int n = (int)(row / Hx), hp = (int)(row - (int64_t)n * Hx), h = hp - P;
-    const bool hin = h >= 0 && h < H;
-    const uint16_t* src = xs + ((int64_t)n * H + (hin ? h : 0)) * W * C;
-    auto elem = [&](int e) -> uint32_t {  // element e of the padded row
-      if (!hin || e >= Wp * C) return 0u;
-      const int wq = e / C - P;
-      return (wq >= 0 && wq < W) ? (uint32_t)src[wq * C + (e - (e / C) * C)] : 0u;
-    };
-    for (int i = threadIdx.x; i < nw; i += blockDim.x) {
-      const uint32_t e0 = elem(2 * i), e1 = elem(2 * i + 1), e2 = elem(2 * i + 2);
-      s_even[i] = e0 | (e1 << 16);
-      s_odd[i] = e1 | (e2 << 16);
+  const bool vec = (W * C) % 8 == 0 && (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
+  const int img0 = pre + P * C, img1 = img0 + W * C;  // image part of a staged row
+  for (int64_t row = blockIdx.x; row < (int64_t)N * Ho; row += gridDim.x) {
+    const int n = (int)(row / Ho), oh = (int)(row - (int64_t)n * Ho);
+    __syncthreads();  // the previous row's readers are done
+    for (int r = 0; r < kh; ++r) {
+      const int ih = oh * S - P + r;
+      uint16_t* dst = s_rows + r * RLp;
+      if (ih < 0 || ih >= H) {
+        for (int i = threadIdx.x; i < RLp / 8; i += blockDim.x) reinterpret_cast<uint4*>(dst)[i] = make_uint4(0, 0, 0, 0);
+        continue;
+      }
+      const uint16_t* src = xs + ((int64_t)n * H + ih) * W * C;
+      for (int i = threadIdx.x; i < img0; i += blockDim.x) dst[i] = 0;
+      for (int i = img1 + threadIdx.x; i < RLp; i += blockDim.x) dst[i] = 0;
+      if (vec) {
+        for (int i = threadIdx.x; i < W * C / 8; i += blockDim.x)
+          reinterpret_cast<uint4*>(dst + img0)[i] = reinterpret_cast<const uint4*>(src)[i];
+      } else {
+        for (int i = threadIdx.x; i < W * C; i += blockDim.x) dst[img0 + i] = src[i];
+      }
     }
     __syncthreads();
-    // consecutive threads write consecutive 16-byte quarters of the output row
-    uint4* dst = reinterpret_cast<uint4*>(xr + row * Wx * 32);
-    for (int j = threadIdx.x; j < Wx * 4; j += blockDim.x) {
-      const int e = (j >> 2) * C, k0 = (j & 3) * 4;
-      const uint32_t* srcw = ((e & 1) ? s_odd : s_even) + (e >> 1);
+    if (p0 >= ppc) continue;  // threads past the last whole pass of pixels
+    uint4* out = reinterpret_cast<uint4*>(xc + row * Wo * Kp) + q;
+    for (int ow = p0; ow < Wo; ow += ppc) {
+      const int base = ow * S * C;
       uint32_t o[4];
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const int kk = k0 + k;
-        o[k] = kk < KW32 ? srcw[kk] : 0u;
-        if (kk == KW32 - 1) o[k] &= last_mask;
+      for (int t = 0; t < 4; ++t) {
+        const uint32_t lo = off[2 * t] >= 0 ? s_rows[off[2 * t] + base] : 0u;
+        const uint32_t hi = off[2 * t + 1] >= 0 ? s_rows[off[2 * t + 1] + base] : 0u;
+        o[t] = lo | (hi << 16);
       }
-      dst[j] = make_uint4(o[0], o[1], o[2], o[3]);
+      out[(int64_t)ow * Q] = make_uint4(o[0], o[1], o[2], o[3]);
     }
-    __syncthreads();
   }
 }
 
@@ -1314,19 +1306,31 @@ cudaError_t launch_clear(const ClearArgs& a, cudaStream_t s) {
   return launch_kernel(clear_kernel, dim3((unsigned)(blocks < cap ? blocks : cap)), dim3(256), 0, s, a);
 }
 
-bool im2row_applies(int C, int kw, int groups) { return groups == 1 && C < 8 && kw > 1 && kw * C <= 32; }
+static size_t im2col_smem(int W, int C, int kh, int P) {
+  const int64_t pre = (8 - (P * C) % 8) % 8;
+  const int64_t RLp = (pre + (int64_t)(W + 2 * P) * C + 7) / 8 * 8;
+  return sizeof(uint16_t) * (size_t)(kh * RLp);
+}
 
-cudaError_t launch_im2row(const __nv_bfloat16* x, int N, int H, int W, int C, int kw, int P, __nv_bfloat16* xr,
-                          cudaStream_t s) {
-  const int64_t rows = (int64_t)N * (H + 2 * P);
-  if (rows <= 0 || W + 2 * P - kw + 1 <= 0) return cudaSuccess;
-  if ((reinterpret_cast<uintptr_t>(xr) & 15u) != 0) return cudaErrorInvalidValue;
-  const size_t nw = ((size_t)(W + 2 * P) * C + 32 + 1) / 2;
-  const size_t smem = 2 * sizeof(uint32_t) * nw;
-  if (smem > 48 * 1024) return cudaErrorInvalidValue;
-  const int64_t cap = 16LL * device_sm_count();
-  return launch_kernel(im2row_kernel, dim3((unsigned)(rows < cap ? rows : cap)), dim3(256), smem, s, x, N, H,
-                       W, C, kw, P, xr);
+int im2col_width(int C, int kh, int kw) { return (kh * kw * C + 31) / 32 * 32; }
+
+bool im2col_applies(int C, int kh, int kw, int groups, int W, int P) {
+  if (groups != 1 || C >= 8 || kh * kw <= 1) return false;
+  const int Kp = im2col_width(C, kh, kw);
+  return Kp <= 512 && im2col_smem(W, C, kh, P) <= 48 * 1024;
+}
+
+cudaError_t launch_im2col(const __nv_bfloat16* x, int N, int H, int W, int C, int kh, int kw, int S, int P,
+                          __nv_bfloat16* xc, cudaStream_t s) {
+  const int Ho = (H + 2 * P - kh) / S + 1, Wo = (W + 2 * P - kw) / S + 1;
+  const int64_t rows = (int64_t)N * Ho;
+  if (rows <= 0 || Wo <= 0) return cudaSuccess;
+  if (!im2col_applies(C, kh, kw, 1, W, P) || (reinterpret_cast<uintptr_t>(xc) & 15u) != 0)
+    return cudaErrorInvalidValue;
+  const int Kp = im2col_width(C, kh, kw);
+  const int64_t cap = 8LL * device_sm_count();
+  return launch_kernel(im2col_kernel, dim3((unsigned)(rows < cap ? rows : cap)), dim3(256),
+                       im2col_smem(W, C, kh, P), s, x, N, H, W, C, kh, kw, S, P, Ho, Wo, Kp, xc);
 }
 
 cudaError_t launch_pad_channels(const __nv_bfloat16* x, int64_t P, int C, int Cp,

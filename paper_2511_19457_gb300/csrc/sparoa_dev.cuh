@@ -525,6 +525,49 @@ __device__ __forceinline__ float gelu_f(float v) {
   return 0.5f * v * (1.f + t);
 }
 
+// Packed fp32 pairs for the fma.rn.f32x2 instruction (two independent
+// fp32 FMAs, each rounded to nearest like fmaf).
+typedef unsigned long long f2_t;  // two fp32 values (low: even channel)
+
+__device__ __forceinline__ f2_t f2(float lo, float hi) {
+  f2_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_split(f2_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ f2_t ffma2(f2_t a, f2_t b, f2_t c) {
+  f2_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+// bit 0 / bit 16 set where the low / high bf16 of w is non-zero (any bit but
+// the sign): adding 0x7FFF to a 15-bit magnitude carries into bit 15 exactly
+// when the magnitude is not zero, and never out of its 16-bit half
+__device__ __forceinline__ uint32_t nz_pairs(uint32_t w) {
+  return (((w & 0x7FFF7FFFu) + 0x7FFF7FFFu) >> 15) & 0x00010001u;
+}
+
+// Two fp32 values through the activation to a bf16 pair (round to nearest
+// even), `lo` in the low half; ReLU is applied by the conversion itself.
+template <int ACT>
+__device__ __forceinline__ uint32_t act_pack2(float lo, float hi) {
+  if (ACT == 2) {
+    lo = fminf(fmaxf(lo, 0.f), 6.f);
+    hi = fminf(fmaxf(hi, 0.f), 6.f);
+  } else if (ACT == 3) {
+    lo = gelu_f(lo);
+    hi = gelu_f(hi);
+  }
+  uint32_t d;
+  if (ACT == 1)
+    asm("cvt.rn.relu.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  else
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  return d;
+}
+
 __device__ __forceinline__ float epi_act(float v, int act) {
   if (act == 1) return v > 0.f ? v : 0.f;
   if (act == 2) return v > 0.f ? (v < 6.f ? v : 6.f) : 0.f;

@@ -172,13 +172,16 @@ bool stats_writes_rows_whole(int64_t R, int C);
 cudaError_t launch_stats(const __nv_bfloat16* x, int64_t R, int C, const OccDev& o, cudaStream_t s,
                          bool early = false, const ClearArgs* zero = nullptr);
 
+// im2col for a convolution with few input channels (k_tiles.cu): x [N, H, W,
+// C] -> xc [N Ho Wo, Kp], each row the [kh][kw][C] window of one output pixel,
+// zero-padded to Kp = im2col_width(C, kh, kw) (see im2col_kernel); for groups
+// == 1, C < 8, kh kw > 1 and small enough windows (im2col_applies).
+int im2col_width(int C, int kh, int kw);
+bool im2col_applies(int C, int kh, int kw, int groups, int W, int P);
+cudaError_t launch_im2col(const __nv_bfloat16* x, int N, int H, int W, int C, int kh, int kw, int S, int P,
+                          __nv_bfloat16* xc, cudaStream_t s);
+
 // Copy [P, C] to [P, Cp] with zero channels C..Cp-1.
-// Window rows for a convolution with few input channels (k_tiles.cu):
-// x [N, H, W, C] -> xr [N, H + 2P, W + 2P - kw + 1, 32] (see im2row_kernel),
-// for groups == 1, C < 8, kw > 1 and kw C <= 32 (im2row_applies).
-bool im2row_applies(int C, int kw, int groups);
-cudaError_t launch_im2row(const __nv_bfloat16* x, int N, int H, int W, int C, int kw, int P, __nv_bfloat16* xr,
-                          cudaStream_t s);
 cudaError_t launch_pad_channels(const __nv_bfloat16* x, int64_t P, int C, int Cp,
                                 __nv_bfloat16* y, cudaStream_t s);
 
