@@ -1222,6 +1222,20 @@ def run_profile(args, rank, local_rank, world, peaks):
         y = torch.empty(32, 56, 56, 64, dtype=torch.bfloat16, device=dev)
         yo = sp.OccupancyBuffer(32 * 56 * 56, 64)
         call = lambda: sp.sparoa_bn_act(ctx, x, y, bn=bnp, act=sp.ACT_RELU, y_occ=yo)
+    elif op == "conv1x1_expand":  # MobileNetV2's first expansion at batch 32, BN + ReLU6
+        x = act(32, 112, 112, 16)
+        w = (torch.randn(96, 1, 1, 16, device=dev, generator=gen) / 4).to(torch.bfloat16)
+        bnp = torch.tensor(synth.identity_bn(96), device=dev)
+        y = torch.empty(32, 112, 112, 96, dtype=torch.bfloat16, device=dev)
+        yo = sp.OccupancyBuffer(32 * 112 * 112, 96)
+        call = lambda: sp.sparoa_conv2d(ctx, x, w, y, bn=bnp, act=sp.ACT_RELU6, y_occ=yo)
+    elif op == "stem7x7":  # ResNet-18's stem at batch 32: im2col rows, then a GEMM; BN + ReLU
+        x = act(32, 224, 224, 3, zero_p=0.0)
+        w = (torch.randn(64, 7, 7, 3, device=dev, generator=gen) / 12).to(torch.bfloat16)
+        bnp = torch.tensor(synth.identity_bn(64), device=dev)
+        y = torch.empty(32, 112, 112, 64, dtype=torch.bfloat16, device=dev)
+        yo = sp.OccupancyBuffer(32 * 112 * 112, 64)
+        call = lambda: sp.sparoa_conv2d(ctx, x, w, y, stride=2, pad=3, bn=bnp, act=sp.ACT_RELU, y_occ=yo)
     elif op == "stats_large":
         x = act(401408, 64)
         oc = sp.OccupancyBuffer(401408, 64)

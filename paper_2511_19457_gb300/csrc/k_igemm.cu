@@ -38,7 +38,7 @@
 //
 // Each tile shape is compiled three times: the general kernel, and lean ones
 // for modes 0 and 2 without a K split or fp32 output, without a residual and
-// with one (N % 32 == 0).  With small K the
+// with one (N % 8 == 0).  With small K the
 // epilogue is the whole cost of a tile and runs at a fraction of an
 // instruction per cycle (few warps, long dependency chains); the lean kernel's
 // smaller, branch-free epilogue issues fewer instructions per tile and misses
@@ -183,18 +183,19 @@ __device__ __forceinline__ int64_t tile_row(const Geo& p, const TileGeo& g, int 
 
 // One row's 32 accumulator values (fp32 bits) through the column affine
 // (scale and shift from shared memory; none when sc is null), the residual
-// (32 bf16 at rp, none when rp is null) and the activation, packed to 16 bf16
+// (bf16 at rp, none when rp is null; only the first rvalid of the 32 columns
+// are read, rvalid a multiple of 8) and the activation, packed to 16 bf16
 // pairs: fp32x2 FMAs, ReLU folded into the conversion.  The same operations
 // in the same order as the general epilogue (fmaf, then + residual, then the
 // activation, then round to bf16).
 template <int ACT, bool RES>
 __device__ __forceinline__ void affine_act_pack32(const uint32_t (&raw)[32], const float* sc, const float* sh,
-                                                  const uint4* rp, uint32_t (&pk)[16]) {
+                                                  const uint4* rp, int rvalid, uint32_t (&pk)[16]) {
   uint4 rv = make_uint4(0u, 0u, 0u, 0u);  // residual values 8 (i / 2) .. + 7
   if (!RES) rp = nullptr;
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
-    if (RES && rp && (i & 1) == 0) rv = rp[i >> 1];
+    if (RES && rp && (i & 1) == 0) rv = 8 * (i >> 1) < rvalid ? rp[i >> 1] : make_uint4(0u, 0u, 0u, 0u);
     if (sc == nullptr && rp == nullptr) {  // the accumulators as they are
       pk[2 * i] = act_pack2<ACT>(__uint_as_float(raw[4 * i]), __uint_as_float(raw[4 * i + 1]));
       pk[2 * i + 1] = act_pack2<ACT>(__uint_as_float(raw[4 * i + 2]), __uint_as_float(raw[4 * i + 3]));
@@ -290,7 +291,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                  const __grid_constant__ CUtensorMap tmB32, const IgemmArgs P) {
   using C = Cfg<BN, BK>;
   const Geo p = make_geo(P);
-  // lean kernels (LEAN 1: no residual, 2: a residual and N % 32 == 0): TMA
+  // lean kernels (LEAN 1: no residual, 2: a residual and N % 8 == 0): TMA
   // producers only (mode 0 or 2), no K split, bf16 output (the host launches
   // them only then)
   if (LEAN) __builtin_assume(p.conv != 1);
@@ -816,6 +817,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool mvalid;
       int img, oh, ow;
       const int64_t m = tile_row(p, g, r, mvalid, img, oh, ow);
+      if (LEAN == 2 && mvalid) {
+        // this row's residual segments into L1 while the accumulator is pending
+        const __nv_bfloat16* rrow = residual + m * p.N + g.n0 + hf * 32;
+        for (int gc = 0; gc < BN / 64; ++gc)
+          if (g.n0 + gc * 64 + hf * 32 < p.N) prefetch_l1(rrow + gc * 64);
+      }
       float* const scb = s_scale + (fixed_cols ? 0 : b * BN);
       float* const shb = s_shift + (fixed_cols ? 0 : b * BN);
       if (!fixed_cols) {
@@ -845,12 +852,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float* shg = shb + gcol * 64 + hf * 32;
         const uint4* rp =
             residual && mvalid ? reinterpret_cast<const uint4*>(residual + m * p.N + ncol0) : nullptr;
+        const int rvalid = p.N - ncol0 < 32 ? p.N - ncol0 : 32;
         uint32_t pk[16];
         constexpr bool kRes = LEAN == 2;
-        if (act == 1) affine_act_pack32<1, kRes>(raw, scg, shg, rp, pk);
-        else if (act == 2) affine_act_pack32<2, kRes>(raw, scg, shg, rp, pk);
-        else if (act == 0) affine_act_pack32<0, kRes>(raw, scg, shg, rp, pk);
-        else affine_act_pack32<3, kRes>(raw, scg, shg, rp, pk);
+        if (act == 1) affine_act_pack32<1, kRes>(raw, scg, shg, rp, rvalid, pk);
+        else if (act == 2) affine_act_pack32<2, kRes>(raw, scg, shg, rp, rvalid, pk);
+        else if (act == 0) affine_act_pack32<0, kRes>(raw, scg, shg, rp, rvalid, pk);
+        else affine_act_pack32<3, kRes>(raw, scg, shg, rp, rvalid, pk);
         const uint32_t row_addr = stg + (uint32_t)lane * 64u;
         const int sx = (lane >> 1) & 3;
 #pragma unroll
@@ -1514,7 +1522,7 @@ cudaError_t launch_igemm(const IgemmArgs& a_in, cudaStream_t s) {
   const int64_t tiles = mtiles * ((a.N + bn - 1) / bn);
   const bool lean = a.conv != 1 && ks == 1 && !a.y_f32 && !a.dense_only &&
                     (a.ep.residual == nullptr ||
-                     (a.N % 32 == 0 && (reinterpret_cast<uintptr_t>(a.ep.residual) & 15u) == 0));
+                     (a.N % 8 == 0 && (reinterpret_cast<uintptr_t>(a.ep.residual) & 15u) == 0));
   if (!lean) return launch_bn<0>(a, bn, bk, tA, tB, tY, tA32, tB32, tiles, s);
   return a.ep.residual ? launch_bn<2>(a, bn, bk, tA, tB, tY, tA32, tB32, tiles, s)
                        : launch_bn<1>(a, bn, bk, tA, tB, tY, tA32, tB32, tiles, s);

@@ -277,6 +277,10 @@ __device__ __forceinline__ void pdl_trigger() {
 
 // Make generic-proxy writes to shared memory visible to the async proxy
 // (tensor cores / TMA).
+// Pull the 128-byte line holding p into L1 (no register result; a hint).
+__device__ __forceinline__ void prefetch_l1(const void* p) {
+  asm volatile("prefetch.global.L1 [%0];" ::"l"(p));
+}
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -551,20 +555,20 @@ __device__ __forceinline__ uint32_t nz_pairs(uint32_t w) {
 
 // Two fp32 values through the activation to a bf16 pair (round to nearest
 // even), `lo` in the low half; ReLU is applied by the conversion itself.
+// ReLU6 clamps after the rounding: min(round(relu(v)), 6) = round(min(relu(v),
+// 6)) because rounding is monotonic and 6 is a bf16 value.
 template <int ACT>
 __device__ __forceinline__ uint32_t act_pack2(float lo, float hi) {
-  if (ACT == 2) {
-    lo = fminf(fmaxf(lo, 0.f), 6.f);
-    hi = fminf(fmaxf(hi, 0.f), 6.f);
-  } else if (ACT == 3) {
+  if (ACT == 3) {
     lo = gelu_f(lo);
     hi = gelu_f(hi);
   }
   uint32_t d;
-  if (ACT == 1)
+  if (ACT == 1 || ACT == 2)
     asm("cvt.rn.relu.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
   else
     asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  if (ACT == 2) asm("min.bf16x2 %0, %0, %1;" : "+r"(d) : "r"(0x40C040C0u));  // 6.0 in both halves
   return d;
 }
 

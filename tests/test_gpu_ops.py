@@ -219,6 +219,7 @@ CONV_CASES = [
     # N, H, W, Cin, Cout, k, stride, pad, act, residual
     (2, 15, 17, 64, 128, 3, 2, 1, 1, False),
     (2, 14, 14, 96, 24, 1, 1, 0, 0, True),     # pointwise (TMA GEMM mode), linear + residual
+    (2, 9, 10, 64, 40, 1, 1, 0, 2, True),      # residual over a block of 8 of 32 columns
     (2, 14, 14, 64, 128, 1, 2, 0, 0, False),   # strided 1x1 downsample
     (1, 32, 30, 3, 64, 7, 2, 3, 1, False),     # stem, C_in padded to 8
     (3, 21, 19, 3, 32, 3, 2, 1, 2, False),     # 3x3 stem; 1197 pixels: a partial 8-pixel group
