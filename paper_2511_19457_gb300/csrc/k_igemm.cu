@@ -484,8 +484,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
           named_bar_sync(1, 128);
-          // no per-tap masks (too many taps, wide rows, or an input without row
-          // bitmaps such as the window rows of a narrow stem): keep every block
+          // no per-tap masks (too many taps, wide rows, or an input given without
+          // row bitmaps): keep every block
           const bool many = p.kh * p.kw > kMaxTaps || in_W64 > 1 || in_rowbm == nullptr;
           for (int w0 = 0; w0 < kblocks && w0 < kMaxKWords * 32; w0 += 128) {
             const int kb = w0 + r;
